@@ -1,0 +1,139 @@
+/*
+ * curvefp.h — C ABI of the CurveFP GB300 library (libcurvefp.so).
+ *
+ * CurveFP ("CurveFP: Co-Designing Numerical Representation and Product
+ * Arithmetic for Language Models") stores each element of a block of G values
+ * as a sign, an exponent and a curve index under one power-of-two block scale
+ * (Sec. 3.1, Eq. 1), multiplies codes exactly by adding curve indices with a
+ * carry into the exponent (Sec. 3.2, Eq. 2), accumulates products per phase
+ * of the radix's phase schedule (Eq. 4, Eq. 5, App. A.1) and combines the
+ * phases with fixed constants 2^{h/H}.  Binary radix (r = 2) only.
+ *
+ * Conventions for every entry point
+ *   - All tensor pointers are DEVICE pointers to caller-owned memory.  The
+ *     library allocates no device memory, never synchronizes, and enqueues its
+ *     kernels on `stream` (a cudaStream_t; NULL = the legacy default stream).
+ *   - Host-checkable errors (NULL pointers, unknown enums, bad sizes or
+ *     alignment) are returned synchronously and nothing is enqueued.
+ *     CURVEFP_ERR_CUDA means a launch failed.
+ *   - Data-dependent conditions are OR-ed into `device_status` (a device
+ *     uint32_t the caller zeroes; may be NULL): CURVEFP_DEV_NAN,
+ *     CURVEFP_DEV_RANGE, CURVEFP_DEV_TIMEOUT.  Read it after the stream has
+ *     synchronized.
+ *   - Row-major layouts; sizes in elements.
+ *
+ * Code byte (App. C.1 packing; reading of Sec. 3.1):
+ *   code = (s << 7) | m,  m = n + B,  n = e*K + k,  B = 2^{E+C-1},
+ *   K = 2^C, e in [-2^{E-1}, 2^{E-1}-1], k in [0, K-1], n in [-(B-1), B-1].
+ *   m = 0 is the zero sentinel (the smallest combination e = -2^{E-1}, k = 0
+ *   is omitted); zero is written as 0x00.  Decoders read m = code & 0x7F
+ *   (E4C3, E5C2) or code & 0x3F (E3C3, whose bit 6 is always 0 in a byte
+ *   container).  Value: x = (-1)^s 2^{a_b} 2^{n/K}.
+ * Block scale a_b (int8, "ceil-absmax", Sec. 3.1 and App. A.2): the smallest
+ *   integer in [-128, 127] with max|x| <= 2^{a_b} 2^{(B-1)/K} over the block
+ *   (NaN excluded); 0 for an all-zero block; 127 if no integer qualifies (Inf).
+ */
+#ifndef CURVEFP_H
+#define CURVEFP_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Table 1: E3C3 (CurveFP7, 7 bits, 63 positive levels, H = 8), E4C3 and E5C2
+ * (CurveFP8, 8 bits, 127 positive levels, H = 8 and 4). */
+typedef enum { CURVEFP_E3C3 = 0, CURVEFP_E4C3 = 1, CURVEFP_E5C2 = 2 } curvefp_format_t;
+
+typedef enum { CURVEFP_F32 = 0, CURVEFP_BF16 = 1 } curvefp_dtype_t;
+
+typedef enum {
+  CURVEFP_OK = 0,
+  CURVEFP_ERR_INVALID_ARG = 1,
+  CURVEFP_ERR_UNSUPPORTED = 2,
+  CURVEFP_ERR_CUDA = 3
+} curvefp_status_t;
+
+/* GEMM kernels.  EXACT: integer-ALU kernel whose per-phase sums are exact
+ * integers (bit-identical to the definition).  TENSOR: tcgen05 tensor-core
+ * kernel over power-of-two phase planes with FP32 per-phase accumulation. */
+typedef enum { CURVEFP_GEMM_EXACT = 0, CURVEFP_GEMM_TENSOR = 1 } curvefp_gemm_algo_t;
+
+/* Bits of the device status word. */
+#define CURVEFP_DEV_NAN 1u     /* quantize: a NaN input was encoded as 0x00        */
+#define CURVEFP_DEV_RANGE 2u   /* gemm: an output's scale spread exceeds the exact
+                                  int128 window (see curvefp_gemm_phases)          */
+#define CURVEFP_DEV_TIMEOUT 4u /* gemm: a pipeline wait gave up (internal error)   */
+
+/* Block-scaled quantization Q(X) (Sec. 3.1; ceil-absmax scale, nearest level in
+ * absolute error over {0} U {2^{n/K}}, saturation at 2^{(B-1)/K}).
+ *   x        : [rows x cols] FP32 or BF16 with leading dimension ld >= cols
+ *              (elements); 16-byte aligned, ld * element size a multiple of 16.
+ *   block    : G in {32, 64, 128, 256, 512}.
+ *   block_axis 0: blocks of G consecutive elements of a row (cols % G == 0);
+ *              codes [rows x cols] dense, scales [rows x cols/G].
+ *   block_axis 1: blocks of G consecutive rows of a column (rows % G == 0);
+ *              the output is the transposed operand, blocked axis contiguous:
+ *              codes [cols x rows] dense, scales [cols x rows/G].
+ *   codes    : 16-byte aligned.
+ * NaN inputs encode as 0x00 and raise CURVEFP_DEV_NAN. */
+curvefp_status_t curvefp_quantize(curvefp_format_t fmt, int block, const void* x, curvefp_dtype_t dtype,
+                                  int64_t rows, int64_t cols, int64_t ld, int block_axis, uint8_t* codes,
+                                  int8_t* scales, uint32_t* device_status, void* stream);
+
+/* Dequantization to FP32 (Eq. 1): out = RN32( RN32(2^{k/K}) * 2^{a_b + e} ) with
+ * the sign applied; zero codes give +0.0.
+ *   codes [rows x cols] (16-byte aligned, cols % block == 0), scales
+ *   [rows x cols/block], out [rows x cols] FP32 (16-byte aligned). */
+curvefp_status_t curvefp_dequantize(curvefp_format_t fmt, int block, const uint8_t* codes, const int8_t* scales,
+                                    int64_t rows, int64_t cols, float* out, void* stream);
+
+/* Closed-product GEMM C = A_hat * B_hat^T (Sec. 3.2, Eq. 2, Eq. 5, App. A.1;
+ * the forward/backward operators of Sec. 3.3 and App. A.2 are all of this form
+ * once each operand is quantized along its own reduction axis).
+ *   a  : [M x K] codes of format fmt_a, K contiguous; sa: [M x K/block].
+ *   b  : [N x K] codes of format fmt_b, K contiguous; sb: [N x K/block].
+ *   c  : [M x N] FP32 output, row-major.
+ * Every nonzero product a (x) b has sign s_a xor s_b, scale a_a + a_b and
+ * lattice exponent u = n_a L/K_a + n_b L/K_b with L = max(K_a, K_b); it lands on
+ * phase h = u mod L with weight 2^{floor(u/L)}.  Per-phase sums S_h are combined
+ * as C = sum_h 2^{h/L} S_h in the epilogue.
+ * Requirements: K % block == 0; a, b 16-byte aligned.
+ * EXACT: S_h exact, combine in FP64, one FP32 rounding; outputs whose scale
+ *   spread leaves the int128 window raise CURVEFP_DEV_RANGE (values undefined).
+ * TENSOR: S_h accumulated in FP32 on the tensor cores, combine in FP32. */
+curvefp_status_t curvefp_gemm(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, curvefp_format_t fmt_b, int block,
+                              const uint8_t* a, const int8_t* sa, const uint8_t* b, const int8_t* sb, int64_t M,
+                              int64_t N, int64_t K, float* c, uint32_t* device_status, void* stream);
+
+/* Validation form of the EXACT GEMM that also exports the per-phase integer
+ * accumulators (Eq. 5 "signed integer counts" summed per phase; App. A.1).
+ *   phase_sums : M*N*H two's-complement int128 values stored as (lo, hi) int64
+ *                pairs, [M][N][H]; S_h at LSB 2^{lsb}.
+ *   phase_lsb  : [M x N] int32, lsb = min_b(sa[i,b] + sb[j,b]) + t_min with
+ *                t_min = floor(-((B_a-1) L/K_a + (B_b-1) L/K_b) / L).
+ *   An output is out of range (CURVEFP_DEV_RANGE, its sums undefined) when
+ *   bitlen(K) + spread + (t_max - t_min) > 127, spread = max_b - min_b of
+ *   sa[i,b] + sb[j,b].
+ *   c may be NULL. */
+curvefp_status_t curvefp_gemm_phases(curvefp_format_t fmt_a, curvefp_format_t fmt_b, int block, const uint8_t* a,
+                                     const int8_t* sa, const uint8_t* b, const int8_t* sb, int64_t M, int64_t N,
+                                     int64_t K, float* c, int64_t* phase_sums, int32_t* phase_lsb,
+                                     uint32_t* device_status, void* stream);
+
+/* Number of phases H of a format pair (Eq. 4 with binary radix, on the shared
+ * lattice L = max(K_a, K_b)); -1 for an unknown format. */
+int curvefp_phase_count(curvefp_format_t fmt_a, curvefp_format_t fmt_b);
+
+/* Static description of a status code. */
+const char* curvefp_status_string(curvefp_status_t status);
+
+/* Library version string. */
+const char* curvefp_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CURVEFP_H */

@@ -1,0 +1,133 @@
+"""CurveFP on GB300: Python binding of the C ABI in ``include/curvefp.h``.
+
+This module only marshals arguments (torch tensors -> device pointers, the
+current CUDA stream) into ``libcurvefp.so``; every step of the quantizer and
+the GEMM runs in the library's CUDA kernels.  There is no CPU fallback: if the
+library is missing or was not built for this machine, the calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+from . import _build
+
+FORMATS = {"E3C3": 0, "E4C3": 1, "E5C2": 2}
+DTYPES = {"f32": 0, "bf16": 1}
+ALGOS = {"exact": 0, "tensor": 1}
+STATUS_BITS = {"nan": 1, "range": 2, "timeout": 4}
+
+_lib = None
+
+
+class CurveFPError(RuntimeError):
+    pass
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_missing: bool = False):
+    """Load libcurvefp.so (raises if it is absent, unless asked to build)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(_build.LIB):
+            if not build_if_missing:
+                raise CurveFPError(f"libcurvefp.so not built ({_build.LIB}); run __graft_entry__.build()")
+            _build.build()
+        lib = ctypes.CDLL(_build.LIB)
+        P, I, L = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64
+        lib.curvefp_quantize.argtypes = [I, I, P, I, L, L, L, I, P, P, P, P]
+        lib.curvefp_dequantize.argtypes = [I, I, P, P, L, L, P, P]
+        lib.curvefp_gemm.argtypes = [I, I, I, I, P, P, P, P, L, L, L, P, P, P]
+        lib.curvefp_gemm_phases.argtypes = [I, I, I, P, P, P, P, L, L, L, P, P, P, P, P]
+        lib.curvefp_phase_count.argtypes = [I, I]
+        lib.curvefp_status_string.argtypes = [I]
+        lib.curvefp_status_string.restype = ctypes.c_char_p
+        lib.curvefp_version.restype = ctypes.c_char_p
+        for f in ("curvefp_quantize", "curvefp_dequantize", "curvefp_gemm", "curvefp_gemm_phases"):
+            getattr(lib, f).restype = I
+        _lib = lib
+    return _lib
+
+
+def _fmt(f) -> int:
+    return FORMATS[f] if isinstance(f, str) else int(f)
+
+
+def _check(rc: int):
+    if rc != 0:
+        raise CurveFPError(load().curvefp_status_string(rc).decode())
+
+
+def _stream(stream):
+    import torch
+
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _p(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def phase_count(fmt_a, fmt_b) -> int:
+    return load().curvefp_phase_count(_fmt(fmt_a), _fmt(fmt_b))
+
+
+def quantize(x, fmt, block: int = 32, block_axis: int = 0, codes=None, scales=None, status=None, stream=None):
+    """Q(X) of a 2-D FP32/BF16 CUDA tensor.  Returns (codes, scales): codes
+    [rows x cols] (block_axis 0) or the transposed [cols x rows] (block_axis 1)."""
+    import torch
+
+    assert x.dim() == 2 and x.is_cuda and x.stride(1) == 1
+    rows, cols = x.shape
+    R, Cc = (cols, rows) if block_axis else (rows, cols)
+    if codes is None:
+        codes = torch.empty((R, Cc), dtype=torch.uint8, device=x.device)
+    if scales is None:
+        scales = torch.empty((R, Cc // block), dtype=torch.int8, device=x.device)
+    dt = {torch.float32: 0, torch.bfloat16: 1}[x.dtype]
+    _check(load().curvefp_quantize(_fmt(fmt), block, _p(x), dt, rows, cols, x.stride(0), block_axis,
+                                   _p(codes), _p(scales), _p(status), _stream(stream)))
+    return codes, scales
+
+
+def dequantize(codes, scales, fmt, block: int = 32, out=None, stream=None):
+    import torch
+
+    if out is None:
+        out = torch.empty(codes.shape, dtype=torch.float32, device=codes.device)
+    _check(load().curvefp_dequantize(_fmt(fmt), block, _p(codes), _p(scales), codes.shape[0], codes.shape[1],
+                                     _p(out), _stream(stream)))
+    return out
+
+
+def gemm(a, sa, b, sb, fmt_a, fmt_b, block: int = 32, algo: str = "tensor", out=None, status=None, stream=None):
+    """C = A_hat B_hat^T for a [M x K] and b [N x K] codes (K contiguous)."""
+    import torch
+
+    M, K = a.shape
+    N = b.shape[0]
+    if out is None:
+        out = torch.empty((M, N), dtype=torch.float32, device=a.device)
+    _check(load().curvefp_gemm(ALGOS[algo], _fmt(fmt_a), _fmt(fmt_b), block, _p(a), _p(sa), _p(b), _p(sb),
+                               M, N, K, _p(out), _p(status), _stream(stream)))
+    return out
+
+
+def gemm_phases(a, sa, b, sb, fmt_a, fmt_b, block: int = 32, status=None, stream=None):
+    """Exact GEMM that also returns the per-phase int128 sums as (lo, hi)
+    int64 pairs [M x N x H x 2] and their LSB exponents [M x N]."""
+    import torch
+
+    M, K = a.shape
+    N = b.shape[0]
+    H = phase_count(fmt_a, fmt_b)
+    c = torch.empty((M, N), dtype=torch.float32, device=a.device)
+    ps = torch.empty((M, N, H, 2), dtype=torch.int64, device=a.device)
+    pl = torch.empty((M, N), dtype=torch.int32, device=a.device)
+    _check(load().curvefp_gemm_phases(_fmt(fmt_a), _fmt(fmt_b), block, _p(a), _p(sa), _p(b), _p(sb), M, N, K,
+                                      _p(c), _p(ps), _p(pl), _p(status), _stream(stream)))
+    return c, ps, pl

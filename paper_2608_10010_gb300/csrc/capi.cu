@@ -1,0 +1,114 @@
+// C ABI of libcurvefp: argument validation, then one asynchronous launch on
+// the caller's stream.  Declarations and the full contract are in
+// include/curvefp.h.  No device memory is allocated here and nothing
+// synchronizes.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/curvefp.h"
+#include "kernels.cuh"
+
+namespace {
+
+bool fmt_ok(int f) { return f == CURVEFP_E3C3 || f == CURVEFP_E4C3 || f == CURVEFP_E5C2; }
+bool block_ok(int g) { return g == 32 || g == 64 || g == 128 || g == 256 || g == 512; }
+bool al16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+int fmt_k(int f) { return f == CURVEFP_E5C2 ? 4 : 8; }
+
+int sm_count() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) return 148;
+  return n;
+}
+
+curvefp_status_t from_cuda(cudaError_t e) { return e == cudaSuccess ? CURVEFP_OK : CURVEFP_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+curvefp_status_t curvefp_quantize(curvefp_format_t fmt, int block, const void* x, curvefp_dtype_t dtype,
+                                  int64_t rows, int64_t cols, int64_t ld, int block_axis, uint8_t* codes,
+                                  int8_t* scales, uint32_t* device_status, void* stream) {
+  if (!fmt_ok(fmt) || !block_ok(block) || (dtype != CURVEFP_F32 && dtype != CURVEFP_BF16)) return CURVEFP_ERR_INVALID_ARG;
+  if (block_axis != 0 && block_axis != 1) return CURVEFP_ERR_INVALID_ARG;
+  if (rows < 0 || cols < 0 || ld < cols) return CURVEFP_ERR_INVALID_ARG;
+  if (rows == 0 || cols == 0) return CURVEFP_OK;
+  if (!x || !codes || !scales) return CURVEFP_ERR_INVALID_ARG;
+  const int64_t esz = dtype == CURVEFP_F32 ? 4 : 2;
+  if (!al16(x) || !al16(codes) || (ld * esz) % 16 != 0) return CURVEFP_ERR_INVALID_ARG;
+  if (block_axis == 0 && cols % block != 0) return CURVEFP_ERR_INVALID_ARG;
+  if (block_axis == 1 && rows % block != 0) return CURVEFP_ERR_INVALID_ARG;
+  if (block_axis == 1 && rows / block > 65535) return CURVEFP_ERR_UNSUPPORTED;
+  if (rows * cols / block > (int64_t)1 << 40) return CURVEFP_ERR_UNSUPPORTED;
+  return from_cuda(cfp::launch_quantize(fmt, block, x, dtype, rows, cols, ld, block_axis, codes, scales,
+                                        device_status, static_cast<cudaStream_t>(stream), sm_count()));
+}
+
+curvefp_status_t curvefp_dequantize(curvefp_format_t fmt, int block, const uint8_t* codes, const int8_t* scales,
+                                    int64_t rows, int64_t cols, float* out, void* stream) {
+  if (!fmt_ok(fmt) || !block_ok(block) || rows < 0 || cols < 0) return CURVEFP_ERR_INVALID_ARG;
+  if (rows == 0 || cols == 0) return CURVEFP_OK;
+  if (!codes || !scales || !out || cols % block != 0 || !al16(codes) || !al16(out)) return CURVEFP_ERR_INVALID_ARG;
+  return from_cuda(cfp::launch_dequantize(fmt, block, codes, scales, rows * cols, out,
+                                          static_cast<cudaStream_t>(stream), sm_count()));
+}
+
+static curvefp_status_t gemm_args(int fa, int fb, int block, const uint8_t* a, const int8_t* sa, const uint8_t* b,
+                                  const int8_t* sb, int64_t M, int64_t N, int64_t K) {
+  if (!fmt_ok(fa) || !fmt_ok(fb) || !block_ok(block)) return CURVEFP_ERR_INVALID_ARG;
+  if (M <= 0 || N <= 0 || K <= 0 || K % block != 0) return CURVEFP_ERR_INVALID_ARG;
+  if (!a || !sa || !b || !sb || !al16(a) || !al16(b)) return CURVEFP_ERR_INVALID_ARG;
+  if (M > INT32_MAX || N > INT32_MAX || K > INT32_MAX) return CURVEFP_ERR_UNSUPPORTED;
+  return CURVEFP_OK;
+}
+
+curvefp_status_t curvefp_gemm(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, curvefp_format_t fmt_b, int block,
+                              const uint8_t* a, const int8_t* sa, const uint8_t* b, const int8_t* sb, int64_t M,
+                              int64_t N, int64_t K, float* c, uint32_t* device_status, void* stream) {
+  curvefp_status_t r = gemm_args(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K);
+  if (r != CURVEFP_OK) return r;
+  if (!c) return CURVEFP_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (algo == CURVEFP_GEMM_EXACT)
+    return from_cuda(cfp::launch_gemm_exact(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, nullptr, nullptr,
+                                            device_status, st));
+  if (algo == CURVEFP_GEMM_TENSOR) {
+    if (!cfp::gemm_tensor_supported(fmt_a, fmt_b)) return CURVEFP_ERR_UNSUPPORTED;
+    return from_cuda(cfp::launch_gemm_tensor(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, device_status, st,
+                                             sm_count()));
+  }
+  return CURVEFP_ERR_INVALID_ARG;
+}
+
+curvefp_status_t curvefp_gemm_phases(curvefp_format_t fmt_a, curvefp_format_t fmt_b, int block, const uint8_t* a,
+                                     const int8_t* sa, const uint8_t* b, const int8_t* sb, int64_t M, int64_t N,
+                                     int64_t K, float* c, int64_t* phase_sums, int32_t* phase_lsb,
+                                     uint32_t* device_status, void* stream) {
+  curvefp_status_t r = gemm_args(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K);
+  if (r != CURVEFP_OK) return r;
+  if (!phase_sums || !phase_lsb) return CURVEFP_ERR_INVALID_ARG;
+  return from_cuda(cfp::launch_gemm_exact(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, phase_sums, phase_lsb,
+                                          device_status, static_cast<cudaStream_t>(stream)));
+}
+
+int curvefp_phase_count(curvefp_format_t fmt_a, curvefp_format_t fmt_b) {
+  if (!fmt_ok(fmt_a) || !fmt_ok(fmt_b)) return -1;
+  const int ka = fmt_k(fmt_a), kb = fmt_k(fmt_b);
+  return ka > kb ? ka : kb;
+}
+
+const char* curvefp_status_string(curvefp_status_t s) {
+  switch (s) {
+    case CURVEFP_OK: return "ok";
+    case CURVEFP_ERR_INVALID_ARG: return "invalid argument";
+    case CURVEFP_ERR_UNSUPPORTED: return "unsupported configuration";
+    case CURVEFP_ERR_CUDA: return "CUDA launch error";
+  }
+  return "unknown status";
+}
+
+const char* curvefp_version(void) { return "curvefp-gb300 0.1 (sm_103a)"; }
+
+}  // extern "C"

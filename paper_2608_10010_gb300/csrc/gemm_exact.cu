@@ -1,0 +1,176 @@
+// Exact closed-product GEMM on the integer ALUs (Sec. 3.2, Eq. 2, Eq. 5,
+// App. A.1): the per-phase Kulisch layout of the paper, realized per output.
+//
+// For every nonzero product of codes a and b the kernel forms
+//   u  = m_a WA + m_b WB           (ranks on the shared lattice L)
+//   h  = u mod L                    (phase)
+//   sh = floor(u / L) = t - t_min   (bin, relative to the smallest product)
+//   delta = +-1 from the sign XOR
+// and adds delta * 2^sh to the phase-h accumulator of the current scale block.
+// Within a block the sums are kept in 16-bit-wide parts (int32 counters in
+// shared memory, indexed by phase and part: no data-dependent register
+// indexing); at the end of each scale block they are shifted by
+// (sa + sb) - min_b(sa + sb) and added into exact int128 per-phase sums.
+// The epilogue combines C = sum_h 2^{h/L} S_h 2^lambda in FP64 and rounds
+// once to FP32; the validation form also writes the int128 sums and lambda.
+#include "cfp_common.cuh"
+#include "kernels.cuh"
+
+namespace cfp {
+
+namespace {
+constexpr int TM = 16, TN = 16, NT = TM * TN, KC = 32;
+
+__device__ __forceinline__ int i128_bitlen_ok(int spread, int dt, int64_t K) {
+  return bitlen64(K) + spread + dt <= 127;
+}
+}  // namespace
+
+template <int FA, int FB>
+__global__ void __launch_bounds__(NT) gemm_exact_kernel(const uint8_t* __restrict__ A, const int8_t* __restrict__ sA,
+                                                        const uint8_t* __restrict__ B, const int8_t* __restrict__ sB,
+                                                        int M, int N, int K, int G, float* __restrict__ C,
+                                                        int64_t* __restrict__ phase_sums,
+                                                        int32_t* __restrict__ phase_lsb, uint32_t* status) {
+  using P = Pair<FA, FB>;
+  constexpr int L = P::L;
+  constexpr int DT = P::TMAX - P::TMIN;   // largest bin offset sh
+  constexpr int PARTS = DT / 16 + 1;      // 16-bit parts of a bin offset
+  constexpr uint32_t MA = Fmt<FA>::MMASK, MB = Fmt<FB>::MMASK;
+
+  __shared__ uint32_t As[TM][KC / 4];
+  __shared__ uint32_t Bs[TN][KC / 4];
+  __shared__ int32_t acc[L * PARTS][NT];
+
+  const int tid = threadIdx.x;
+  const int ty = tid / TN, tx = tid % TN;
+  const int i = blockIdx.y * TM + ty, j = blockIdx.x * TN + tx;
+  const bool live = i < M && j < N;
+  const int nb = K / G;
+
+  // lambda = min_b(sa + sb) + t_min; the int128 window check
+  int smin = 1 << 20, smax = -(1 << 20);
+  if (live)
+    for (int b = 0; b < nb; ++b) {
+      int s = (int)sA[(int64_t)i * nb + b] + (int)sB[(int64_t)j * nb + b];
+      smin = min(smin, s);
+      smax = max(smax, s);
+    }
+  const bool in_range = live && i128_bitlen_ok(smax - smin, DT, K);
+  if (live && !in_range && status) atomicOr(status, CURVEFP_DEV_RANGE);
+
+  __int128 S[L];
+#pragma unroll
+  for (int h = 0; h < L; ++h) S[h] = 0;
+#pragma unroll
+  for (int q = 0; q < L * PARTS; ++q) acc[q][tid] = 0;
+
+  for (int k0 = 0; k0 < K; k0 += KC) {
+    // stage a 16x32 code tile of A and of B (one 32-bit word per lane)
+    {
+      const int r = (tid & 127) >> 3, w = tid & 7;
+      if (tid < 128) {
+        const int gi = blockIdx.y * TM + r;
+        As[r][w] = gi < M ? __ldg(reinterpret_cast<const uint32_t*>(A + (int64_t)gi * K + k0) + w) : 0u;
+      } else {
+        const int gj = blockIdx.x * TN + r;
+        Bs[r][w] = gj < N ? __ldg(reinterpret_cast<const uint32_t*>(B + (int64_t)gj * K + k0) + w) : 0u;
+      }
+    }
+    __syncthreads();
+    if (in_range) {
+#pragma unroll
+      for (int w = 0; w < KC / 4; ++w) {
+        const uint32_t aw = As[ty][w], bw = Bs[tx][w];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const uint32_t ca = (aw >> (8 * q)) & 0xFFu, cb = (bw >> (8 * q)) & 0xFFu;
+          const uint32_t ma = ca & MA, mb = cb & MB;
+          if (ma != 0u && mb != 0u) {
+            const uint32_t u = ma * P::WA + mb * P::WB;
+            const uint32_t sh = u >> P::LOG2L;
+            const int idx = (int)(u & (L - 1)) * PARTS + (int)(sh >> 4);
+            const int32_t v = (int32_t)(1u << (sh & 15u));
+            acc[idx][tid] += ((ca ^ cb) & 0x80u) ? -v : v;
+          }
+        }
+      }
+    }
+    __syncthreads();
+    // end of a scale block: fold the parts into the int128 phase sums
+    if (((k0 + KC) % G) == 0) {
+      if (in_range) {
+        const int b = (k0 + KC) / G - 1;
+        const int sb = (int)sA[(int64_t)i * nb + b] + (int)sB[(int64_t)j * nb + b] - smin;
+#pragma unroll
+        for (int h = 0; h < L; ++h)
+#pragma unroll
+          for (int p = 0; p < PARTS; ++p) {
+            const int32_t part = acc[h * PARTS + p][tid];
+            if (part != 0) S[h] += ((__int128)part) << (16 * p + sb);
+          }
+      }
+#pragma unroll
+      for (int q = 0; q < L * PARTS; ++q) acc[q][tid] = 0;
+    }
+  }
+
+  if (!live) return;
+  const int lambda = smin + P::TMIN;
+  const int64_t o = (int64_t)i * N + j;
+  if (C) {
+    float out;
+    if (in_range) {
+      double c = 0.0;
+#pragma unroll
+      for (int h = 0; h < L; ++h) {
+        const int64_t hi = (int64_t)(S[h] >> 64);
+        const uint64_t lo = (uint64_t)S[h];
+        const double sd = fma((double)hi, 18446744073709551616.0, (double)lo);
+        const uint64_t cb = L == 8 ? CFP_PHASE_F64_L8_DEV[h] : CFP_PHASE_F64_L4_DEV[h];
+        c = fma(__longlong_as_double((long long)cb), sd, c);
+      }
+      out = (float)scalbn(c, lambda);
+    } else {
+      out = __int_as_float(0x7fc00000);
+    }
+    C[o] = out;
+  }
+  if (phase_sums) {
+#pragma unroll
+    for (int h = 0; h < L; ++h) {
+      phase_sums[(o * L + h) * 2 + 0] = (int64_t)(uint64_t)S[h];
+      phase_sums[(o * L + h) * 2 + 1] = (int64_t)(S[h] >> 64);
+    }
+  }
+  if (phase_lsb) phase_lsb[o] = lambda;
+}
+
+template <int FA, int FB>
+static cudaError_t launch_exact_t(int G, const uint8_t* a, const int8_t* sa, const uint8_t* b, const int8_t* sb,
+                                  int64_t M, int64_t N, int64_t K, float* c, int64_t* ps, int32_t* pl, uint32_t* st,
+                                  cudaStream_t s) {
+  dim3 grid((unsigned)((N + TN - 1) / TN), (unsigned)((M + TM - 1) / TM));
+  gemm_exact_kernel<FA, FB><<<grid, NT, 0, s>>>(a, sa, b, sb, (int)M, (int)N, (int)K, G, c, ps, pl, st);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gemm_exact(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
+                              const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, int64_t* ps,
+                              int32_t* pl, uint32_t* st, cudaStream_t s) {
+#define CFP_E(X, Y) \
+  if (fa == X && fb == Y) return launch_exact_t<X, Y>(G, a, sa, b, sb, M, N, K, c, ps, pl, st, s);
+  CFP_E(CURVEFP_E3C3, CURVEFP_E3C3)
+  CFP_E(CURVEFP_E3C3, CURVEFP_E4C3)
+  CFP_E(CURVEFP_E3C3, CURVEFP_E5C2)
+  CFP_E(CURVEFP_E4C3, CURVEFP_E3C3)
+  CFP_E(CURVEFP_E4C3, CURVEFP_E4C3)
+  CFP_E(CURVEFP_E4C3, CURVEFP_E5C2)
+  CFP_E(CURVEFP_E5C2, CURVEFP_E3C3)
+  CFP_E(CURVEFP_E5C2, CURVEFP_E4C3)
+  CFP_E(CURVEFP_E5C2, CURVEFP_E5C2)
+#undef CFP_E
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace cfp

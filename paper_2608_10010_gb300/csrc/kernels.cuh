@@ -1,0 +1,21 @@
+// Host-side launchers of the CurveFP kernels (argument validation is done by
+// the C ABI in capi.cu before any of these is called).
+#pragma once
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace cfp {
+
+cudaError_t launch_quantize(int fmt, int G, const void* x, int dtype, int64_t rows, int64_t cols, int64_t ld,
+                            int axis, uint8_t* codes, int8_t* scales, uint32_t* status, cudaStream_t st, int sms);
+cudaError_t launch_dequantize(int fmt, int G, const uint8_t* codes, const int8_t* scales, int64_t n, float* out,
+                              cudaStream_t st, int sms);
+cudaError_t launch_gemm_exact(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
+                              const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, int64_t* phase_sums,
+                              int32_t* phase_lsb, uint32_t* status, cudaStream_t st);
+cudaError_t launch_gemm_tensor(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
+                               const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, uint32_t* status,
+                               cudaStream_t st, int sms);
+bool gemm_tensor_supported(int fa, int fb);
+
+}  // namespace cfp

@@ -1,0 +1,403 @@
+// CurveFP block-scaled quantization and dequantization (Sec. 3.1, Eq. 1).
+//
+// Quantizer: one HBM streaming pass.  Each block of G values is read with
+// 16-byte vector loads by a group of lanes, reduced to max|x| with warp
+// shuffles, turned into the ceil-absmax scale a_b by integer exponent and
+// mantissa arithmetic, and every element is encoded without a search loop:
+//   t  = bits(|x|) - a_b * 2^23           (exponent subtraction = x * 2^{-a_b})
+//   j  = number of midpoints (2^{k/K} + 2^{(k+1)/K})/2 below the mantissa,
+//        from a 256-entry LUT on the top mantissa bits plus one compare
+//   m  = K * (exponent of t) + j + bias   (nearest lattice point, as a rank)
+//   m  = 0 below L_nmin/2, >= 1 otherwise; code = sign << 7 | m.
+// All thresholds are irrational, so no FP32 input ties.  Blocks containing
+// NaN, Inf or values that need subnormal care take an exact slow path.
+#include "cfp_common.cuh"
+#include "kernels.cuh"
+
+namespace cfp {
+
+// Unsigned exponent/mantissa split of a positive finite FP32 bit pattern,
+// normalizing subnormals.
+__device__ __forceinline__ void split_f32(uint32_t absb, int& F, uint32_t& mant) {
+  if (absb >= 0x00800000u) {
+    F = (int)(absb >> 23) - 127;
+    mant = absb & 0x7FFFFFu;
+  } else {
+    int p = 31 - __clz(absb);
+    F = p - 149;
+    mant = (absb << (23 - p)) & 0x7FFFFFu;
+  }
+}
+
+// Number of midpoint thresholds at or below a 23-bit mantissa.
+__device__ __forceinline__ int mid_count(const uint32_t* lut, uint32_t mant) {
+  uint32_t e = lut[mant >> 15];
+  return (int)(e >> 24) + (mant >= (e & 0xFFFFFFu) ? 1 : 0);
+}
+
+// Ceil-absmax block scale from the bit pattern of max|x| (NaN excluded).
+template <int FMT>
+__device__ __forceinline__ int block_scale(uint32_t amaxb) {
+  using F = Fmt<FMT>;
+  if (amaxb == 0u) return 0;
+  if (amaxb >= 0x7F800000u) return 127;
+  int Fx;
+  uint32_t mant;
+  split_f32(amaxb, Fx, mant);
+  int a = Fx - F::EMAX + (mant >= RadixConst<F::K>::MU_SAT ? 1 : 0);
+  return a < -128 ? -128 : (a > 127 ? 127 : a);
+}
+
+// Fast-path encode: finite input, block scale a in [-100, 127].
+template <int FMT>
+__device__ __forceinline__ uint32_t encode_fast(const uint32_t* lut, uint32_t bits, int32_t ashift) {
+  using F = Fmt<FMT>;
+  constexpr int32_t T0 = ((ZeroBoundary<FMT>::FZ + 127) << 23) | (int32_t)RadixConst<F::K>::MU_Z;
+  int32_t t = (int32_t)(bits & 0x7FFFFFFFu) - ashift;
+  uint32_t e = lut[(t >> 15) & 0xFF];
+  int j = (int)(e >> 24) + (((uint32_t)t & 0x7FFFFFu) >= (e & 0xFFFFFFu) ? 1 : 0);
+  int m = ((t >> 23) << F::C) + j + (F::B - 127 * F::K);
+  m = m < 1 ? 1 : m;
+  m = t < T0 ? 0 : m;
+  return (uint32_t)m | ((bits >> 24) & 0x80u);
+}
+
+// Exact encode for any input and scale.  Sets *nan if the input is NaN.
+template <int FMT>
+__device__ __forceinline__ uint32_t encode_slow(const uint32_t* lut, uint32_t bits, int a, bool& nan) {
+  using F = Fmt<FMT>;
+  uint32_t absb = bits & 0x7FFFFFFFu;
+  int m;
+  if (absb > 0x7F800000u) {
+    nan = true;
+    return 0u;
+  } else if (absb == 0x7F800000u) {
+    m = 2 * F::B - 1;
+  } else if (absb == 0u) {
+    return 0u;
+  } else {
+    int Fx;
+    uint32_t mant;
+    split_f32(absb, Fx, mant);
+    int Fv = Fx - a;
+    int j = mid_count(lut, mant);
+    if (Fv > F::EMAX || (Fv == F::EMAX && j == F::K)) {
+      m = 2 * F::B - 1;
+    } else if (Fv < ZeroBoundary<FMT>::FZ || (Fv == ZeroBoundary<FMT>::FZ && mant < RadixConst<F::K>::MU_Z)) {
+      return 0u;
+    } else {
+      m = F::K * Fv + j + F::B;
+      m = m < 1 ? 1 : m;
+    }
+  }
+  return (uint32_t)m | ((bits >> 24) & 0x80u);
+}
+
+template <typename T>
+struct Elem;
+template <>
+struct Elem<float> {
+  static constexpr int VEC = 4;
+  __device__ static __forceinline__ uint32_t bits(const uint4& v, int i) {
+    return i == 0 ? v.x : i == 1 ? v.y : i == 2 ? v.z : v.w;
+  }
+};
+template <>
+struct Elem<uint16_t> {  // BF16 storage
+  static constexpr int VEC = 8;
+  __device__ static __forceinline__ uint32_t bits(const uint4& v, int i) {
+    uint32_t w = (i >> 1) == 0 ? v.x : (i >> 1) == 1 ? v.y : (i >> 1) == 2 ? v.z : v.w;
+    return (i & 1) ? (w & 0xFFFF0000u) : (w << 16);
+  }
+};
+
+template <int K>
+__device__ __forceinline__ const uint32_t* lut_src() {
+  return K == 8 ? CFP_LUT_K8_DEV : CFP_LUT_K4_DEV;
+}
+
+// ---------------------------------------------------------------------------
+// block_axis 0: blocks of G consecutive elements along a row.
+// TPB lanes cooperate on one block; each lane holds VPT 16-byte vectors.
+template <int FMT, typename T, int G>
+__global__ void __launch_bounds__(256) quantize_rows_kernel(const T* __restrict__ x, int64_t rows, int64_t cols,
+                                                            int64_t ld, uint8_t* __restrict__ codes,
+                                                            int8_t* __restrict__ scales, uint32_t* status) {
+  using F = Fmt<FMT>;
+  constexpr int VEC = Elem<T>::VEC;
+  constexpr int VPB = G / VEC;              // vectors per block
+  constexpr int TPB = VPB < 8 ? VPB : 8;    // lanes per block
+  constexpr int VPT = VPB / TPB;            // vectors per lane
+  constexpr int BPW = 32 / TPB;             // blocks per warp step
+  constexpr int UNROLL = VPT >= 4 ? 1 : 4 / VPT;
+
+  __shared__ uint32_t lut[256];
+  for (int i = threadIdx.x; i < 256; i += blockDim.x) lut[i] = lut_src<F::K>()[i];
+  __syncthreads();
+
+  const int lane = threadIdx.x & 31;
+  const int sub = lane % TPB;
+  const int64_t nbc = cols / G;
+  const int64_t nblk = rows * nbc;
+  const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const bool dense = (ld == cols);
+  bool saw_nan = false;
+
+  for (int64_t base = warp * BPW * UNROLL; base < nblk; base += nwarps * BPW * UNROLL) {
+    uint4 v[UNROLL][VPT];
+    int64_t blk[UNROLL];
+#pragma unroll
+    for (int u = 0; u < UNROLL; ++u) {
+      blk[u] = base + (int64_t)u * BPW + lane / TPB;
+      const bool ok = blk[u] < nblk;
+      int64_t off = 0;
+      if (ok) off = dense ? blk[u] * G : (blk[u] / nbc) * ld + (blk[u] % nbc) * G;
+      const uint4* src = reinterpret_cast<const uint4*>(x + off);
+#pragma unroll
+      for (int q = 0; q < VPT; ++q) v[u][q] = ok ? __ldcs(src + q * TPB + sub) : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int u = 0; u < UNROLL; ++u) {
+      // max |x| over the block as an unsigned bit pattern (NaN sorts above Inf)
+      uint32_t mx = 0u;
+#pragma unroll
+      for (int q = 0; q < VPT; ++q)
+#pragma unroll
+        for (int i = 0; i < VEC; ++i) mx = max(mx, Elem<T>::bits(v[u][q], i) & 0x7FFFFFFFu);
+#pragma unroll
+      for (int o = TPB / 2; o > 0; o >>= 1) mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      const bool ok = blk[u] < nblk;
+      int a = block_scale<FMT>(mx);
+      const bool fast = mx < 0x7F800000u && a >= -100;
+      if (__any_sync(0xffffffffu, !fast)) {  // rare: NaN / Inf / subnormal-scale blocks
+        uint32_t mx2 = 0u;
+#pragma unroll
+        for (int q = 0; q < VPT; ++q)
+#pragma unroll
+          for (int i = 0; i < VEC; ++i) {
+            uint32_t b = Elem<T>::bits(v[u][q], i) & 0x7FFFFFFFu;
+            mx2 = max(mx2, b > 0x7F800000u ? 0u : b);
+          }
+#pragma unroll
+        for (int o = TPB / 2; o > 0; o >>= 1) mx2 = max(mx2, __shfl_xor_sync(0xffffffffu, mx2, o));
+        if (!fast) a = block_scale<FMT>(mx2);
+      }
+      if (!ok) continue;
+      uint8_t* dst = codes + blk[u] * G;
+      if (sub == 0) scales[blk[u]] = (int8_t)a;
+      const int32_t ashift = a * (1 << 23);
+#pragma unroll
+      for (int q = 0; q < VPT; ++q) {
+        uint32_t c[VEC];
+        if (fast) {
+#pragma unroll
+          for (int i = 0; i < VEC; ++i) c[i] = encode_fast<FMT>(lut, Elem<T>::bits(v[u][q], i), ashift);
+        } else {
+#pragma unroll
+          for (int i = 0; i < VEC; ++i) c[i] = encode_slow<FMT>(lut, Elem<T>::bits(v[u][q], i), a, saw_nan);
+        }
+        uint8_t* d = dst + (q * TPB + sub) * VEC;
+        if (VEC == 4) {
+          *reinterpret_cast<uint32_t*>(d) = c[0] | (c[1] << 8) | (c[2] << 16) | (c[3] << 24);
+        } else {
+          uint2 w;
+          w.x = c[0] | (c[1] << 8) | (c[2] << 16) | (c[3] << 24);
+          w.y = c[4] | (c[5] << 8) | (c[6] << 16) | (c[7] << 24);
+          *reinterpret_cast<uint2*>(d) = w;
+        }
+      }
+    }
+  }
+  if (saw_nan && status) atomicOr(status, CURVEFP_DEV_NAN);
+}
+
+// ---------------------------------------------------------------------------
+// block_axis 1: blocks of G consecutive rows of one column; the output is the
+// transposed operand (codes [cols x rows]).  One lane owns one column and one
+// row-block: its loads are coalesced across the warp (consecutive columns),
+// its G codes are one contiguous run of the output row.
+template <int FMT, typename T, int G>
+__global__ void __launch_bounds__(256) quantize_cols_kernel(const T* __restrict__ x, int64_t rows, int64_t cols,
+                                                            int64_t ld, uint8_t* __restrict__ codes,
+                                                            int8_t* __restrict__ scales, uint32_t* status) {
+  using F = Fmt<FMT>;
+  __shared__ uint32_t lut[256];
+  for (int i = threadIdx.x; i < 256; i += blockDim.x) lut[i] = lut_src<F::K>()[i];
+  __syncthreads();
+  const int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  const int64_t rb = blockIdx.y;
+  if (c >= cols) return;
+  const int64_t nrb = rows / G;
+  const T* src = x + rb * G * ld + c;
+  auto load_bits = [&](int i) -> uint32_t {
+    if (sizeof(T) == 4) return __float_as_uint(__ldcs(reinterpret_cast<const float*>(src) + i * ld));
+    return (uint32_t)__ldcs(reinterpret_cast<const unsigned short*>(src) + i * ld) << 16;
+  };
+  uint32_t mx = 0u, mxn = 0u;
+  constexpr int KEEP = G <= 32 ? G : 1;
+  uint32_t keep[KEEP];
+#pragma unroll 8
+  for (int i = 0; i < G; ++i) {
+    uint32_t b = load_bits(i);
+    if (G <= 32) keep[i % KEEP] = b;
+    uint32_t ab = b & 0x7FFFFFFFu;
+    mx = max(mx, ab);
+    mxn = max(mxn, ab > 0x7F800000u ? 0u : ab);
+  }
+  const int a = block_scale<FMT>(mxn);
+  const bool fast = mx < 0x7F800000u && a >= -100;
+  scales[c * nrb + rb] = (int8_t)a;
+  const int32_t ashift = a * (1 << 23);
+  bool saw_nan = false;
+  uint8_t* dst = codes + c * rows + rb * G;
+#pragma unroll 1
+  for (int i0 = 0; i0 < G; i0 += 16) {
+    uint32_t w[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      uint32_t acc = 0;
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        const int i = i0 + 4 * q + r;
+        uint32_t b = G <= 32 ? keep[i % KEEP] : load_bits(i);
+        uint32_t code = fast ? encode_fast<FMT>(lut, b, ashift) : encode_slow<FMT>(lut, b, a, saw_nan);
+        acc |= code << (8 * r);
+      }
+      w[q] = acc;
+    }
+    *reinterpret_cast<uint4*>(dst + i0) = make_uint4(w[0], w[1], w[2], w[3]);
+  }
+  if (saw_nan && status) atomicOr(status, CURVEFP_DEV_NAN);
+}
+
+// ---------------------------------------------------------------------------
+// Dequantization: 16 codes per lane (one 16-byte load, four 16-byte stores).
+// Fast path: RN32(2^{k/K}) 2^{e} comes from a 128-entry table indexed by the
+// rank and the block scale is added to the exponent field; blocks whose
+// results could leave the normal FP32 range multiply twice with one rounding.
+template <int FMT>
+__global__ void __launch_bounds__(256) dequantize_kernel(const uint8_t* __restrict__ codes,
+                                                         const int8_t* __restrict__ scales, int64_t n, int G,
+                                                         float* __restrict__ out) {
+  using F = Fmt<FMT>;
+  constexpr int EMIN = -(F::EMAX + 1);
+  __shared__ uint32_t tab[128];
+  for (int m = threadIdx.x; m < 128; m += blockDim.x) {
+    uint32_t v = 0u;
+    if (m >= 1 && m <= 2 * F::B - 1) {
+      int nn = m - F::B;
+      int e = nn >> F::C, k = nn & (F::K - 1);
+      uint32_t ck = F::K == 8 ? CFP_CK_F32_K8_DEV[k] : CFP_CK_F32_K4_DEV[k];
+      v = ck + (uint32_t)(e * (1 << 23));
+    }
+    tab[m] = v;
+  }
+  __syncthreads();
+  const int64_t nchunks = n / 16;
+  for (int64_t ch = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; ch < nchunks;
+       ch += (int64_t)gridDim.x * blockDim.x) {
+    uint4 cv = __ldcs(reinterpret_cast<const uint4*>(codes) + ch);
+    const int a = scales[(ch * 16) / G];
+    const bool fast = (a + EMIN >= -126) && (a + F::EMAX <= 126);
+    uint32_t cw[4] = {cv.x, cv.y, cv.z, cv.w};
+    uint32_t o[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      uint32_t code = (cw[i >> 2] >> (8 * (i & 3))) & 0xFFu;
+      uint32_t m = code & F::MMASK;
+      uint32_t r;
+      if (fast) {
+        r = m ? tab[m] + (uint32_t)(a * (1 << 23)) : 0u;
+      } else if (m == 0u) {
+        r = 0u;
+      } else {
+        int nn = (int)m - F::B;
+        int e = nn >> F::C, k = nn & (F::K - 1);
+        float ck = __uint_as_float(F::K == 8 ? CFP_CK_F32_K8_DEV[k] : CFP_CK_F32_K4_DEV[k]);
+        int E = a + e;
+        int E1 = E < -126 ? -126 : (E > 127 ? 127 : E);
+        int E2 = E - E1;  // in [-18, 15]
+        float y = __fmul_rn(ck, __uint_as_float((uint32_t)(E1 + 127) << 23));
+        y = __fmul_rn(y, __uint_as_float((uint32_t)(E2 + 127) << 23));
+        r = __float_as_uint(y);
+      }
+      o[i] = m ? (r | ((code & 0x80u) << 24)) : 0u;
+    }
+    uint4* d = reinterpret_cast<uint4*>(out) + ch * 4;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) __stcs(d + q, make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]));
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Host-side launchers (called by the C ABI after argument validation).
+
+template <int FMT, typename T, int G>
+static cudaError_t launch_q(const void* x, int64_t rows, int64_t cols, int64_t ld, int axis, uint8_t* codes,
+                            int8_t* scales, uint32_t* status, cudaStream_t st, int sms) {
+  if (axis == 0) {
+    constexpr int VEC = Elem<T>::VEC;
+    constexpr int TPB = (G / VEC) < 8 ? (G / VEC) : 8;
+    const int64_t nblk = rows * (cols / G);
+    constexpr int VPT = (G / VEC) / TPB;
+    constexpr int PER_WARP = (32 / TPB) * (VPT >= 4 ? 1 : 4 / VPT);
+    const int64_t warps_needed = (nblk + PER_WARP - 1) / PER_WARP;
+    int64_t grid = (warps_needed + 7) / 8;
+    const int64_t cap = (int64_t)sms * 8;  // 8 resident CTAs of 256 lanes per SM
+    if (grid > cap) grid = cap;
+    if (grid < 1) grid = 1;
+    quantize_rows_kernel<FMT, T, G><<<(unsigned)grid, 256, 0, st>>>(static_cast<const T*>(x), rows, cols, ld,
+                                                                      codes, scales, status);
+  } else {
+    dim3 grid((unsigned)((cols + 255) / 256), (unsigned)(rows / G));
+    quantize_cols_kernel<FMT, T, G><<<grid, 256, 0, st>>>(static_cast<const T*>(x), rows, cols, ld, codes, scales,
+                                                           status);
+  }
+  return cudaGetLastError();
+}
+
+template <int FMT, typename T>
+static cudaError_t launch_q_g(int G, const void* x, int64_t rows, int64_t cols, int64_t ld, int axis,
+                              uint8_t* codes, int8_t* scales, uint32_t* status, cudaStream_t st, int sms) {
+  switch (G) {
+    case 32: return launch_q<FMT, T, 32>(x, rows, cols, ld, axis, codes, scales, status, st, sms);
+    case 64: return launch_q<FMT, T, 64>(x, rows, cols, ld, axis, codes, scales, status, st, sms);
+    case 128: return launch_q<FMT, T, 128>(x, rows, cols, ld, axis, codes, scales, status, st, sms);
+    case 256: return launch_q<FMT, T, 256>(x, rows, cols, ld, axis, codes, scales, status, st, sms);
+    case 512: return launch_q<FMT, T, 512>(x, rows, cols, ld, axis, codes, scales, status, st, sms);
+  }
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_quantize(int fmt, int G, const void* x, int dtype, int64_t rows, int64_t cols, int64_t ld,
+                            int axis, uint8_t* codes, int8_t* scales, uint32_t* status, cudaStream_t st, int sms) {
+#define CFP_Q(FMT)                                                                                     \
+  return dtype == CURVEFP_F32                                                                          \
+             ? launch_q_g<FMT, float>(G, x, rows, cols, ld, axis, codes, scales, status, st, sms)      \
+             : launch_q_g<FMT, uint16_t>(G, x, rows, cols, ld, axis, codes, scales, status, st, sms);
+  switch (fmt) {
+    case CURVEFP_E3C3: CFP_Q(CURVEFP_E3C3)
+    case CURVEFP_E4C3: CFP_Q(CURVEFP_E4C3)
+    case CURVEFP_E5C2: CFP_Q(CURVEFP_E5C2)
+  }
+#undef CFP_Q
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_dequantize(int fmt, int G, const uint8_t* codes, const int8_t* scales, int64_t n, float* out,
+                              cudaStream_t st, int sms) {
+  int64_t grid = (n / 16 + 255) / 256;
+  const int64_t cap = (int64_t)sms * 8;
+  if (grid > cap) grid = cap;
+  if (grid < 1) grid = 1;
+  switch (fmt) {
+    case CURVEFP_E3C3: dequantize_kernel<CURVEFP_E3C3><<<(unsigned)grid, 256, 0, st>>>(codes, scales, n, G, out); break;
+    case CURVEFP_E4C3: dequantize_kernel<CURVEFP_E4C3><<<(unsigned)grid, 256, 0, st>>>(codes, scales, n, G, out); break;
+    case CURVEFP_E5C2: dequantize_kernel<CURVEFP_E5C2><<<(unsigned)grid, 256, 0, st>>>(codes, scales, n, G, out); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace cfp

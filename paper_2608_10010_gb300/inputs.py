@@ -89,3 +89,19 @@ def bandwidth_tensor(n: int, cols: int = 4096, seed: int = 3) -> np.ndarray:
     with 0.1 % x100 element outliers.  Returned as float32; BF16 callers
     round it once."""
     return elementwise_outliers((n // cols, cols), seed)
+
+
+def bandwidth_tensor_cuda(n: int, cols: int = 4096, seed: int = 3):
+    """Device-side generator for the quantize-only sweep (sizes up to 2^30
+    elements are too slow to draw on the host): BF16 [n/cols x cols], N(0,1)
+    with each element independently (p = 0.001) scaled by 100.  Uses torch's
+    CUDA generator, so values differ from ``bandwidth_tensor`` but follow the
+    same distribution."""
+    import torch
+
+    g = torch.Generator(device="cuda").manual_seed(seed)
+    x = torch.randn((n // cols, cols), device="cuda", generator=g, dtype=torch.float32)
+    mask = torch.rand((n // cols, cols), device="cuda", generator=g) < 0.001
+    x = torch.where(mask, x * 100.0, x)
+    del mask
+    return x.to(torch.bfloat16)

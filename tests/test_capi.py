@@ -1,0 +1,85 @@
+"""The C-ABI library loads, exports every entry point that include/curvefp.h
+declares, and rejects bad arguments on the host (no GPU needed: argument
+validation happens before any CUDA call)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "curvefp.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_10010_gb300 import _build, load
+
+    _build.build()
+    return load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(curvefp_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for f in ("curvefp_quantize", "curvefp_dequantize", "curvefp_gemm", "curvefp_gemm_phases"):
+        assert f in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_static_queries(lib):
+    assert lib.curvefp_phase_count(0, 0) == 8
+    assert lib.curvefp_phase_count(1, 1) == 8
+    assert lib.curvefp_phase_count(2, 2) == 4
+    assert lib.curvefp_phase_count(2, 1) == 8
+    assert lib.curvefp_phase_count(7, 1) == -1
+    assert lib.curvefp_status_string(0) == b"ok"
+    assert lib.curvefp_status_string(1) == b"invalid argument"
+    assert b"sm_103a" in lib.curvefp_version()
+
+
+def test_host_side_validation(lib):
+    P = ctypes.c_void_p
+    dummy = P(4096)  # never dereferenced: every call below fails validation first
+    INVALID = 1
+    # bad format, bad block, bad dtype, bad axis, ld < cols
+    assert lib.curvefp_quantize(9, 32, dummy, 0, 4, 64, 64, 0, dummy, dummy, None, None) == INVALID
+    assert lib.curvefp_quantize(1, 33, dummy, 0, 4, 64, 64, 0, dummy, dummy, None, None) == INVALID
+    assert lib.curvefp_quantize(1, 32, dummy, 5, 4, 64, 64, 0, dummy, dummy, None, None) == INVALID
+    assert lib.curvefp_quantize(1, 32, dummy, 0, 4, 64, 64, 2, dummy, dummy, None, None) == INVALID
+    assert lib.curvefp_quantize(1, 32, dummy, 0, 4, 64, 32, 0, dummy, dummy, None, None) == INVALID
+    # cols not a multiple of the block (axis 0), rows not (axis 1)
+    assert lib.curvefp_quantize(1, 32, dummy, 0, 4, 48, 48, 0, dummy, dummy, None, None) == INVALID
+    assert lib.curvefp_quantize(1, 32, dummy, 0, 48, 64, 64, 1, dummy, dummy, None, None) == INVALID
+    # NULL and misaligned pointers
+    assert lib.curvefp_quantize(1, 32, None, 0, 4, 64, 64, 0, dummy, dummy, None, None) == INVALID
+    assert lib.curvefp_quantize(1, 32, P(4100), 0, 4, 64, 64, 0, dummy, dummy, None, None) == INVALID
+    # empty input is a no-op
+    assert lib.curvefp_quantize(1, 32, None, 0, 0, 64, 64, 0, None, None, None, None) == 0
+    assert lib.curvefp_dequantize(1, 32, None, None, 0, 64, None, None) == 0
+    assert lib.curvefp_dequantize(1, 32, dummy, dummy, 4, 48, dummy, None) == INVALID
+    # GEMM: K not a multiple of the block, non-positive sizes, bad algo
+    assert lib.curvefp_gemm(0, 1, 1, 32, dummy, dummy, dummy, dummy, 4, 4, 48, dummy, None, None) == INVALID
+    assert lib.curvefp_gemm(0, 1, 1, 32, dummy, dummy, dummy, dummy, 0, 4, 64, dummy, None, None) == INVALID
+    assert lib.curvefp_gemm(7, 1, 1, 32, dummy, dummy, dummy, dummy, 4, 4, 64, dummy, None, None) == INVALID
+    assert lib.curvefp_gemm_phases(1, 1, 32, dummy, dummy, dummy, dummy, 4, 4, 64, None, None, dummy, None, None) == INVALID
+
+
+def test_product_path_does_not_touch_the_oracle():
+    """The CUDA library and its binding neither import nor link the oracle."""
+    pkg = os.path.join(ROOT, "paper_2608_10010_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h")):
+                text = open(os.path.join(dirpath, f)).read()
+                assert not re.search(r"^\s*(import|from)\s+oracle\b", text, flags=re.M), f
+                assert "liboracle" not in text and "curvefp_oracle" not in text, f
