@@ -5,7 +5,8 @@ One step = one pass of the whole path over the E3C3 Llama-7B-like linear:
 quantize W[4096x4096] and X[2048x4096] (FP32 in, block 32 along K), the
 closed-product GEMM C = X_hat W_hat^T on the tensor cores, and the
 dequantization of X's codes.  Inputs are resident in HBM; L2 is flushed
-between steps (a 256 MiB write outside the per-step events).
+between steps (a 256 MiB write and a 256 MiB read, outside the per-step
+events).
 
 Prints ONE JSON line (rank 0).  `value` is whole-job throughput in
 algorithmic TOPS (2*M*N*K per step / step time; one closed product plus one
@@ -148,7 +149,14 @@ def run_ours(args):
     C = torch.empty((M, N), dtype=torch.float32, device=dev)
     Xh = torch.empty((M, K), dtype=torch.float32, device=dev)
     status = torch.zeros(1, dtype=torch.int32, device=dev)
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    flush_w = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    flush_r = torch.ones(64 << 20, dtype=torch.float32, device=dev)
+
+    def flush_l2():
+        # write 256 MiB, then read 256 MiB: L2 (129 MB) ends up holding clean,
+        # unrelated lines, so no kernel inherits dirty write-backs
+        flush_w.fill_(1)
+        flush_r.sum()
     stream = torch.cuda.current_stream(dev)
 
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
@@ -170,7 +178,7 @@ def run_ours(args):
             ev[4].record(stream)
 
     for _ in range(args.warmup):
-        flush.fill_(1)
+        flush_l2()
         step()
     torch.cuda.synchronize()
     assert int(status.item()) == 0, f"device status {int(status.item())}"
@@ -182,7 +190,7 @@ def run_ours(args):
     with ClockSampler(local) as clk:
         wall0 = time.perf_counter()
         for _ in range(args.steps):
-            flush.fill_(1)  # L2 flush, outside the step's events
+            flush_l2()  # outside the step's events
             step(record=True)
             ev[4].synchronize()
             per["quant_w"].append(ev[0].elapsed_time(ev[1]))
@@ -236,7 +244,7 @@ def run_ours(args):
     torch.cuda.synchronize()
     e2e_ms = []
     for _ in range(args.steps):
-        flush.fill_(1)
+        flush_l2()
         e0.record(stream)
         e2e_step()
         e1.record(stream)
@@ -271,7 +279,7 @@ def run_ours(args):
         "data": "synthetic (seeded; stands in for real LLM weights/activations)",
         "config": {"workload": WORKLOAD, "M": M, "N": N, "K": K, "block": G, "format": FMT,
                    "input": "fp32", "gemm_kernel": "tensor (tcgen05 phase planes)",
-                   "l2": "flushed between steps (256 MiB write outside the per-step events)",
+                   "l2": "flushed between steps (256 MiB write + 256 MiB read, outside the per-step events)",
                    "parallelism": f"replicas x{ws}"},
         "roofline": {"bound": "tensor", "achieved": round(gemm_tops, 4), "peak": bf16_sus,
                      "unit": "TFLOP/s", "frac": round(gemm_tops / bf16_sus, 6), "traffic": None,
@@ -353,7 +361,7 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -69,7 +69,8 @@ typedef enum { CURVEFP_GEMM_EXACT = 0, CURVEFP_GEMM_TENSOR = 1 } curvefp_gemm_al
 /* Block-scaled quantization Q(X) (Sec. 3.1; ceil-absmax scale, nearest level in
  * absolute error over {0} U {2^{n/K}}, saturation at 2^{(B-1)/K}).
  *   x        : [rows x cols] FP32 or BF16 with leading dimension ld >= cols
- *              (elements); 16-byte aligned, ld * element size a multiple of 16.
+ *              (elements), aligned to its element size; for block_axis 0 also
+ *              16-byte aligned with ld * element size a multiple of 16.
  *   block    : G in {32, 64, 128, 256, 512}.
  *   block_axis 0: blocks of G consecutive elements of a row (cols % G == 0);
  *              codes [rows x cols] dense, scales [rows x cols/G].

@@ -37,7 +37,9 @@ curvefp_status_t curvefp_quantize(curvefp_format_t fmt, int block, const void* x
   if (rows == 0 || cols == 0) return CURVEFP_OK;
   if (!x || !codes || !scales) return CURVEFP_ERR_INVALID_ARG;
   const int64_t esz = dtype == CURVEFP_F32 ? 4 : 2;
-  if (!al16(x) || !al16(codes) || (ld * esz) % 16 != 0) return CURVEFP_ERR_INVALID_ARG;
+  if (!al16(codes) || (reinterpret_cast<uintptr_t>(x) % esz) != 0) return CURVEFP_ERR_INVALID_ARG;
+  // the row-blocked kernel reads 16-byte vectors; the column-blocked one reads elements
+  if (block_axis == 0 && (!al16(x) || (ld * esz) % 16 != 0)) return CURVEFP_ERR_INVALID_ARG;
   if (block_axis == 0 && cols % block != 0) return CURVEFP_ERR_INVALID_ARG;
   if (block_axis == 1 && rows % block != 0) return CURVEFP_ERR_INVALID_ARG;
   if (block_axis == 1 && rows / block > 65535) return CURVEFP_ERR_UNSUPPORTED;

@@ -24,6 +24,18 @@ constexpr int TM = 16, TN = 16, NT = TM * TN, KC = 32;
 __device__ __forceinline__ int i128_bitlen_ok(int spread, int dt, int64_t K) {
   return bitlen64(K) + spread + dt <= 127;
 }
+
+// int128 -> double without cancellation: split the magnitude, not the
+// two's-complement words (error <= 2^-52 relative).
+__device__ __forceinline__ double i128_to_double(__int128 v) {
+  const int64_t hi = (int64_t)(v >> 64);
+  const uint64_t lo = (uint64_t)v;
+  if ((hi == 0 && (int64_t)lo >= 0) || (hi == -1 && (int64_t)lo < 0)) return (double)(int64_t)lo;
+  const bool neg = hi < 0;
+  const unsigned __int128 m = neg ? (unsigned __int128)0 - (unsigned __int128)v : (unsigned __int128)v;
+  const double d = fma((double)(uint64_t)(m >> 64), 18446744073709551616.0, (double)(uint64_t)m);
+  return neg ? -d : d;
+}
 }  // namespace
 
 template <int FA, int FB>
@@ -107,7 +119,7 @@ __global__ void __launch_bounds__(NT) gemm_exact_kernel(const uint8_t* __restric
 #pragma unroll
           for (int p = 0; p < PARTS; ++p) {
             const int32_t part = acc[h * PARTS + p][tid];
-            if (part != 0) S[h] += ((__int128)part) << (16 * p + sb);
+            if (part != 0) S[h] += (__int128)((unsigned __int128)(__int128)part << (16 * p + sb));
           }
       }
 #pragma unroll
@@ -124,9 +136,7 @@ __global__ void __launch_bounds__(NT) gemm_exact_kernel(const uint8_t* __restric
       double c = 0.0;
 #pragma unroll
       for (int h = 0; h < L; ++h) {
-        const int64_t hi = (int64_t)(S[h] >> 64);
-        const uint64_t lo = (uint64_t)S[h];
-        const double sd = fma((double)hi, 18446744073709551616.0, (double)lo);
+        const double sd = i128_to_double(S[h]);
         const uint64_t cb = L == 8 ? CFP_PHASE_F64_L8_DEV[h] : CFP_PHASE_F64_L4_DEV[h];
         c = fma(__longlong_as_double((long long)cb), sd, c);
       }

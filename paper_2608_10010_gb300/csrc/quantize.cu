@@ -58,8 +58,8 @@ __device__ __forceinline__ uint32_t encode_fast(const uint32_t* lut, uint32_t bi
   int j = (int)(e >> 24) + (((uint32_t)t & 0x7FFFFFu) >= (e & 0xFFFFFFu) ? 1 : 0);
   int m = ((t >> 23) << F::C) + j + (F::B - 127 * F::K);
   m = m < 1 ? 1 : m;
-  m = t < T0 ? 0 : m;
-  return (uint32_t)m | ((bits >> 24) & 0x80u);
+  const uint32_t code = (uint32_t)m | ((bits >> 24) & 0x80u);
+  return t < T0 ? 0u : code;  // zero is always 0x00, whatever the sign
 }
 
 // Exact encode for any input and scale.  Sets *nan if the input is NaN.
