@@ -22,13 +22,15 @@
 // PP = 3 phases over the whole K; each pass adds its part of
 // sum_h 2^{h/L} S_h into C.
 //
-// Roles (288 threads):
-//   warps 0-3  A producers: codes -> planes in registers -> TMEM (tcgen05.st);
+// Roles (544 threads; every 32-byte run of codes of a row is split between
+// two producer threads so that each SM sub-partition has several producer
+// warps to hide latency):
+//   warps 0-7  A producers: codes -> planes in registers -> TMEM (tcgen05.st);
 //              A is the TMEM operand of the MMA and costs no shared-memory
 //              bandwidth.  At the end of each pass they run the epilogue.
-//   warps 4-7  B producers: codes -> the planes (and x2 carry planes) that the
+//   warps 8-15 B producers: codes -> the planes (and x2 carry planes) that the
 //              current pass needs -> shared memory, K-major core-matrix layout.
-//   warp 8     TMEM allocation and the single MMA-issuing thread.
+//   warp 16    TMEM allocation and the single MMA-issuing thread.
 // mbarriers hand stages between the roles; every wait is bounded.
 #include "cfp_common.cuh"
 #include "kernels.cuh"
@@ -49,19 +51,29 @@ struct TcCfg {
   using P = Pair<FA, FB>;
   static constexpr int KA = Fmt<FA>::K, KB = Fmt<FB>::K, L = P::L, WA = P::WA, WB = P::WB, LOG2L = P::LOG2L;
   static constexpr int FA_ = FA, FB_ = FB;
-  static constexpr int BM = 128, BN = 128;
+  static constexpr int BM = 128;
   static constexpr int KS = PT == PLANE_BF16 ? 16 : 32;  // K per MMA = K per pipeline step (32 bytes per row)
-  static constexpr int PP = 3;                            // phases per pass
+  // Columns per CTA (= MMA N) and phases per pass: 4 accumulators of 96
+  // columns leave 128 TMEM columns for A; N = 96 still runs the MMA at full
+  // rate (the per-instruction floor is ~45 cycles, a 128x96x32 FP8 MMA is 48).
+  static constexpr int BN = 96;
+  static constexpr int PP = 4;                            // phases per pass
   static constexpr int NP = (L + PP - 1) / PP;            // passes
   static constexpr int ACC_COLS = PP * BN;
-  static constexpr int ACOLS = KA * 8;                    // TMEM columns of one A step (8 per plane)
+  // A is staged in half-steps ("units"): unit 2g + ph holds planes
+  // [ph APH, (ph + 1) APH) of step g, 8 TMEM columns per plane; NAU units rotate.
+  static constexpr int APH = KA / 2;
+  static constexpr int AU_COLS = APH * 8;
+  static constexpr int NAU = 4;
   static constexpr int ACOL0 = ACC_COLS;
-  static_assert(ACC_COLS + 2 * ACOLS <= 512, "TMEM budget");
+  static_assert(ACC_COLS + NAU * AU_COLS <= 512, "TMEM budget");
   static constexpr int PLANE_BYTES = BN * 32;             // 128 rows x 32 bytes
   static constexpr int NSB = 4;                           // B stages
   static constexpr int PBA = FA == CURVEFP_E5C2 ? 1 : 0;  // plane exponent bias
   static constexpr int PBB = FB == CURVEFP_E5C2 ? 1 : 0;
-  static constexpr int THREADS = 288;
+  static constexpr int NBT = 2 * BN;                      // B producer threads (two per row)
+  static constexpr int THREADS = 256 + NBT + 32;          // A producers, B producers, MMA warp
+  static constexpr int MMA_WARP = (256 + NBT) / 32;
   // D = F32, A = B = BF16 (kind::f16) or E5M2 (kind::f8f6f4): same bit pattern
   static constexpr uint32_t IDESC = tc::idesc_bf16_f32(BM, BN);
 
@@ -108,10 +120,10 @@ struct TcCfg {
 };
 
 struct TcShared {
-  uint64_t a_full[2], a_empty[2], b_full[4], b_empty[4], acc_full, drain;
+  uint64_t a_full[4], a_empty[4], b_full[4], b_empty[4], acc_full, drain;
   uint32_t tmem_base;
   int abort_flag;
-  int refB[128];
+  int refB[128];  // >= BN
 };
 
 __device__ __forceinline__ void raise_flag(uint32_t* status, uint32_t bit) {
@@ -203,26 +215,26 @@ __device__ __forceinline__ uint32_t plane_of(uint32_t v, const uint32_t (&mk)[3]
   return r;
 }
 
-// Decode one 32-byte code run (KS codes) of a row: eight value words in the
-// order the MMA operands expect along K (word w holds elements 4w..4w+3 as
-// E5M2 bytes, or 2w..2w+1 as BF16 halves), the x2 carry words if asked, and
-// the curve-index masks of every word.
+// Decode one half of a 32-byte code run (KS/2 codes) of a row: four value
+// words in the order the MMA operands expect along K (word w holds elements
+// 4w..4w+3 as E5M2 bytes, or 2w..2w+1 as BF16 halves), the x2 carry words if
+// asked, and the curve-index masks of every word.
 template <int FMT, int PT>
-__device__ __forceinline__ void decode_run(const uint4 (&cw)[2], int off, uint32_t (&v)[8], uint32_t (&vc)[8],
-                                           uint32_t (&mk)[8][3], bool want_carry) {
+__device__ __forceinline__ void decode_half(const uint4& cw, int off, uint32_t (&v)[4], uint32_t (&vc)[4],
+                                            uint32_t (&mk)[4][3], bool want_carry) {
   constexpr int KBITS = Fmt<FMT>::C;
   if (PT == PLANE_E5M2) {
-    const uint32_t w[8] = {cw[0].x, cw[0].y, cw[0].z, cw[0].w, cw[1].x, cw[1].y, cw[1].z, cw[1].w};
+    const uint32_t w[4] = {cw.x, cw.y, cw.z, cw.w};
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
+    for (int i = 0; i < 4; ++i) {
       v[i] = e5m2_word<FMT>(w[i], off);
       vc[i] = want_carry ? e5m2_word<FMT>(w[i], off + 1) : 0u;
       k_masks<PT, KBITS>(w[i], mk[i]);
     }
   } else {
-    const uint32_t w[4] = {cw[0].x, cw[0].y, cw[0].z, cw[0].w};
+    const uint32_t w[2] = {cw.x, cw.y};
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
+    for (int i = 0; i < 4; ++i) {
       const uint32_t w2 = __byte_perm(w[i >> 1], 0u, (i & 1) ? 0x4342u : 0x4140u);
       v[i] = bf16_word<FMT>(w2, off);
       vc[i] = want_carry ? bf16_word<FMT>(w2, off + 1) : 0u;
@@ -231,57 +243,74 @@ __device__ __forceinline__ void decode_run(const uint4 (&cw)[2], int off, uint32
   }
 }
 
+// One 16-byte core-matrix row (chunk kc of the run) of every B plane the pass needs.
 template <class Cfg, int PT, int PASS>
-__device__ __forceinline__ void write_b_planes(uint8_t* stage, int row, const uint32_t (&v)[8],
-                                               const uint32_t (&vc)[8], const uint32_t (&mk)[8][3]) {
+__device__ __forceinline__ void write_b_planes(uint8_t* stage, int row, int kc, const uint32_t (&v)[4],
+                                               const uint32_t (&vc)[4], const uint32_t (&mk)[4][3]) {
   constexpr int KBITS = Fmt<Cfg::FB_>::C;
-  const uint32_t core = (uint32_t)((row >> 3) * 256 + (row & 7) * 16);
+  const uint32_t core = (uint32_t)((row >> 3) * 256 + kc * 128 + (row & 7) * 16);
 #pragma unroll
   for (int c = 0; c < 2; ++c)
 #pragma unroll
     for (int k2 = 0; k2 < Cfg::KB; ++k2) {
       const int sl = Cfg::slot(PASS, c, k2);
       if (sl < 0) continue;
+      uint32_t o[4];
 #pragma unroll
-      for (int kc = 0; kc < 2; ++kc) {
-        uint32_t o[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) o[q] = plane_of<KBITS>(c ? vc[4 * kc + q] : v[4 * kc + q], mk[4 * kc + q], k2);
-        *reinterpret_cast<uint4*>(stage + (size_t)sl * Cfg::PLANE_BYTES + core + kc * 128) =
-            make_uint4(o[0], o[1], o[2], o[3]);
-      }
+      for (int q = 0; q < 4; ++q) o[q] = plane_of<KBITS>(c ? vc[q] : v[q], mk[q], k2);
+      *reinterpret_cast<uint4*>(stage + (size_t)sl * Cfg::PLANE_BYTES + core) = make_uint4(o[0], o[1], o[2], o[3]);
     }
 }
 
-template <class Cfg, int PT, int PASS>
-__device__ __forceinline__ void issue_pass(uint32_t tmem, uint64_t bdesc0, int abuf, int bstage, bool first_step) {
+template <class Cfg, int PT, int PASS, int PH>
+__device__ __forceinline__ void issue_pass(uint32_t leader, uint32_t tmem, uint64_t bdesc0, int abuf, int bstage,
+                                           bool first_step) {
 #pragma unroll
-  for (int k1 = 0; k1 < Cfg::KA; ++k1)
+  for (int k1 = PH * Cfg::APH; k1 < (PH + 1) * Cfg::APH; ++k1)
 #pragma unroll
     for (int k2 = 0; k2 < Cfg::KB; ++k2) {
       const int h = Cfg::phase(k1, k2);
       if (h / Cfg::PP != PASS) continue;
       const int sl = Cfg::slot(PASS, Cfg::carry(k1, k2), k2);
-      const uint32_t a_t = tmem + Cfg::ACOL0 + abuf * Cfg::ACOLS + k1 * 8;
+      const uint32_t a_t = tmem + Cfg::ACOL0 + abuf * Cfg::AU_COLS + (k1 - PH * Cfg::APH) * 8;
       const uint64_t bd = bdesc0 + (uint64_t)((bstage * Cfg::BSTAGE + sl * Cfg::PLANE_BYTES) >> 4);
       const uint32_t d_t = tmem + (h - PASS * Cfg::PP) * Cfg::BN;
       const uint32_t accum = (first_step && Cfg::first_of_phase(k1, k2)) ? 0u : 1u;
       if (PT == PLANE_BF16)
-        tc::mma_f16_ts(d_t, a_t, bd, Cfg::IDESC, accum);
+        tc::mma_f16_ts_if(leader, d_t, a_t, bd, Cfg::IDESC, accum);
       else
-        tc::mma_f8_ts(d_t, a_t, bd, Cfg::IDESC, accum);
+        tc::mma_f8_ts_if(leader, d_t, a_t, bd, Cfg::IDESC, accum);
     }
+}
+
+template <class Cfg, int PT, int PH>
+__device__ __forceinline__ void issue_step(uint32_t leader, int p, uint32_t tmem, uint64_t bdesc0, int abuf,
+                                           int bstage, bool first_step) {
+  if (p == 0) issue_pass<Cfg, PT, 0, PH>(leader, tmem, bdesc0, abuf, bstage, first_step);
+  if (Cfg::NP > 1 && p == 1)
+    issue_pass<Cfg, PT, (Cfg::NP > 1 ? 1 : 0), PH>(leader, tmem, bdesc0, abuf, bstage, first_step);
+  if (Cfg::NP > 2 && p == 2)
+    issue_pass<Cfg, PT, (Cfg::NP > 2 ? 2 : 0), PH>(leader, tmem, bdesc0, abuf, bstage, first_step);
+}
+
+__device__ __forceinline__ float phase_const(int L, int h) {
+  return __uint_as_float(L == 8 ? CFP_PHASE_F32_L8_DEV[h] : CFP_PHASE_F32_L4_DEV[h]);
 }
 
 }  // namespace
 
+// Thread layout: warps 0-7 produce A (warp w: TMEM lane group w & 3, half
+// w >> 2 of each 32-byte run) and run the epilogue (columns [BN/2 half,
+// BN/2 (half + 1))); the next 2 BN threads produce B (thread 256 + t: row
+// t % BN, half t / BN); the last warp allocates TMEM and issues the MMAs.
 template <int FA, int FB, int PT>
-__global__ void __launch_bounds__(288, 1) gemm_tc_kernel(const uint8_t* __restrict__ A, const int8_t* __restrict__ sA,
+__global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(const uint8_t* __restrict__ A, const int8_t* __restrict__ sA,
                                                          const uint8_t* __restrict__ B, const int8_t* __restrict__ sB,
                                                          int M, int N, int K, int G, float* __restrict__ C,
                                                          uint32_t* status) {
   using Cfg = TcCfg<FA, FB, PT>;
   constexpr int L = Cfg::L, PP = Cfg::PP, NP = Cfg::NP, BN = Cfg::BN, NSB = Cfg::NSB;
+  constexpr int HALF_BYTES = 16;  // bytes of codes per producer thread and step (E5M2); 8 for BF16
   static_assert(NP <= 3, "pass dispatch");
   extern __shared__ __align__(1024) uint8_t smem[];
   uint8_t* bstage = smem;
@@ -292,102 +321,100 @@ __global__ void __launch_bounds__(288, 1) gemm_tc_kernel(const uint8_t* __restri
   const int nb = K / G, nsub = K / Cfg::KS, total = NP * nsub;
 
   if (tid == 0) {
-    for (int s = 0; s < 2; ++s) {
-      tc::mbar_init(&sh.a_full[s], 128);
+    for (int s = 0; s < Cfg::NAU; ++s) {
+      tc::mbar_init(&sh.a_full[s], 256);
       tc::mbar_init(&sh.a_empty[s], 1);
     }
     for (int s = 0; s < NSB; ++s) {
-      tc::mbar_init(&sh.b_full[s], 128);
+      tc::mbar_init(&sh.b_full[s], Cfg::NBT);
       tc::mbar_init(&sh.b_empty[s], 1);
     }
     tc::mbar_init(&sh.acc_full, 1);
     tc::mbar_init(&sh.drain, 1);
     sh.abort_flag = 0;
   }
-  if (warp == 8) {
+  if (warp == Cfg::MMA_WARP) {
     tc::tmem_alloc(&sh.tmem_base, 512);
     tc::tmem_relinquish();
   }
-  // reference exponents: largest block scale of each A row / B row
+  // producer geometry and the row's reference exponent (largest block scale)
+  const bool is_a = warp < 8;
+  const bool is_prod = warp < Cfg::MMA_WARP;
+  const int rloc = is_a ? ((warp & 3) * 32 + lane) : ((tid - 256) % BN);
+  const int half = is_a ? (warp >> 2) : ((tid - 256) / BN);
+  const int r = (is_a ? m0 : n0) + rloc;
+  const bool rowok = is_prod && r < (is_a ? M : N);
   int ref = -128;
-  if (warp < 8) {
-    const int r = warp < 4 ? m0 + tid : n0 + tid - 128;
-    const int lim = warp < 4 ? M : N;
-    const int8_t* s = warp < 4 ? sA : sB;
-    if (r < lim) {
+  if (rowok) {
+    const int8_t* s = (is_a ? sA : sB) + (int64_t)r * nb;
 #pragma unroll 8
-      for (int b = 0; b < nb; ++b) ref = max(ref, (int)__ldg(s + (int64_t)r * nb + b));
-    }
-    if (warp >= 4) sh.refB[tid - 128] = ref;
+    for (int b = 0; b < nb; ++b) ref = max(ref, (int)__ldg(s + b));
   }
+  if (!is_a && is_prod && half == 0) sh.refB[rloc] = ref;
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = sh.tmem_base;
 
-  if (warp < 8) {
+  if (is_prod) {
     // ------------------------------ producers ------------------------------
-    const bool is_a = warp < 4;
-    const int rloc = is_a ? tid : tid - 128;
-    const int r = (is_a ? m0 : n0) + rloc;
-    const bool rowok = r < (is_a ? M : N);
-    const uint8_t* src = (is_a ? A : B) + (int64_t)r * K;
+    const uint8_t* src = (is_a ? A : B) + (int64_t)r * K + half * (PT == PLANE_E5M2 ? HALF_BYTES : 8);
     const int8_t* srow = (is_a ? sA : sB) + (int64_t)r * nb;
     const int bias = is_a ? Cfg::PBA : Cfg::PBB;
-    auto load = [&](int g, uint4 (&cw)[2], int& off) {
-      cw[0] = cw[1] = make_uint4(0, 0, 0, 0);
+    auto load = [&](int g, uint4& cw, int& off) {
+      cw = make_uint4(0, 0, 0, 0);
       off = 0;
       if (rowok && g < total) {
         const int s = g % nsub;
-        const uint4* p = reinterpret_cast<const uint4*>(src + (int64_t)s * Cfg::KS);
-        cw[0] = __ldg(p);
-        if (Cfg::KS == 32) cw[1] = __ldg(p + 1);
-        off = (int)__ldg(srow + (s * Cfg::KS) / G) - ref - bias;
+        const uint8_t* p = src + (int64_t)s * Cfg::KS;
+        if (PT == PLANE_E5M2) {
+          cw = __ldg(reinterpret_cast<const uint4*>(p));
+        } else {
+          const uint2 t = __ldg(reinterpret_cast<const uint2*>(p));
+          cw.x = t.x;
+          cw.y = t.y;
+        }
+        off = (int)__ldg(srow + (s * Cfg::KS) / G);  // raw scale: consumed two steps later
       }
     };
-    uint4 n1[2], n2[2];
-    int o1, o2;
-    load(0, n1, o1);
-    load(1, n2, o2);
-    const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
-    float cf[L];
-#pragma unroll
-    for (int h = 0; h < L; ++h) cf[h] = __uint_as_float(L == 8 ? CFP_PHASE_F32_L8_DEV[h] : CFP_PHASE_F32_L4_DEV[h]);
-
-    for (int g = 0; g < total; ++g) {
-      uint4 cw[2] = {n1[0], n1[1]};
-      const int off = o1;
-      n1[0] = n2[0];
-      n1[1] = n2[1];
-      o1 = o2;
-      load(g + 2, n2, o2);  // keep two steps of codes in flight
+    const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+    // One pipeline step of this producer thread; false ends the loop (abort).
+    auto step = [&](const int g, const uint4 cw, const int raw_scale) -> bool {
+      const int off = raw_scale - ref - bias;
       const int p = g / nsub, s = g % nsub;
-      uint32_t v[8], vc[8], mk[8][3];
+      uint32_t v[4], vc[4], mk[4][3];
       if (is_a) {
-        const int buf = g & 1;
+        decode_half<FA, PT>(cw, off, v, vc, mk, false);
         bool fail = false;
-        if (g >= 2) {
-          fail = !tc::mbar_wait(&sh.a_empty[buf], ((g >> 1) - 1) & 1);
-          tc::fence_after_sync();
-        }
-        if (fail) {
-          raise_flag(status, CURVEFP_DEV_TIMEOUT);
-          sh.abort_flag = 1;
-        }
-        if (__any_sync(0xffffffffu, fail || read_abort(&sh.abort_flag))) break;
-        decode_run<FA, PT>(cw, off, v, vc, mk, false);
 #pragma unroll
-        for (int g4 = 0; g4 < Cfg::KA / 4; ++g4) {
-          uint32_t reg[32];
+        for (int ph = 0; ph < 2; ++ph) {
+          const int u = 2 * g + ph, buf = u & (Cfg::NAU - 1);
+          if (u >= Cfg::NAU) {
+            fail = !tc::mbar_wait(&sh.a_empty[buf], ((u / Cfg::NAU) - 1) & 1);
+            tc::fence_after_sync();
+          }
+          if (fail) {
+            raise_flag(status, CURVEFP_DEV_TIMEOUT);
+            sh.abort_flag = 1;
+          }
+          if (__any_sync(0xffffffffu, fail || read_abort(&sh.abort_flag))) {
+            fail = true;
+            return false;
+          }
+          // plane k1 of the half occupies 8 columns of the unit; this thread's
+          // half of the 32-byte run is columns 4 half .. 4 half + 3
 #pragma unroll
-          for (int pl = 0; pl < 4; ++pl)
+          for (int j = 0; j < Cfg::APH; ++j) {
+            uint32_t reg[4];
 #pragma unroll
-            for (int c = 0; c < 8; ++c) reg[pl * 8 + c] = plane_of<Fmt<FA>::C>(v[c], mk[c], 4 * g4 + pl);
-          tc::tmem_st32(lane_base + Cfg::ACOL0 + buf * Cfg::ACOLS + g4 * 32, reg);
+            for (int c = 0; c < 4; ++c) reg[c] = plane_of<Fmt<FA>::C>(v[c], mk[c], ph * Cfg::APH + j);
+            tc::tmem_st4(lane_base + Cfg::ACOL0 + buf * Cfg::AU_COLS + j * 8 + half * 4, reg);
+          }
+          tc::tmem_wait_st();
+          tc::fence_before_sync();
+          tc::mbar_arrive(&sh.a_full[buf]);
         }
-        tc::tmem_wait_st();
-        tc::fence_before_sync();
-        tc::mbar_arrive(&sh.a_full[buf]);
+        if (fail) return false;
 
         if (s == nsub - 1) {
           // ---------------- epilogue of pass p -----------------------------
@@ -398,29 +425,42 @@ __global__ void __launch_bounds__(288, 1) gemm_tc_kernel(const uint8_t* __restri
           }
           tc::fence_after_sync();
 #pragma unroll 1
-          for (int c0 = 0; c0 < BN; c0 += 8) {
+          for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 8) {
             uint32_t acc[PP][8];
 #pragma unroll
             for (int q = 0; q < PP; ++q)
               if (p * PP + q < L) tc::tmem_ld8(lane_base + q * BN + c0, acc[q]);
             tc::tmem_wait_ld();
             if (rowok && ok) {
+              float y[8];
 #pragma unroll
               for (int c = 0; c < 8; ++c) {
-                const int col = n0 + c0 + c;
-                if (col < N) {
-                  float y = 0.f;
+                float t = 0.f;
 #pragma unroll
-                  for (int q = 0; q < PP; ++q)
-                    if (p * PP + q < L) y = fmaf(cf[p * PP + q], __uint_as_float(acc[q][c]), y);
-                  y = scalbnf(y, ref + Cfg::PBA + sh.refB[c0 + c] + Cfg::PBB);
-                  float* dst = C + (int64_t)r * N + col;
-                  *dst = p == 0 ? y : *dst + y;
+                for (int q = 0; q < PP; ++q)
+                  if (p * PP + q < L) t = fmaf(phase_const(L, p * PP + q), __uint_as_float(acc[q][c]), t);
+                y[c] = scalbnf(t, ref + Cfg::PBA + sh.refB[c0 + c] + Cfg::PBB);
+              }
+              float* dst = C + (int64_t)r * N + n0 + c0;
+              const bool full8 = n0 + c0 + 8 <= N && ((reinterpret_cast<uintptr_t>(dst) & 15) == 0);
+              if (full8) {
+                float4* d4 = reinterpret_cast<float4*>(dst);
+                float4 a0 = make_float4(y[0], y[1], y[2], y[3]), a1 = make_float4(y[4], y[5], y[6], y[7]);
+                if (p > 0) {
+                  const float4 b0 = d4[0], b1 = d4[1];
+                  a0.x += b0.x; a0.y += b0.y; a0.z += b0.z; a0.w += b0.w;
+                  a1.x += b1.x; a1.y += b1.y; a1.z += b1.z; a1.w += b1.w;
                 }
+                d4[0] = a0;
+                d4[1] = a1;
+              } else {
+#pragma unroll
+                for (int c = 0; c < 8; ++c)
+                  if (n0 + c0 + c < N) dst[c] = p == 0 ? y[c] : dst[c] + y[c];
               }
             }
           }
-          if (!ok) break;
+          if (!ok) return false;
         }
       } else {
         const int st = g % NSB;
@@ -430,48 +470,70 @@ __global__ void __launch_bounds__(288, 1) gemm_tc_kernel(const uint8_t* __restri
           raise_flag(status, CURVEFP_DEV_TIMEOUT);
           sh.abort_flag = 1;
         }
-        if (fail || read_abort(&sh.abort_flag)) break;
-        decode_run<FB, PT>(cw, off, v, vc, mk, true);
+        if (fail || read_abort(&sh.abort_flag)) return false;
+        decode_half<FB, PT>(cw, off, v, vc, mk, true);
         uint8_t* stg = bstage + (size_t)st * Cfg::BSTAGE;
-        if (p == 0) write_b_planes<Cfg, PT, 0>(stg, rloc, v, vc, mk);
-        if (NP > 1 && p == 1) write_b_planes<Cfg, PT, (NP > 1 ? 1 : 0)>(stg, rloc, v, vc, mk);
-        if (NP > 2 && p == 2) write_b_planes<Cfg, PT, (NP > 2 ? 2 : 0)>(stg, rloc, v, vc, mk);
+        if (p == 0) write_b_planes<Cfg, PT, 0>(stg, rloc, half, v, vc, mk);
+        if (NP > 1 && p == 1) write_b_planes<Cfg, PT, (NP > 1 ? 1 : 0)>(stg, rloc, half, v, vc, mk);
+        if (NP > 2 && p == 2) write_b_planes<Cfg, PT, (NP > 2 ? 2 : 0)>(stg, rloc, half, v, vc, mk);
         tc::fence_proxy_async_smem();
         tc::mbar_arrive(&sh.b_full[st]);
       }
+      return true;
+    };
+    // Two register sets of codes, each loaded two steps before it is used and
+    // never copied, so that no register move waits on an in-flight load.
+    uint4 q0, q1;
+    int r0, r1;
+    load(0, q0, r0);
+    load(1, q1, r1);
+    for (int g = 0; g < total; g += 2) {
+      if (!step(g, q0, r0)) break;
+      load(g + 2, q0, r0);
+      if (g + 1 >= total) break;
+      if (!step(g + 1, q1, r1)) break;
+      load(g + 3, q1, r1);
     }
   } else {
     // ------------------------------ MMA issuer -------------------------------
-    if (lane == 0) {
-      const uint64_t bdesc0 = tc::smem_desc(tc::smem_u32(bstage), 128, 256);
-      for (int g = 0; g < total; ++g) {
-        const int p = g / nsub, s = g % nsub;
-        const int abuf = g & 1, st = g % NSB;
-        bool ok = tc::mbar_wait(&sh.a_full[abuf], (g >> 1) & 1);
-        ok = ok && tc::mbar_wait(&sh.b_full[st], (g / NSB) & 1);
-        if (!ok || read_abort(&sh.abort_flag)) {
-          raise_flag(status, CURVEFP_DEV_TIMEOUT);
-          sh.abort_flag = 1;
-          break;
-        }
+    // The whole warp runs the loop; the elected lane issues MMAs and commits.
+    const uint32_t leader = tc::elect_one();
+    const uint64_t bdesc0 = tc::smem_desc(tc::smem_u32(bstage), 128, 256);
+    bool ok = true;
+    for (int g = 0; g < total && ok; ++g) {
+      const int p = g / nsub, s = g % nsub;
+      const int st = g % NSB;
+      ok = __all_sync(0xffffffffu, tc::mbar_wait(&sh.b_full[st], (g / NSB) & 1));
+#pragma unroll
+      for (int ph = 0; ph < 2; ++ph) {
+        const int u = 2 * g + ph, buf = u & (Cfg::NAU - 1);
+        ok = ok && __all_sync(0xffffffffu, tc::mbar_wait(&sh.a_full[buf], (u / Cfg::NAU) & 1));
+        ok = ok && !read_abort(&sh.abort_flag);
+        if (!ok) break;
         tc::fence_after_sync();
-        if (p == 0) issue_pass<Cfg, PT, 0>(tmem, bdesc0, abuf, st, s == 0);
-        if (NP > 1 && p == 1) issue_pass<Cfg, PT, (NP > 1 ? 1 : 0)>(tmem, bdesc0, abuf, st, s == 0);
-        if (NP > 2 && p == 2) issue_pass<Cfg, PT, (NP > 2 ? 2 : 0)>(tmem, bdesc0, abuf, st, s == 0);
-        tc::mma_commit(&sh.a_empty[abuf]);
-        tc::mma_commit(&sh.b_empty[st]);
-        if (s == nsub - 1) tc::mma_commit(&sh.acc_full);
+        if (ph == 0)
+          issue_step<Cfg, PT, 0>(leader, p, tmem, bdesc0, buf, st, s == 0);
+        else
+          issue_step<Cfg, PT, 1>(leader, p, tmem, bdesc0, buf, st, s == 0);
+        tc::mma_commit_if(leader, &sh.a_empty[buf]);
       }
-      // every issued MMA retires before TMEM is released (also on abort)
-      tc::mma_commit(&sh.drain);
-      if (!tc::mbar_wait(&sh.drain, 0)) raise_flag(status, CURVEFP_DEV_TIMEOUT);
+      if (!ok) break;
+      tc::mma_commit_if(leader, &sh.b_empty[st]);
+      if (s == nsub - 1) tc::mma_commit_if(leader, &sh.acc_full);
     }
+    if (!ok && lane == 0) {
+      raise_flag(status, CURVEFP_DEV_TIMEOUT);
+      sh.abort_flag = 1;
+    }
+    // every issued MMA retires before TMEM is released (also on abort)
+    tc::mma_commit_if(leader, &sh.drain);
+    if (!tc::mbar_wait(&sh.drain, 0) && lane == 0) raise_flag(status, CURVEFP_DEV_TIMEOUT);
     __syncwarp();
   }
 
   tc::fence_before_sync();
   __syncthreads();
-  if (warp == 8) {
+  if (warp == Cfg::MMA_WARP) {
     tc::fence_after_sync();
     tc::tmem_dealloc(tmem, 512);
   }
