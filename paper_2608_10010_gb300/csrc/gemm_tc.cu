@@ -205,7 +205,7 @@ __device__ __forceinline__ void k_masks(uint32_t w, uint32_t (&mk)[3]) {
 }
 
 // Lanes of value word v whose curve index is kap (compile-time kap; the
-// compiler folds the three mask terms into 3-input logic operations).
+// compiler folds the mask terms into 3-input logic operations).
 template <int KBITS>
 __device__ __forceinline__ uint32_t plane_of(uint32_t v, const uint32_t (&mk)[3], int kap) {
   uint32_t r = v;
@@ -213,6 +213,21 @@ __device__ __forceinline__ uint32_t plane_of(uint32_t v, const uint32_t (&mk)[3]
   r &= (kap & 2) ? mk[1] : ~mk[1];
   if (KBITS > 2) r &= (kap & 4) ? mk[2] : ~mk[2];
   return r;
+}
+
+// All 2^KBITS planes of a value word: the four products of v with the two
+// low-bit masks are shared, the third bit splits each of them in two.
+template <int KBITS>
+__device__ __forceinline__ void planes_of(uint32_t v, const uint32_t (&mk)[3], uint32_t (&out)[8]) {
+  const uint32_t p0 = v & ~mk[0] & ~mk[1], p1 = v & mk[0] & ~mk[1];
+  const uint32_t p2 = v & ~mk[0] & mk[1], p3 = v & mk[0] & mk[1];
+  if (KBITS > 2) {
+    out[0] = p0 & ~mk[2]; out[1] = p1 & ~mk[2]; out[2] = p2 & ~mk[2]; out[3] = p3 & ~mk[2];
+    out[4] = p0 & mk[2];  out[5] = p1 & mk[2];  out[6] = p2 & mk[2];  out[7] = p3 & mk[2];
+  } else {
+    out[0] = p0; out[1] = p1; out[2] = p2; out[3] = p3;
+    out[4] = out[5] = out[6] = out[7] = 0u;
+  }
 }
 
 // Decode one half of a 32-byte code run (KS/2 codes) of a row: four value
@@ -250,16 +265,22 @@ __device__ __forceinline__ void write_b_planes(uint8_t* stage, int row, int kc, 
   constexpr int KBITS = Fmt<Cfg::FB_>::C;
   const uint32_t core = (uint32_t)((row >> 3) * 256 + kc * 128 + (row & 7) * 16);
 #pragma unroll
-  for (int c = 0; c < 2; ++c)
+  for (int c = 0; c < 2; ++c) {
+    bool any = false;
+#pragma unroll
+    for (int k2 = 0; k2 < Cfg::KB; ++k2) any = any || Cfg::slot(PASS, c, k2) >= 0;
+    if (!any) continue;
+    uint32_t pw[4][8];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) planes_of<KBITS>(c ? vc[q] : v[q], mk[q], pw[q]);
 #pragma unroll
     for (int k2 = 0; k2 < Cfg::KB; ++k2) {
       const int sl = Cfg::slot(PASS, c, k2);
       if (sl < 0) continue;
-      uint32_t o[4];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) o[q] = plane_of<KBITS>(c ? vc[q] : v[q], mk[q], k2);
-      *reinterpret_cast<uint4*>(stage + (size_t)sl * Cfg::PLANE_BYTES + core) = make_uint4(o[0], o[1], o[2], o[3]);
+      *reinterpret_cast<uint4*>(stage + (size_t)sl * Cfg::PLANE_BYTES + core) =
+          make_uint4(pw[0][k2], pw[1][k2], pw[2][k2], pw[3][k2]);
     }
+  }
 }
 
 template <class Cfg, int PT, int PASS, int PH>
@@ -306,8 +327,8 @@ __device__ __forceinline__ float phase_const(int L, int h) {
 template <int FA, int FB, int PT>
 __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(const uint8_t* __restrict__ A, const int8_t* __restrict__ sA,
                                                          const uint8_t* __restrict__ B, const int8_t* __restrict__ sB,
-                                                         int M, int N, int K, int G, float* __restrict__ C,
-                                                         uint32_t* status) {
+                                                         int M, int N, int K, int G, int gshift,
+                                                         float* __restrict__ C, uint32_t* status) {
   using Cfg = TcCfg<FA, FB, PT>;
   constexpr int L = Cfg::L, PP = Cfg::PP, NP = Cfg::NP, BN = Cfg::BN, NSB = Cfg::NSB;
   constexpr int HALF_BYTES = 16;  // bytes of codes per producer thread and step (E5M2); 8 for BF16
@@ -361,11 +382,12 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
     const uint8_t* src = (is_a ? A : B) + (int64_t)r * K + half * (PT == PLANE_E5M2 ? HALF_BYTES : 8);
     const int8_t* srow = (is_a ? sA : sB) + (int64_t)r * nb;
     const int bias = is_a ? Cfg::PBA : Cfg::PBB;
+    auto pass_of = [&](int g) { return (NP > 1 && g >= nsub ? 1 : 0) + (NP > 2 && g >= 2 * nsub ? 1 : 0); };
     auto load = [&](int g, uint4& cw, int& off) {
       cw = make_uint4(0, 0, 0, 0);
       off = 0;
       if (rowok && g < total) {
-        const int s = g % nsub;
+        const int s = g - pass_of(g) * nsub;
         const uint8_t* p = src + (int64_t)s * Cfg::KS;
         if (PT == PLANE_E5M2) {
           cw = __ldg(reinterpret_cast<const uint4*>(p));
@@ -374,31 +396,32 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
           cw.x = t.x;
           cw.y = t.y;
         }
-        off = (int)__ldg(srow + (s * Cfg::KS) / G);  // raw scale: consumed two steps later
+        off = (int)__ldg(srow + (s >> gshift));  // raw scale: consumed two steps later
       }
     };
     const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
     // One pipeline step of this producer thread; false ends the loop (abort).
     auto step = [&](const int g, const uint4 cw, const int raw_scale) -> bool {
       const int off = raw_scale - ref - bias;
-      const int p = g / nsub, s = g % nsub;
+      const int p = pass_of(g), s = g - p * nsub;
       uint32_t v[4], vc[4], mk[4][3];
       if (is_a) {
         decode_half<FA, PT>(cw, off, v, vc, mk, false);
+        uint32_t pl[4][8];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) planes_of<Fmt<FA>::C>(v[c], mk[c], pl[c]);
         bool fail = false;
 #pragma unroll
         for (int ph = 0; ph < 2; ++ph) {
           const int u = 2 * g + ph, buf = u & (Cfg::NAU - 1);
           if (u >= Cfg::NAU) {
-            fail = !tc::mbar_wait(&sh.a_empty[buf], ((u / Cfg::NAU) - 1) & 1);
+            // warp-uniform outcome: the TMEM stores below are warp-collective
+            fail = !__all_sync(0xffffffffu, tc::mbar_wait(&sh.a_empty[buf], ((u / Cfg::NAU) - 1) & 1));
             tc::fence_after_sync();
           }
           if (fail) {
-            raise_flag(status, CURVEFP_DEV_TIMEOUT);
+            if (lane == 0) raise_flag(status, CURVEFP_DEV_TIMEOUT);
             sh.abort_flag = 1;
-          }
-          if (__any_sync(0xffffffffu, fail || read_abort(&sh.abort_flag))) {
-            fail = true;
             return false;
           }
           // plane k1 of the half occupies 8 columns of the unit; this thread's
@@ -407,7 +430,7 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
           for (int j = 0; j < Cfg::APH; ++j) {
             uint32_t reg[4];
 #pragma unroll
-            for (int c = 0; c < 4; ++c) reg[c] = plane_of<Fmt<FA>::C>(v[c], mk[c], ph * Cfg::APH + j);
+            for (int c = 0; c < 4; ++c) reg[c] = pl[c][ph * Cfg::APH + j];
             tc::tmem_st4(lane_base + Cfg::ACOL0 + buf * Cfg::AU_COLS + j * 8 + half * 4, reg);
           }
           tc::tmem_wait_st();
@@ -469,8 +492,8 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
         if (fail) {
           raise_flag(status, CURVEFP_DEV_TIMEOUT);
           sh.abort_flag = 1;
+          return false;
         }
-        if (fail || read_abort(&sh.abort_flag)) return false;
         decode_half<FB, PT>(cw, off, v, vc, mk, true);
         uint8_t* stg = bstage + (size_t)st * Cfg::BSTAGE;
         if (p == 0) write_b_planes<Cfg, PT, 0>(stg, rloc, half, v, vc, mk);
@@ -501,7 +524,7 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
     const uint64_t bdesc0 = tc::smem_desc(tc::smem_u32(bstage), 128, 256);
     bool ok = true;
     for (int g = 0; g < total && ok; ++g) {
-      const int p = g / nsub, s = g % nsub;
+      const int p = (NP > 1 && g >= nsub ? 1 : 0) + (NP > 2 && g >= 2 * nsub ? 1 : 0), s = g - p * nsub;
       const int st = g % NSB;
       ok = __all_sync(0xffffffffu, tc::mbar_wait(&sh.b_full[st], (g / NSB) & 1));
 #pragma unroll
@@ -549,7 +572,9 @@ static cudaError_t launch_tc_t(int G, const uint8_t* a, const int8_t* sa, const 
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg::SMEM);
   if (e != cudaSuccess) return e;
   dim3 grid((unsigned)((N + Cfg::BN - 1) / Cfg::BN), (unsigned)((M + Cfg::BM - 1) / Cfg::BM));
-  kern<<<grid, Cfg::THREADS, Cfg::SMEM, s>>>(a, sa, b, sb, (int)M, (int)N, (int)K, G, c, st);
+  int gshift = 0;  // scale block of step s is s >> gshift (G / KS is a power of two)
+  while ((Cfg::KS << gshift) < G) ++gshift;
+  kern<<<grid, Cfg::THREADS, Cfg::SMEM, s>>>(a, sa, b, sb, (int)M, (int)N, (int)K, G, gshift, c, st);
   return cudaGetLastError();
 }
 
