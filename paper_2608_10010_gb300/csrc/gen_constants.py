@@ -110,6 +110,50 @@ def lut_for(K: int) -> list[int]:
     return out
 
 
+FORMATS = {"E3C3": (3, 3), "E4C3": (4, 3), "E5C2": (5, 2)}
+
+
+def rank_table(E: int, C: int) -> tuple[int, list[int]]:
+    """Rank lookup for the quantizer's fast path, indexed by (binade offset fo,
+    top 7 mantissa bits m7) of the scaled value v = |x| 2^{-a}:
+    binade F = F_z + fo, mantissa bucket [m7 2^16, m7 2^16 + 2^16).
+    Entry = rank below the bucket's threshold | rank at/above it << 8 |
+    threshold's low 16 mantissa bits << 16 (0 and equal ranks if none).
+    Ranks follow the nearest-level rule: 0 below L_nmin/2, saturating at
+    2^{E+C} - 1; at most one decision threshold falls in a bucket."""
+    K = 1 << C
+    B = 1 << (E + C - 1)
+    nmax = B - 1
+    emax = (1 << (E - 1)) - 1
+    fz = (-nmax - K - 1) // K
+    mu_z = mant_threshold_fix(fix_pow2(1, K), False)
+    thr = [midpoint_threshold(k, K) for k in range(K)]
+
+    def rank(F: int, mant: int) -> int:
+        if F < fz or (F == fz and mant < mu_z):
+            return 0
+        j = sum(1 for t in thr if mant >= t)
+        n = K * F + j
+        if n > nmax:
+            return 2 * B - 1
+        return max(n + B, 1)
+
+    nbin = emax - fz + 1
+    out = []
+    for fo in range(nbin):
+        F = fz + fo
+        for m7 in range(128):
+            lo, hi = m7 << 16, (m7 << 16) | 0xFFFF
+            r_lo, r_hi = rank(F, lo), rank(F, hi)
+            cuts = [t for t in thr + [mu_z] if lo < t <= hi and rank(F, t - 1) != rank(F, t)]
+            assert len(cuts) <= 1
+            t16 = (cuts[0] & 0xFFFF) if cuts else 0
+            if not cuts:
+                assert r_lo == r_hi
+            out.append(r_lo | (r_hi << 8) | (t16 << 16))
+    return nbin, out
+
+
 def main(out=sys.stdout):
     w = out.write
     w("/* Generated by gen_constants.py from exact integer arithmetic; do not edit. */\n")
@@ -125,6 +169,13 @@ def main(out=sys.stdout):
             w("  " + ", ".join(f"0x{v:08x}u" for v in lut[i:i + 8]) + ", \\\n")
         w("}\n")
         w(f"#define CFP_CK_F32_K{K}_INIT {{" + ", ".join(f"0x{f32_bits_pow2(k, K):08x}u" for k in range(K)) + "}\n\n")
+    for name, (E, C) in FORMATS.items():
+        nbin, tab = rank_table(E, C)
+        w(f"#define CFP_RANK_{name}_NBIN {nbin}\n")
+        w(f"#define CFP_RANK_{name}_INIT {{ \\\n")
+        for i in range(0, len(tab), 8):
+            w("  " + ", ".join(f"0x{v:08x}u" for v in tab[i:i + 8]) + ", \\\n")
+        w("}\n")
     for L in (4, 8):
         w(f"#define CFP_PHASE_F32_L{L}_INIT {{" + ", ".join(f"0x{f32_bits_pow2(h, L):08x}u" for h in range(L)) + "}\n")
         w(f"#define CFP_PHASE_F64_L{L}_INIT {{" + ", ".join(f"0x{f64_bits_pow2(h, L):016x}ull" for h in range(L)) + "}\n")

@@ -112,27 +112,103 @@ struct Elem<uint16_t> {  // BF16 storage
 };
 
 template <int K>
-__device__ __forceinline__ const uint32_t* lut_src() {
-  return K == 8 ? CFP_LUT_K8_DEV : CFP_LUT_K4_DEV;
+__device__ __forceinline__ const uint32_t* lut_src();
+
+// Rank tables of the fast path, indexed by (binade offset, top 7 mantissa bits)
+// of the scaled value; entry = rank below | rank above << 8 | the in-bucket
+// threshold's low 16 mantissa bits << 16 (generated exactly on the host).
+// (global memory, not __constant__: every thread copies a different entry)
+static __device__ const uint32_t CFP_RANK_E3C3_DEV[CFP_RANK_E3C3_NBIN * 128] = CFP_RANK_E3C3_INIT;
+static __device__ const uint32_t CFP_RANK_E4C3_DEV[CFP_RANK_E4C3_NBIN * 128] = CFP_RANK_E4C3_INIT;
+static __device__ const uint32_t CFP_RANK_E5C2_DEV[CFP_RANK_E5C2_NBIN * 128] = CFP_RANK_E5C2_INIT;
+static __device__ const uint32_t CFP_LUT_K4_G[256] = CFP_LUT_K4_INIT;
+static __device__ const uint32_t CFP_LUT_K8_G[256] = CFP_LUT_K8_INIT;
+
+template <>
+__device__ __forceinline__ const uint32_t* lut_src<4>() {
+  return CFP_LUT_K4_G;
+}
+template <>
+__device__ __forceinline__ const uint32_t* lut_src<8>() {
+  return CFP_LUT_K8_G;
+}
+
+template <int FMT>
+struct RankTab;
+template <>
+struct RankTab<CURVEFP_E3C3> {
+  static constexpr int NBIN = CFP_RANK_E3C3_NBIN;
+  __device__ static const uint32_t* src() { return CFP_RANK_E3C3_DEV; }
+};
+template <>
+struct RankTab<CURVEFP_E4C3> {
+  static constexpr int NBIN = CFP_RANK_E4C3_NBIN;
+  __device__ static const uint32_t* src() { return CFP_RANK_E4C3_DEV; }
+};
+template <>
+struct RankTab<CURVEFP_E5C2> {
+  static constexpr int NBIN = CFP_RANK_E5C2_NBIN;
+  __device__ static const uint32_t* src() { return CFP_RANK_E5C2_DEV; }
+};
+
+// Table key of a magnitude bit pattern (FP32 bits >> 16, or BF16 bits) for
+// block scale a: (binade - F_z) * 128 + top 7 mantissa bits, clamped at 0
+// (everything below binade F_z encodes as zero).  kb = (127 + a + F_z) << 7.
+__device__ __forceinline__ int rank_key(uint32_t hi16, int kb) {
+  const int k = (int)hi16 - kb;
+  return k < 0 ? 0 : k;
+}
+
+// Merge signs into four packed ranks: a sign bit is kept only on nonzero codes
+// (zero is always 0x00).  s4 holds each element's sign in bit 7 of its byte.
+__device__ __forceinline__ uint32_t merge_signs(uint32_t r4, uint32_t s4) {
+  const uint32_t nz = (r4 + 0x7F7F7F7Fu) & 0x80808080u;  // rank >= 1
+  return r4 | (s4 & nz);
+}
+
+__device__ __forceinline__ uint32_t max_u16x2(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("max.u16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
 }
 
 // ---------------------------------------------------------------------------
 // block_axis 0: blocks of G consecutive elements along a row.
 // TPB lanes cooperate on one block; each lane holds VPT 16-byte vectors.
+// Fast path (finite block, scale >= -100): one shared-memory rank lookup per
+// element (BF16: the byte itself; FP32: plus one 16-bit compare), signs merged
+// four at a time.  Other blocks take the exact per-element slow path.
 template <int FMT, typename T, int G>
 __global__ void __launch_bounds__(256) quantize_rows_kernel(const T* __restrict__ x, int64_t rows, int64_t cols,
                                                             int64_t ld, uint8_t* __restrict__ codes,
                                                             int8_t* __restrict__ scales, uint32_t* status) {
   using F = Fmt<FMT>;
   constexpr int VEC = Elem<T>::VEC;
+  constexpr bool BF16 = sizeof(T) == 2;
   constexpr int VPB = G / VEC;              // vectors per block
-  constexpr int TPB = VPB < 8 ? VPB : 8;    // lanes per block
+  // BF16 blocks of 32: two lanes share a block (two 16-byte vectors each), which
+  // keeps every load instruction on whole 32-byte sectors while halving the
+  // per-block work (one shuffle, the scale computed by two lanes); otherwise up
+  // to 8 lanes share a block
+  constexpr int TPB = (BF16 && G == 32) ? 2 : (VPB < 8 ? VPB : 8);  // lanes per block
   constexpr int VPT = VPB / TPB;            // vectors per lane
   constexpr int BPW = 32 / TPB;             // blocks per warp step
   constexpr int UNROLL = VPT >= 4 ? 1 : 4 / VPT;
+  constexpr int NTAB = RankTab<FMT>::NBIN * 128;
 
   __shared__ uint32_t lut[256];
-  for (int i = threadIdx.x; i < 256; i += blockDim.x) lut[i] = lut_src<F::K>()[i];
+  // FP32: full entries; BF16: the low byte of each entry only (its low 16
+  // mantissa bits are zero, so the in-bucket compare never fires)
+  __shared__ __align__(16) uint32_t tab[BF16 ? 1 : NTAB];
+  __shared__ __align__(16) uint8_t tab8[BF16 ? NTAB : 1];
+  for (int i = threadIdx.x; i < 256; i += blockDim.x) lut[i] = __ldg(lut_src<F::K>() + i);
+  for (int i = threadIdx.x; i < NTAB; i += blockDim.x) {
+    const uint32_t e = __ldg(RankTab<FMT>::src() + i);
+    if (BF16)
+      tab8[i] = (uint8_t)(e & 0xFFu);
+    else
+      tab[i] = e;
+  }
   __syncthreads();
 
   const int lane = threadIdx.x & 31;
@@ -162,9 +238,18 @@ __global__ void __launch_bounds__(256) quantize_rows_kernel(const T* __restrict_
       // max |x| over the block as an unsigned bit pattern (NaN sorts above Inf)
       uint32_t mx = 0u;
 #pragma unroll
-      for (int q = 0; q < VPT; ++q)
+      for (int q = 0; q < VPT; ++q) {
+        const uint32_t w[4] = {v[u][q].x, v[u][q].y, v[u][q].z, v[u][q].w};
+        if (BF16) {
+          uint32_t m2 = 0u;
 #pragma unroll
-        for (int i = 0; i < VEC; ++i) mx = max(mx, Elem<T>::bits(v[u][q], i) & 0x7FFFFFFFu);
+          for (int i = 0; i < 4; ++i) m2 = max_u16x2(m2, w[i] & 0x7FFF7FFFu);
+          mx = max(mx, max(m2 & 0xFFFFu, m2 >> 16) << 16);
+        } else {
+#pragma unroll
+          for (int i = 0; i < 4; ++i) mx = max(mx, w[i] & 0x7FFFFFFFu);
+        }
+      }
 #pragma unroll
       for (int o = TPB / 2; o > 0; o >>= 1) mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
       const bool ok = blk[u] < nblk;
@@ -186,25 +271,52 @@ __global__ void __launch_bounds__(256) quantize_rows_kernel(const T* __restrict_
       if (!ok) continue;
       uint8_t* dst = codes + blk[u] * G;
       if (sub == 0) scales[blk[u]] = (int8_t)a;
-      const int32_t ashift = a * (1 << 23);
+      const int kb = (127 + a + ZeroBoundary<FMT>::FZ) << 7;
 #pragma unroll
       for (int q = 0; q < VPT; ++q) {
-        uint32_t c[VEC];
+        const uint32_t w[4] = {v[u][q].x, v[u][q].y, v[u][q].z, v[u][q].w};
+        uint8_t* d = dst + (q * TPB + sub) * VEC;
         if (fast) {
+          if (BF16) {
+            // two keys per word: clamp each 16-bit magnitude at kb with a
+            // SIMD max, then one 32-bit subtract (no lane can borrow)
+            const uint32_t kb2 = (uint32_t)kb * 0x00010001u;
+            uint32_t out[2];
 #pragma unroll
-          for (int i = 0; i < VEC; ++i) c[i] = encode_fast<FMT>(lut, Elem<T>::bits(v[u][q], i), ashift);
+            for (int h = 0; h < 2; ++h) {
+              const uint32_t w0 = w[2 * h], w1 = w[2 * h + 1];
+              const uint32_t k0 = max_u16x2(w0 & 0x7FFF7FFFu, kb2) - kb2;
+              const uint32_t k1 = max_u16x2(w1 & 0x7FFF7FFFu, kb2) - kb2;
+              const uint32_t r0 = tab8[k0 & 0xFFFFu], r1 = tab8[k0 >> 16];
+              const uint32_t r2 = tab8[k1 & 0xFFFFu], r3 = tab8[k1 >> 16];
+              const uint32_t r4 = __byte_perm(__byte_perm(r0, r1, 0x0040), __byte_perm(r2, r3, 0x0040), 0x5410);
+              out[h] = merge_signs(r4, __byte_perm(w0, w1, 0x7531));
+            }
+            *reinterpret_cast<uint2*>(d) = make_uint2(out[0], out[1]);
+          } else {
+            uint32_t r[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const uint32_t ab = w[i] & 0x7FFFFFFFu;
+              const uint32_t e = tab[max(ab >> 16, (uint32_t)kb) - (uint32_t)kb];
+              r[i] = ((ab & 0xFFFFu) >= (e >> 16)) ? ((e >> 8) & 0xFFu) : (e & 0xFFu);
+            }
+            const uint32_t r4 = r[0] | (r[1] << 8) | (r[2] << 16) | (r[3] << 24);
+            const uint32_t s4 = __byte_perm(__byte_perm(w[0], w[1], 0x0073), __byte_perm(w[2], w[3], 0x7300), 0x7610);
+            *reinterpret_cast<uint32_t*>(d) = merge_signs(r4, s4);
+          }
         } else {
+          uint32_t c[VEC];
 #pragma unroll
           for (int i = 0; i < VEC; ++i) c[i] = encode_slow<FMT>(lut, Elem<T>::bits(v[u][q], i), a, saw_nan);
-        }
-        uint8_t* d = dst + (q * TPB + sub) * VEC;
-        if (VEC == 4) {
-          *reinterpret_cast<uint32_t*>(d) = c[0] | (c[1] << 8) | (c[2] << 16) | (c[3] << 24);
-        } else {
-          uint2 w;
-          w.x = c[0] | (c[1] << 8) | (c[2] << 16) | (c[3] << 24);
-          w.y = c[4] | (c[5] << 8) | (c[6] << 16) | (c[7] << 24);
-          *reinterpret_cast<uint2*>(d) = w;
+          if (VEC == 4) {
+            *reinterpret_cast<uint32_t*>(d) = c[0] | (c[1] << 8) | (c[2] << 16) | (c[3] << 24);
+          } else {
+            uint2 wv;
+            wv.x = c[0] | (c[1] << 8) | (c[2] << 16) | (c[3] << 24);
+            wv.y = c[4] | (c[5] << 8) | (c[6] << 16) | (c[7] << 24);
+            *reinterpret_cast<uint2*>(d) = wv;
+          }
         }
       }
     }
@@ -223,7 +335,7 @@ __global__ void __launch_bounds__(256) quantize_cols_kernel(const T* __restrict_
                                                             int8_t* __restrict__ scales, uint32_t* status) {
   using F = Fmt<FMT>;
   __shared__ uint32_t lut[256];
-  for (int i = threadIdx.x; i < 256; i += blockDim.x) lut[i] = lut_src<F::K>()[i];
+  for (int i = threadIdx.x; i < 256; i += blockDim.x) lut[i] = __ldg(lut_src<F::K>() + i);
   __syncthreads();
   const int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   const int64_t rb = blockIdx.y;
@@ -338,7 +450,7 @@ static cudaError_t launch_q(const void* x, int64_t rows, int64_t cols, int64_t l
                             int8_t* scales, uint32_t* status, cudaStream_t st, int sms) {
   if (axis == 0) {
     constexpr int VEC = Elem<T>::VEC;
-    constexpr int TPB = (G / VEC) < 8 ? (G / VEC) : 8;
+    constexpr int TPB = (sizeof(T) == 2 && G == 32) ? 2 : ((G / VEC) < 8 ? (G / VEC) : 8);
     const int64_t nblk = rows * (cols / G);
     constexpr int VPT = (G / VEC) / TPB;
     constexpr int PER_WARP = (32 / TPB) * (VPT >= 4 ? 1 : 4 / VPT);
