@@ -37,6 +37,11 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 M, N, K, G = 2048, 4096, 4096, 32
+# DRAM bytes (read + written) of one launch of the tensor-core GEMM at this
+# size, from an ncu capture (dram__bytes_read.sum + dram__bytes_write.sum) of
+# the kernel as it stands; set to None whenever the kernel changes until it is
+# captured again.
+GEMM_DRAM_TRAFFIC = 26_021_888 + 2_540_800
 FMT = "E3C3"
 WORKLOAD = "E3C3 Llama-7B-like linear: X[2048x4096] (1% outlier channels x20) . W[4096x4096]^T, block 32"
 METRIC = "CurveFP GEMM TOPS & quantize GB/s at 1 GB300, as % of roofline"
@@ -305,7 +310,8 @@ def run_ours(args):
                    "l2": "flushed between steps (256 MiB write + 256 MiB read, outside the per-step events)",
                    "parallelism": f"replicas x{ws}"},
         "roofline": {"bound": "tensor", "achieved": round(gemm_tops, 4), "peak": round(fp8_peak, 1),
-                     "unit": "TFLOP/s", "frac": round(gemm_tops / fp8_peak, 6), "traffic": None,
+                     "unit": "TFLOP/s", "frac": round(gemm_tops / fp8_peak, 6), "traffic": GEMM_DRAM_TRAFFIC,
+                     "bytes_algorithmic": M * K + N * K + (M + N) * K // G + 4 * M * N,
                      "peak_source": f"FP8 dense = 2 x bf16 burst ({bf16} TFLOP/s, {peak_src})",
                      "kernel": "gemm_tc_kernel (tcgen05 kind::f8f6f4, E5M2 curve planes)",
                      "tensor_work_frac": round(gemm_tops * planes / fp8_peak, 4),
