@@ -16,25 +16,36 @@
 // BF16 or FP8 E5M2 (every power of two in [2^-16, 2^15] is exact in E5M2; E5C2
 // planes are stored one binade low so that the carry still fits).
 //
-// Shape.  A CTA owns a 128 x 128 tile of C.  tcgen05.mma runs at full rate
-// only for N >= 128, and TMEM (512 columns) holds three 128-column phase
-// accumulators plus two A stages, so the L phases are processed in passes of
-// PP = 3 phases over the whole K; each pass adds its part of
-// sum_h 2^{h/L} S_h into C.
+// Shape.  A CTA owns a 128 x 96 tile of C.  A 128 x 96 x 32 FP8 MMA runs at
+// the full tensor rate (the per-instruction floor is ~45 cycles, this shape
+// takes 48); TMEM (512 columns) holds four 96-column phase accumulators plus
+// two steps of A planes, so the L phases are processed in passes of PP = 4
+// phases over the whole K; each pass adds its part of sum_h 2^{h/L} S_h to C.
 //
-// Roles (544 threads; every 32-byte run of codes of a row is split between
-// two producer threads so that each SM sub-partition has several producer
-// warps to hide latency):
-//   warps 0-7  A producers: codes -> planes in registers -> TMEM (tcgen05.st);
-//              A is the TMEM operand of the MMA and costs no shared-memory
-//              bandwidth.  At the end of each pass they run the epilogue.
-//   warps 8-15 B producers: codes -> the planes (and x2 carry planes) that the
-//              current pass needs -> shared memory, K-major core-matrix layout.
-//   warp 16    TMEM allocation and the single MMA-issuing thread.
-// mbarriers hand stages between the roles; every wait is bounded.
+// Roles (480 threads):
+//   warps 0-7   A producers (two threads per row, 16 codes each per step):
+//               codes -> planes in registers -> TMEM (tcgen05.st); A is the
+//               TMEM operand of the MMA and costs no shared-memory bandwidth.
+//               At the end of each pass they run the epilogue.
+//   warps 8-13  B producers (two threads per row): codes -> the planes (and
+//               x2 carry planes) that the current pass needs -> shared memory,
+//               K-major core-matrix layout.
+//   warp 14     TMEM allocation and MMA issue (one elected lane of the
+//               converged warp).
+// One mbarrier hand-off per pipeline step and operand: every wait and commit
+// sits on the path between two MMAs, so the stages are whole steps.  Every
+// wait is bounded.
 #include "cfp_common.cuh"
 #include "kernels.cuh"
 #include "tc_ptx.cuh"
+
+#ifndef CFP_TC_ATPR
+#define CFP_TC_ATPR 2  // A producer threads per row (2 or 4)
+#endif
+
+#ifndef CFP_TC_UPS
+#define CFP_TC_UPS 1  // A staging units per pipeline step (1, 2 or 4)
+#endif
 
 #ifndef CFP_TC_PLANE
 #define CFP_TC_PLANE 1  // 0: BF16 planes (K = 16 per MMA), 1: E5M2 planes (K = 32 per MMA)
@@ -60,20 +71,26 @@ struct TcCfg {
   static constexpr int PP = 4;                            // phases per pass
   static constexpr int NP = (L + PP - 1) / PP;            // passes
   static constexpr int ACC_COLS = PP * BN;
-  // A is staged in half-steps ("units"): unit 2g + ph holds planes
-  // [ph APH, (ph + 1) APH) of step g, 8 TMEM columns per plane; NAU units rotate.
-  static constexpr int APH = KA / 2;
+  // A is staged in units of APH planes: unit UPS g + ph holds planes
+  // [ph APH, (ph + 1) APH) of step g, 8 TMEM columns per plane; NAU units
+  // (two steps) rotate.
+  static constexpr int UPS = CFP_TC_UPS < KA ? CFP_TC_UPS : KA;  // units per step
+  static constexpr int APH = KA / UPS;                              // planes per unit
   static constexpr int AU_COLS = APH * 8;
-  static constexpr int NAU = 4;
+  static constexpr int NAU = 2 * UPS;                               // two steps in flight
   static constexpr int ACOL0 = ACC_COLS;
   static_assert(ACC_COLS + NAU * AU_COLS <= 512, "TMEM budget");
   static constexpr int PLANE_BYTES = BN * 32;             // 128 rows x 32 bytes
   static constexpr int NSB = 4;                           // B stages
   static constexpr int PBA = FA == CURVEFP_E5C2 ? 1 : 0;  // plane exponent bias
   static constexpr int PBB = FB == CURVEFP_E5C2 ? 1 : 0;
+  static constexpr int ATPR = CFP_TC_ATPR;                // A producer threads per row
+  static constexpr int NAW = 4 * ATPR;                    // A producer warps (4 TMEM lane groups)
+  static constexpr int NWA = 8 / ATPR;                    // TMEM columns per A thread and plane
   static constexpr int NBT = 2 * BN;                      // B producer threads (two per row)
-  static constexpr int THREADS = 256 + NBT + 32;          // A producers, B producers, MMA warp
-  static constexpr int MMA_WARP = (256 + NBT) / 32;
+  static constexpr int THREADS = NAW * 32 + NBT + 32;     // A producers, B producers, MMA warp
+  static constexpr int MMA_WARP = (NAW * 32 + NBT) / 32;
+  static_assert(NBT % 32 == 0 && BN % (8 * ATPR) == 0 && 8 % ATPR == 0, "producer warps");
   // D = F32, A = B = BF16 (kind::f16) or E5M2 (kind::f8f6f4): same bit pattern
   static constexpr uint32_t IDESC = tc::idesc_bf16_f32(BM, BN);
 
@@ -119,8 +136,10 @@ struct TcCfg {
   static constexpr size_t SMEM = (size_t)NSB * BSTAGE + 2048;
 };
 
+constexpr int TC_MAX_RING = 8;  // capacity of the barrier rings below (>= NAU, NSB)
+
 struct TcShared {
-  uint64_t a_full[4], a_empty[4], b_full[4], b_empty[4], acc_full, drain;
+  uint64_t a_full[TC_MAX_RING], a_empty[TC_MAX_RING], b_full[TC_MAX_RING], b_empty[TC_MAX_RING], acc_full, drain;
   uint32_t tmem_base;
   int abort_flag;
   int refB[128];  // >= BN
@@ -137,40 +156,67 @@ __device__ __forceinline__ int read_abort(const int* f) { return *reinterpret_ca
 // A code byte is s | m with m = e_b K + k (e_b = e + 2^{E-1}, App. C.1), so
 //   k   = the low C bits,  e_b = the next E bits,  s = bit 7.
 // Plane value +-2^{x}, x = e_b - 2^{E-1} + off (off = block scale - row
-// reference - plane bias; +1 for a carry plane):
-//   E5M2:  byte (x + 15) << 2 for x >= -14 (smaller values flush to zero:
-//          they sit 2^14 below the row's largest element);
-//   BF16:  half (x + 127) << 7 for x >= -126.
-// The test "x is representable" is done with a guard bit: per lane
-// u = e_b + c + (bias) has its top bit set exactly when the value is kept, so
-// no lane borrows from its neighbour.
+// reference - plane bias).  An element is kept when x >= -14 (E5M2 normal
+// range; smaller elements sit 2^14 below the row's largest element and flush
+// to zero) or x >= -126 (BF16); its carry-plane copy is 2^{x+1}, which still
+// fits (x <= 2^{E-1} - 1 - bias, so x + 1 + 15 <= 30).
+//   E5M2:  byte s | (x + 15) << 2;   BF16:  half s | (x + 127) << 7.
+// "Kept" is a threshold on the rank: e_b >= T  <=>  m >= max(K T, 1) = mt
+// (m != 0 excludes the zero code), so bit 7 of m + (128 - mt) is the keep bit
+// of each lane (m <= 127 and 128 - mt <= 127: no carry into the next lane).
 
-// Per-byte 0xFF where the lane's top bit (bit 7) is set.
-__device__ __forceinline__ uint32_t byte_mask_from_bit7(uint32_t v7) { return ((v7 >> 7) & 0x01010101u) * 0xFFu; }
-__device__ __forceinline__ uint32_t half_mask_from_bit15(uint32_t v15) {
-  return ((v15 >> 15) & 0x00010001u) * 0xFFFFu;
+// prmt with sign replication: byte i of the result is 0xFF where bit 7 of
+// byte sel_i of v is set (selector nibbles 8..B pick bytes 0..3 with the sign
+// mode).
+__device__ __forceinline__ uint32_t prmt_sign(uint32_t v, uint32_t sel) {
+  uint32_t r;
+  asm("prmt.b32 %0, %1, 0, %2;" : "=r"(r) : "r"(v), "r"(sel));
+  return r;
 }
 
 template <int FMT>
 struct CodeBits {
   using F = Fmt<FMT>;
-  static constexpr uint32_t MM = F::MMASK * 0x01010101u;             // rank bits
-  static constexpr uint32_t EBM = ((1u << F::E) - 1u) * 0x01010101u;  // e_b bits after >> C
+  static constexpr uint32_t MM = F::MMASK * 0x01010101u;                    // rank bits
+  static constexpr uint32_t EB2 = (((1u << F::E) - 1u) << 2) * 0x01010101u;  // e_b << 2 after >> (C - 2)
 };
 
-// E5M2 plane bytes of four codes for exponent offset off (c = 15 - 2^{E-1} + off).
+// Per-step constants of a producer thread's block for E5M2 planes.
+struct E5Const {
+  uint32_t kt;  // per lane 128 - mt
+  uint32_t kp;  // per lane 4 max(c5, 0)
+  uint32_t km;  // per lane 4 max(-c5, 0)
+};
+
 template <int FMT>
-__device__ __forceinline__ uint32_t e5m2_word(uint32_t w, int off) {
+__device__ __forceinline__ E5Const e5_const(int off) {
   using F = Fmt<FMT>;
-  int c = 15 - (1 << (F::E - 1)) + off;
-  c = c < -127 ? -127 : c;                                  // everything flushes
+  const int t = (1 << (F::E - 1)) - 14 - off;  // smallest kept e_b
+  int mt = t * F::K;
+  mt = mt < 1 ? 1 : (mt > 128 ? 128 : mt);
+  // exponent field e5 = x + 15 = e_b + c5; when nothing is kept (mt = 128)
+  // c5 is clamped so that the lane arithmetic below stays inside its byte
+  int c5 = 15 - (1 << (F::E - 1)) + off;
+  c5 = c5 < -30 ? -30 : c5;
+  E5Const k;
+  k.kt = (uint32_t)(128 - mt) * 0x01010101u;
+  k.kp = (uint32_t)(4 * (c5 > 0 ? c5 : 0)) * 0x01010101u;
+  k.km = (uint32_t)(4 * (c5 < 0 ? -c5 : 0)) * 0x01010101u;
+  return k;
+}
+
+// E5M2 plane bytes of four codes and the lane keep mask.  The exponent byte
+// is formed as (e_b << 2 | 0x80) + 4 max(c5,0) - 4 max(-c5,0): the guard bit
+// 0x80 absorbs the subtraction (4 max(-c5,0) <= 120) and the addition stays
+// below 256 (e5 <= 31), so no lane borrows from or carries into a neighbour.
+template <int FMT>
+__device__ __forceinline__ uint32_t e5m2_word(uint32_t w, const E5Const& k, uint32_t& keep) {
+  using F = Fmt<FMT>;
   const uint32_t m4 = w & CodeBits<FMT>::MM;
-  const uint32_t eb4 = (w >> F::C) & CodeBits<FMT>::EBM;
-  const uint32_t u4 = eb4 + (uint32_t)(c + 127) * 0x01010101u;  // bit 7 <=> x >= -14
-  const uint32_t nz = m4 + 0x7F7F7F7Fu;                          // bit 7 <=> m != 0
-  const uint32_t keep = byte_mask_from_bit7(u4 & nz & 0x80808080u);
-  const uint32_t t = ((u4 & 0x7F7F7F7Fu) + 0x01010101u) & keep;  // x + 15 where kept
-  return (t << 2) | (w & 0x80808080u & keep);
+  keep = prmt_sign(m4 + k.kt, 0xBA98u);
+  const uint32_t eb = ((w >> (F::C - 2)) & CodeBits<FMT>::EB2) | 0x80808080u;
+  const uint32_t x = eb + k.kp - k.km;
+  return ((w & 0x80808080u) | (x & 0x7F7F7F7Fu)) & keep;
 }
 
 // BF16 plane halves of two codes (bytes 0 and 1 of w2 = codes c0 | c1 << 16).
@@ -184,35 +230,22 @@ __device__ __forceinline__ uint32_t bf16_word(uint32_t w2, int off) {
   const uint32_t eb2 = (w2 >> F::C) & EB2;
   const uint32_t u2 = eb2 + (uint32_t)(c - 1 + 0x8000) * 0x00010001u;  // bit 15 <=> e_b + c >= 1
   const uint32_t nz = m2 + 0x7FFF7FFFu;                                 // bit 15 <=> m != 0
-  const uint32_t keep = half_mask_from_bit15(u2 & nz & 0x80008000u);
+  const uint32_t keep = prmt_sign(u2 & nz & 0x80008000u, 0xBB99u);
   const uint32_t t = ((u2 & 0x7FFF7FFFu) + 0x00010001u) & keep;       // biased exponent where kept
   return (t << 7) | ((w2 & 0x00800080u & keep) << 8);
 }
 
-// Masks of the curve-index bits (0xFF / 0xFFFF per lane where bit b of k is 1).
+// Masks of the curve-index bits (0xFF / 0xFFFF per lane where bit b of k is 1):
+// shift bit b of every lane's low byte to bit 7, then replicate it.
 template <int PT, int KBITS>
 __device__ __forceinline__ void k_masks(uint32_t w, uint32_t (&mk)[3]) {
 #pragma unroll
   for (int b = 0; b < 3; ++b) {
-    if (b >= KBITS) {
+    if (b >= KBITS)
       mk[b] = 0u;
-    } else if (PT == PLANE_E5M2) {
-      mk[b] = ((w >> b) & 0x01010101u) * 0xFFu;
-    } else {
-      mk[b] = ((w >> b) & 0x00010001u) * 0xFFFFu;
-    }
+    else
+      mk[b] = prmt_sign(w << (7 - b), PT == PLANE_E5M2 ? 0xBA98u : 0xAA88u);
   }
-}
-
-// Lanes of value word v whose curve index is kap (compile-time kap; the
-// compiler folds the mask terms into 3-input logic operations).
-template <int KBITS>
-__device__ __forceinline__ uint32_t plane_of(uint32_t v, const uint32_t (&mk)[3], int kap) {
-  uint32_t r = v;
-  r &= (kap & 1) ? mk[0] : ~mk[0];
-  r &= (kap & 2) ? mk[1] : ~mk[1];
-  if (KBITS > 2) r &= (kap & 4) ? mk[2] : ~mk[2];
-  return r;
 }
 
 // All 2^KBITS planes of a value word: the four products of v with the two
@@ -230,26 +263,27 @@ __device__ __forceinline__ void planes_of(uint32_t v, const uint32_t (&mk)[3], u
   }
 }
 
-// Decode one half of a 32-byte code run (KS/2 codes) of a row: four value
-// words in the order the MMA operands expect along K (word w holds elements
-// 4w..4w+3 as E5M2 bytes, or 2w..2w+1 as BF16 halves), the x2 carry words if
-// asked, and the curve-index masks of every word.
-template <int FMT, int PT>
-__device__ __forceinline__ void decode_half(const uint4& cw, int off, uint32_t (&v)[4], uint32_t (&vc)[4],
-                                            uint32_t (&mk)[4][3], bool want_carry) {
+// Decode a thread's share of a row's 32-byte plane run: NW value words in the
+// order the MMA operands expect along K (word w holds elements 4w..4w+3 as
+// E5M2 bytes, or 2w..2w+1 as BF16 halves), the x2 carry words if asked, and
+// the curve-index masks of every word.
+template <int FMT, int PT, int NW>
+__device__ __forceinline__ void decode_words(const uint4& cw, int off, uint32_t (&v)[NW], uint32_t (&vc)[NW],
+                                             uint32_t (&mk)[NW][3], bool want_carry) {
   constexpr int KBITS = Fmt<FMT>::C;
+  const uint32_t w[4] = {cw.x, cw.y, cw.z, cw.w};
   if (PT == PLANE_E5M2) {
-    const uint32_t w[4] = {cw.x, cw.y, cw.z, cw.w};
+    const E5Const k = e5_const<FMT>(off);
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      v[i] = e5m2_word<FMT>(w[i], off);
-      vc[i] = want_carry ? e5m2_word<FMT>(w[i], off + 1) : 0u;
+    for (int i = 0; i < NW; ++i) {
+      uint32_t keep;
+      v[i] = e5m2_word<FMT>(w[i], k, keep);
+      vc[i] = want_carry ? v[i] + (keep & 0x04040404u) : 0u;  // exponent + 1
       k_masks<PT, KBITS>(w[i], mk[i]);
     }
   } else {
-    const uint32_t w[2] = {cw.x, cw.y};
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
+    for (int i = 0; i < NW; ++i) {
       const uint32_t w2 = __byte_perm(w[i >> 1], 0u, (i & 1) ? 0x4342u : 0x4140u);
       v[i] = bf16_word<FMT>(w2, off);
       vc[i] = want_carry ? bf16_word<FMT>(w2, off + 1) : 0u;
@@ -320,10 +354,11 @@ __device__ __forceinline__ float phase_const(int L, int h) {
 
 }  // namespace
 
-// Thread layout: warps 0-7 produce A (warp w: TMEM lane group w & 3, half
-// w >> 2 of each 32-byte run) and run the epilogue (columns [BN/2 half,
-// BN/2 (half + 1))); the next 2 BN threads produce B (thread 256 + t: row
-// t % BN, half t / BN); the last warp allocates TMEM and issues the MMAs.
+// Thread layout: warps 0 .. NAW-1 produce A (warp w: TMEM lane group w & 3,
+// share w >> 2 of each 32-byte run: NWA columns per plane) and run the
+// epilogue (columns [BN/ATPR share, BN/ATPR (share + 1))); the next 2 BN
+// threads produce B (thread 32 NAW + t: row t % BN, half t / BN); the last
+// warp allocates TMEM and issues the MMAs.
 template <int FA, int FB, int PT>
 __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(const uint8_t* __restrict__ A, const int8_t* __restrict__ sA,
                                                          const uint8_t* __restrict__ B, const int8_t* __restrict__ sB,
@@ -331,8 +366,10 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
                                                          float* __restrict__ C, uint32_t* status) {
   using Cfg = TcCfg<FA, FB, PT>;
   constexpr int L = Cfg::L, PP = Cfg::PP, NP = Cfg::NP, BN = Cfg::BN, NSB = Cfg::NSB;
-  constexpr int HALF_BYTES = 16;  // bytes of codes per producer thread and step (E5M2); 8 for BF16
+  constexpr int NAW = Cfg::NAW, NWA = Cfg::NWA, ATPR = Cfg::ATPR;
+  constexpr int CB = PT == PLANE_E5M2 ? 4 : 2;  // code bytes per TMEM column / value word
   static_assert(NP <= 3, "pass dispatch");
+  static_assert(Cfg::NAU <= TC_MAX_RING && NSB <= TC_MAX_RING, "barrier rings");
   extern __shared__ __align__(1024) uint8_t smem[];
   uint8_t* bstage = smem;
   TcShared& sh = *reinterpret_cast<TcShared*>(smem + (size_t)NSB * Cfg::BSTAGE);
@@ -343,11 +380,11 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
 
   if (tid == 0) {
     for (int s = 0; s < Cfg::NAU; ++s) {
-      tc::mbar_init(&sh.a_full[s], 256);
+      tc::mbar_init(&sh.a_full[s], NAW);  // one arrival per producer warp
       tc::mbar_init(&sh.a_empty[s], 1);
     }
     for (int s = 0; s < NSB; ++s) {
-      tc::mbar_init(&sh.b_full[s], Cfg::NBT);
+      tc::mbar_init(&sh.b_full[s], Cfg::NBT / 32);
       tc::mbar_init(&sh.b_empty[s], 1);
     }
     tc::mbar_init(&sh.acc_full, 1);
@@ -359,19 +396,31 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
     tc::tmem_relinquish();
   }
   // producer geometry and the row's reference exponent (largest block scale)
-  const bool is_a = warp < 8;
+  const bool is_a = warp < NAW;
   const bool is_prod = warp < Cfg::MMA_WARP;
-  const int rloc = is_a ? ((warp & 3) * 32 + lane) : ((tid - 256) % BN);
-  const int half = is_a ? (warp >> 2) : ((tid - 256) / BN);
+  const int rloc = is_a ? ((warp & 3) * 32 + lane) : ((tid - NAW * 32) % BN);
+  const int part = is_a ? (warp >> 2) : ((tid - NAW * 32) / BN);  // share of the 32-byte run
   const int r = (is_a ? m0 : n0) + rloc;
   const bool rowok = is_prod && r < (is_a ? M : N);
   int ref = -128;
   if (rowok) {
     const int8_t* s = (is_a ? sA : sB) + (int64_t)r * nb;
+    if ((nb & 15) == 0 && (reinterpret_cast<uintptr_t>(s) & 15) == 0) {
+      // 16 scales per load, all loads in flight at once, byte-wise signed max
+      uint32_t m4 = 0x80808080u;
 #pragma unroll 8
-    for (int b = 0; b < nb; ++b) ref = max(ref, (int)__ldg(s + b));
+      for (int b = 0; b < nb; b += 16) {
+        const uint4 q = __ldg(reinterpret_cast<const uint4*>(s + b));
+        m4 = __vmaxs4(m4, __vmaxs4(__vmaxs4(q.x, q.y), __vmaxs4(q.z, q.w)));
+      }
+      ref = max(max((int)(int8_t)(m4 & 0xFF), (int)(int8_t)((m4 >> 8) & 0xFF)),
+                max((int)(int8_t)((m4 >> 16) & 0xFF), (int)(int8_t)(m4 >> 24)));
+    } else {
+#pragma unroll 8
+      for (int b = 0; b < nb; ++b) ref = max(ref, (int)__ldg(s + b));
+    }
   }
-  if (!is_a && is_prod && half == 0) sh.refB[rloc] = ref;
+  if (!is_a && is_prod && part == 0) sh.refB[rloc] = ref;
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
@@ -379,7 +428,7 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
 
   if (is_prod) {
     // ------------------------------ producers ------------------------------
-    const uint8_t* src = (is_a ? A : B) + (int64_t)r * K + half * (PT == PLANE_E5M2 ? HALF_BYTES : 8);
+    const uint8_t* src = (is_a ? A : B) + (int64_t)r * K + part * (is_a ? NWA : 4) * CB;
     const int8_t* srow = (is_a ? sA : sB) + (int64_t)r * nb;
     const int bias = is_a ? Cfg::PBA : Cfg::PBB;
     auto pass_of = [&](int g) { return (NP > 1 && g >= nsub ? 1 : 0) + (NP > 2 && g >= 2 * nsub ? 1 : 0); };
@@ -389,12 +438,15 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
       if (rowok && g < total) {
         const int s = g - pass_of(g) * nsub;
         const uint8_t* p = src + (int64_t)s * Cfg::KS;
-        if (PT == PLANE_E5M2) {
+        const int nbytes = (is_a ? NWA : 4) * CB;  // 16, 8 or 4
+        if (nbytes == 16) {
           cw = __ldg(reinterpret_cast<const uint4*>(p));
-        } else {
+        } else if (nbytes == 8) {
           const uint2 t = __ldg(reinterpret_cast<const uint2*>(p));
           cw.x = t.x;
           cw.y = t.y;
+        } else {
+          cw.x = __ldg(reinterpret_cast<const uint32_t*>(p));
         }
         off = (int)__ldg(srow + (s >> gshift));  // raw scale: consumed two steps later
       }
@@ -404,16 +456,16 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
     auto step = [&](const int g, const uint4 cw, const int raw_scale) -> bool {
       const int off = raw_scale - ref - bias;
       const int p = pass_of(g), s = g - p * nsub;
-      uint32_t v[4], vc[4], mk[4][3];
       if (is_a) {
-        decode_half<FA, PT>(cw, off, v, vc, mk, false);
-        uint32_t pl[4][8];
+        uint32_t v[NWA], vc[NWA], mk[NWA][3];
+        decode_words<FA, PT, NWA>(cw, off, v, vc, mk, false);
+        uint32_t pl[NWA][8];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) planes_of<Fmt<FA>::C>(v[c], mk[c], pl[c]);
+        for (int c = 0; c < NWA; ++c) planes_of<Fmt<FA>::C>(v[c], mk[c], pl[c]);
         bool fail = false;
 #pragma unroll
-        for (int ph = 0; ph < 2; ++ph) {
-          const int u = 2 * g + ph, buf = u & (Cfg::NAU - 1);
+        for (int ph = 0; ph < Cfg::UPS; ++ph) {
+          const int u = Cfg::UPS * g + ph, buf = u & (Cfg::NAU - 1);
           if (u >= Cfg::NAU) {
             // warp-uniform outcome: the TMEM stores below are warp-collective
             fail = !__all_sync(0xffffffffu, tc::mbar_wait(&sh.a_empty[buf], ((u / Cfg::NAU) - 1) & 1));
@@ -424,18 +476,21 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
             sh.abort_flag = 1;
             return false;
           }
-          // plane k1 of the half occupies 8 columns of the unit; this thread's
-          // half of the 32-byte run is columns 4 half .. 4 half + 3
+          // plane k1 of the half-step occupies 8 columns of the unit; this
+          // thread's share of the 32-byte run is columns NWA part .. NWA part + NWA - 1
 #pragma unroll
           for (int j = 0; j < Cfg::APH; ++j) {
-            uint32_t reg[4];
+            uint32_t reg[NWA];
 #pragma unroll
-            for (int c = 0; c < 4; ++c) reg[c] = pl[c][ph * Cfg::APH + j];
-            tc::tmem_st4(lane_base + Cfg::ACOL0 + buf * Cfg::AU_COLS + j * 8 + half * 4, reg);
+            for (int c = 0; c < NWA; ++c) reg[c] = pl[c][ph * Cfg::APH + j];
+            const uint32_t ta = lane_base + Cfg::ACOL0 + buf * Cfg::AU_COLS + j * 8 + part * NWA;
+            if constexpr (NWA == 2) tc::tmem_st2(ta, reg);
+            else tc::tmem_st4(ta, reg);
           }
           tc::tmem_wait_st();
           tc::fence_before_sync();
-          tc::mbar_arrive(&sh.a_full[buf]);
+          __syncwarp();
+          if (lane == 0) tc::mbar_arrive(&sh.a_full[buf]);
         }
         if (fail) return false;
 
@@ -448,7 +503,7 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
           }
           tc::fence_after_sync();
 #pragma unroll 1
-          for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 8) {
+          for (int c0 = part * (BN / ATPR); c0 < (part + 1) * (BN / ATPR); c0 += 8) {
             uint32_t acc[PP][8];
 #pragma unroll
             for (int q = 0; q < PP; ++q)
@@ -488,19 +543,21 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
       } else {
         const int st = g % NSB;
         bool fail = false;
-        if (g >= NSB) fail = !tc::mbar_wait(&sh.b_empty[st], ((g / NSB) - 1) & 1);
+        if (g >= NSB) fail = !__all_sync(0xffffffffu, tc::mbar_wait(&sh.b_empty[st], ((g / NSB) - 1) & 1));
         if (fail) {
-          raise_flag(status, CURVEFP_DEV_TIMEOUT);
+          if (lane == 0) raise_flag(status, CURVEFP_DEV_TIMEOUT);
           sh.abort_flag = 1;
           return false;
         }
-        decode_half<FB, PT>(cw, off, v, vc, mk, true);
+        uint32_t v[4], vc[4], mk[4][3];
+        decode_words<FB, PT, 4>(cw, off, v, vc, mk, true);
         uint8_t* stg = bstage + (size_t)st * Cfg::BSTAGE;
-        if (p == 0) write_b_planes<Cfg, PT, 0>(stg, rloc, half, v, vc, mk);
-        if (NP > 1 && p == 1) write_b_planes<Cfg, PT, (NP > 1 ? 1 : 0)>(stg, rloc, half, v, vc, mk);
-        if (NP > 2 && p == 2) write_b_planes<Cfg, PT, (NP > 2 ? 2 : 0)>(stg, rloc, half, v, vc, mk);
+        if (p == 0) write_b_planes<Cfg, PT, 0>(stg, rloc, part, v, vc, mk);
+        if (NP > 1 && p == 1) write_b_planes<Cfg, PT, (NP > 1 ? 1 : 0)>(stg, rloc, part, v, vc, mk);
+        if (NP > 2 && p == 2) write_b_planes<Cfg, PT, (NP > 2 ? 2 : 0)>(stg, rloc, part, v, vc, mk);
         tc::fence_proxy_async_smem();
-        tc::mbar_arrive(&sh.b_full[st]);
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&sh.b_full[st]);
       }
       return true;
     };
@@ -528,16 +585,19 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
       const int st = g % NSB;
       ok = __all_sync(0xffffffffu, tc::mbar_wait(&sh.b_full[st], (g / NSB) & 1));
 #pragma unroll
-      for (int ph = 0; ph < 2; ++ph) {
-        const int u = 2 * g + ph, buf = u & (Cfg::NAU - 1);
+      for (int ph = 0; ph < Cfg::UPS; ++ph) {
+        const int u = Cfg::UPS * g + ph, buf = u & (Cfg::NAU - 1);
         ok = ok && __all_sync(0xffffffffu, tc::mbar_wait(&sh.a_full[buf], (u / Cfg::NAU) & 1));
-        ok = ok && !read_abort(&sh.abort_flag);
+        // a producer that gave up also stops arriving, so the waits above end
+        // the loop anyway; the flag only shortens that, and is read rarely
+        // because every cycle of this loop delays the next MMA
+        if ((g & 7) == 0 && ph == 0) ok = ok && !read_abort(&sh.abort_flag);
         if (!ok) break;
         tc::fence_after_sync();
-        if (ph == 0)
-          issue_step<Cfg, PT, 0>(leader, p, tmem, bdesc0, buf, st, s == 0);
-        else
-          issue_step<Cfg, PT, 1>(leader, p, tmem, bdesc0, buf, st, s == 0);
+        if (ph == 0) issue_step<Cfg, PT, 0>(leader, p, tmem, bdesc0, buf, st, s == 0);
+        if (Cfg::UPS > 1 && ph == 1) issue_step<Cfg, PT, (Cfg::UPS > 1 ? 1 : 0)>(leader, p, tmem, bdesc0, buf, st, s == 0);
+        if (Cfg::UPS > 2 && ph == 2) issue_step<Cfg, PT, (Cfg::UPS > 2 ? 2 : 0)>(leader, p, tmem, bdesc0, buf, st, s == 0);
+        if (Cfg::UPS > 3 && ph == 3) issue_step<Cfg, PT, (Cfg::UPS > 3 ? 3 : 0)>(leader, p, tmem, bdesc0, buf, st, s == 0);
         tc::mma_commit_if(leader, &sh.a_empty[buf]);
       }
       if (!ok) break;
