@@ -43,10 +43,6 @@
 #define CFP_TC_ATPR 2  // A producer threads per row (2 or 4)
 #endif
 
-#ifndef CFP_TC_UPS
-#define CFP_TC_UPS 1  // A staging units per pipeline step (1, 2 or 4)
-#endif
-
 #ifndef CFP_TC_PLANE
 #define CFP_TC_PLANE 1  // 0: BF16 planes (K = 16 per MMA), 1: E5M2 planes (K = 32 per MMA)
 #endif
@@ -71,13 +67,10 @@ struct TcCfg {
   static constexpr int PP = 4;                            // phases per pass
   static constexpr int NP = (L + PP - 1) / PP;            // passes
   static constexpr int ACC_COLS = PP * BN;
-  // A is staged in units of APH planes: unit UPS g + ph holds planes
-  // [ph APH, (ph + 1) APH) of step g, 8 TMEM columns per plane; NAU units
-  // (two steps) rotate.
-  static constexpr int UPS = CFP_TC_UPS < KA ? CFP_TC_UPS : KA;  // units per step
-  static constexpr int APH = KA / UPS;                              // planes per unit
-  static constexpr int AU_COLS = APH * 8;
-  static constexpr int NAU = 2 * UPS;                               // two steps in flight
+  // A planes of a step occupy AU_COLS TMEM columns (8 per plane); two steps
+  // rotate (NAU units).
+  static constexpr int AU_COLS = KA * 8;
+  static constexpr int NAU = 2;
   static constexpr int ACOL0 = ACC_COLS;
   static_assert(ACC_COLS + NAU * AU_COLS <= 512, "TMEM budget");
   static constexpr int PLANE_BYTES = BN * 32;             // 128 rows x 32 bytes
@@ -136,10 +129,15 @@ struct TcCfg {
   static constexpr size_t SMEM = (size_t)NSB * BSTAGE + 2048;
 };
 
-constexpr int TC_MAX_RING = 8;  // capacity of the barrier rings below (>= NAU, NSB)
+constexpr int TC_MAX_RING = 4;  // capacity of the barrier rings below (= NSB)
 
+// Step g is handed over on full[g % NSB] (A and B producers arrive once per
+// warp) and released on empty[g % NSB] (one MMA commit): one wait and one
+// commit per step on the MMA warp's path.  A producers refill TMEM unit g % 2
+// after empty[(g - 2) % NSB]; B producers refill stage g % NSB after
+// empty[(g - NSB) % NSB].
 struct TcShared {
-  uint64_t a_full[TC_MAX_RING], a_empty[TC_MAX_RING], b_full[TC_MAX_RING], b_empty[TC_MAX_RING], acc_full, drain;
+  uint64_t full[TC_MAX_RING], empty[TC_MAX_RING], acc_full, drain;
   uint32_t tmem_base;
   int abort_flag;
   int refB[128];  // >= BN
@@ -317,17 +315,17 @@ __device__ __forceinline__ void write_b_planes(uint8_t* stage, int row, int kc, 
   }
 }
 
-template <class Cfg, int PT, int PASS, int PH>
+template <class Cfg, int PT, int PASS>
 __device__ __forceinline__ void issue_pass(uint32_t leader, uint32_t tmem, uint64_t bdesc0, int abuf, int bstage,
                                            bool first_step) {
 #pragma unroll
-  for (int k1 = PH * Cfg::APH; k1 < (PH + 1) * Cfg::APH; ++k1)
+  for (int k1 = 0; k1 < Cfg::KA; ++k1)
 #pragma unroll
     for (int k2 = 0; k2 < Cfg::KB; ++k2) {
       const int h = Cfg::phase(k1, k2);
       if (h / Cfg::PP != PASS) continue;
       const int sl = Cfg::slot(PASS, Cfg::carry(k1, k2), k2);
-      const uint32_t a_t = tmem + Cfg::ACOL0 + abuf * Cfg::AU_COLS + (k1 - PH * Cfg::APH) * 8;
+      const uint32_t a_t = tmem + Cfg::ACOL0 + abuf * Cfg::AU_COLS + k1 * 8;
       const uint64_t bd = bdesc0 + (uint64_t)((bstage * Cfg::BSTAGE + sl * Cfg::PLANE_BYTES) >> 4);
       const uint32_t d_t = tmem + (h - PASS * Cfg::PP) * Cfg::BN;
       const uint32_t accum = (first_step && Cfg::first_of_phase(k1, k2)) ? 0u : 1u;
@@ -338,14 +336,12 @@ __device__ __forceinline__ void issue_pass(uint32_t leader, uint32_t tmem, uint6
     }
 }
 
-template <class Cfg, int PT, int PH>
+template <class Cfg, int PT>
 __device__ __forceinline__ void issue_step(uint32_t leader, int p, uint32_t tmem, uint64_t bdesc0, int abuf,
                                            int bstage, bool first_step) {
-  if (p == 0) issue_pass<Cfg, PT, 0, PH>(leader, tmem, bdesc0, abuf, bstage, first_step);
-  if (Cfg::NP > 1 && p == 1)
-    issue_pass<Cfg, PT, (Cfg::NP > 1 ? 1 : 0), PH>(leader, tmem, bdesc0, abuf, bstage, first_step);
-  if (Cfg::NP > 2 && p == 2)
-    issue_pass<Cfg, PT, (Cfg::NP > 2 ? 2 : 0), PH>(leader, tmem, bdesc0, abuf, bstage, first_step);
+  if (p == 0) issue_pass<Cfg, PT, 0>(leader, tmem, bdesc0, abuf, bstage, first_step);
+  if (Cfg::NP > 1 && p == 1) issue_pass<Cfg, PT, (Cfg::NP > 1 ? 1 : 0)>(leader, tmem, bdesc0, abuf, bstage, first_step);
+  if (Cfg::NP > 2 && p == 2) issue_pass<Cfg, PT, (Cfg::NP > 2 ? 2 : 0)>(leader, tmem, bdesc0, abuf, bstage, first_step);
 }
 
 __device__ __forceinline__ float phase_const(int L, int h) {
@@ -369,7 +365,7 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
   constexpr int NAW = Cfg::NAW, NWA = Cfg::NWA, ATPR = Cfg::ATPR;
   constexpr int CB = PT == PLANE_E5M2 ? 4 : 2;  // code bytes per TMEM column / value word
   static_assert(NP <= 3, "pass dispatch");
-  static_assert(Cfg::NAU <= TC_MAX_RING && NSB <= TC_MAX_RING, "barrier rings");
+  static_assert(NSB == TC_MAX_RING && Cfg::NAU == 2, "barrier rings");
   extern __shared__ __align__(1024) uint8_t smem[];
   uint8_t* bstage = smem;
   TcShared& sh = *reinterpret_cast<TcShared*>(smem + (size_t)NSB * Cfg::BSTAGE);
@@ -379,13 +375,9 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
   const int nb = K / G, nsub = K / Cfg::KS, total = NP * nsub;
 
   if (tid == 0) {
-    for (int s = 0; s < Cfg::NAU; ++s) {
-      tc::mbar_init(&sh.a_full[s], NAW);  // one arrival per producer warp
-      tc::mbar_init(&sh.a_empty[s], 1);
-    }
     for (int s = 0; s < NSB; ++s) {
-      tc::mbar_init(&sh.b_full[s], Cfg::NBT / 32);
-      tc::mbar_init(&sh.b_empty[s], 1);
+      tc::mbar_init(&sh.full[s], NAW + Cfg::NBT / 32);  // one arrival per producer warp
+      tc::mbar_init(&sh.empty[s], 1);
     }
     tc::mbar_init(&sh.acc_full, 1);
     tc::mbar_init(&sh.drain, 1);
@@ -462,37 +454,33 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
         uint32_t pl[NWA][8];
 #pragma unroll
         for (int c = 0; c < NWA; ++c) planes_of<Fmt<FA>::C>(v[c], mk[c], pl[c]);
-        bool fail = false;
-#pragma unroll
-        for (int ph = 0; ph < Cfg::UPS; ++ph) {
-          const int u = Cfg::UPS * g + ph, buf = u & (Cfg::NAU - 1);
-          if (u >= Cfg::NAU) {
-            // warp-uniform outcome: the TMEM stores below are warp-collective
-            fail = !__all_sync(0xffffffffu, tc::mbar_wait(&sh.a_empty[buf], ((u / Cfg::NAU) - 1) & 1));
-            tc::fence_after_sync();
-          }
-          if (fail) {
+        const int buf = g & 1;
+        if (g >= 2) {
+          // warp-uniform outcome: the TMEM stores below are warp-collective
+          const int gr = g - 2;
+          const bool ok = __all_sync(0xffffffffu, tc::mbar_wait(&sh.empty[gr % NSB], (gr / NSB) & 1));
+          tc::fence_after_sync();
+          if (!ok) {
             if (lane == 0) raise_flag(status, CURVEFP_DEV_TIMEOUT);
             sh.abort_flag = 1;
             return false;
           }
-          // plane k1 of the half-step occupies 8 columns of the unit; this
-          // thread's share of the 32-byte run is columns NWA part .. NWA part + NWA - 1
-#pragma unroll
-          for (int j = 0; j < Cfg::APH; ++j) {
-            uint32_t reg[NWA];
-#pragma unroll
-            for (int c = 0; c < NWA; ++c) reg[c] = pl[c][ph * Cfg::APH + j];
-            const uint32_t ta = lane_base + Cfg::ACOL0 + buf * Cfg::AU_COLS + j * 8 + part * NWA;
-            if constexpr (NWA == 2) tc::tmem_st2(ta, reg);
-            else tc::tmem_st4(ta, reg);
-          }
-          tc::tmem_wait_st();
-          tc::fence_before_sync();
-          __syncwarp();
-          if (lane == 0) tc::mbar_arrive(&sh.a_full[buf]);
         }
-        if (fail) return false;
+        // plane k1 occupies 8 columns of the unit; this thread's share of
+        // the 32-byte run is columns NWA part .. NWA part + NWA - 1
+#pragma unroll
+        for (int j = 0; j < Cfg::KA; ++j) {
+          uint32_t reg[NWA];
+#pragma unroll
+          for (int c = 0; c < NWA; ++c) reg[c] = pl[c][j];
+          const uint32_t ta = lane_base + Cfg::ACOL0 + buf * Cfg::AU_COLS + j * 8 + part * NWA;
+          if constexpr (NWA == 2) tc::tmem_st2(ta, reg);
+          else tc::tmem_st4(ta, reg);
+        }
+        tc::tmem_wait_st();
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&sh.full[g % NSB]);
 
         if (s == nsub - 1) {
           // ---------------- epilogue of pass p -----------------------------
@@ -543,7 +531,7 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
       } else {
         const int st = g % NSB;
         bool fail = false;
-        if (g >= NSB) fail = !__all_sync(0xffffffffu, tc::mbar_wait(&sh.b_empty[st], ((g / NSB) - 1) & 1));
+        if (g >= NSB) fail = !__all_sync(0xffffffffu, tc::mbar_wait(&sh.empty[st], ((g / NSB) - 1) & 1));
         if (fail) {
           if (lane == 0) raise_flag(status, CURVEFP_DEV_TIMEOUT);
           sh.abort_flag = 1;
@@ -557,7 +545,7 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
         if (NP > 2 && p == 2) write_b_planes<Cfg, PT, (NP > 2 ? 2 : 0)>(stg, rloc, part, v, vc, mk);
         tc::fence_proxy_async_smem();
         __syncwarp();
-        if (lane == 0) tc::mbar_arrive(&sh.b_full[st]);
+        if (lane == 0) tc::mbar_arrive(&sh.full[st]);
       }
       return true;
     };
@@ -583,25 +571,15 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
     for (int g = 0; g < total && ok; ++g) {
       const int p = (NP > 1 && g >= nsub ? 1 : 0) + (NP > 2 && g >= 2 * nsub ? 1 : 0), s = g - p * nsub;
       const int st = g % NSB;
-      ok = __all_sync(0xffffffffu, tc::mbar_wait(&sh.b_full[st], (g / NSB) & 1));
-#pragma unroll
-      for (int ph = 0; ph < Cfg::UPS; ++ph) {
-        const int u = Cfg::UPS * g + ph, buf = u & (Cfg::NAU - 1);
-        ok = ok && __all_sync(0xffffffffu, tc::mbar_wait(&sh.a_full[buf], (u / Cfg::NAU) & 1));
-        // a producer that gave up also stops arriving, so the waits above end
-        // the loop anyway; the flag only shortens that, and is read rarely
-        // because every cycle of this loop delays the next MMA
-        if ((g & 7) == 0 && ph == 0) ok = ok && !read_abort(&sh.abort_flag);
-        if (!ok) break;
-        tc::fence_after_sync();
-        if (ph == 0) issue_step<Cfg, PT, 0>(leader, p, tmem, bdesc0, buf, st, s == 0);
-        if (Cfg::UPS > 1 && ph == 1) issue_step<Cfg, PT, (Cfg::UPS > 1 ? 1 : 0)>(leader, p, tmem, bdesc0, buf, st, s == 0);
-        if (Cfg::UPS > 2 && ph == 2) issue_step<Cfg, PT, (Cfg::UPS > 2 ? 2 : 0)>(leader, p, tmem, bdesc0, buf, st, s == 0);
-        if (Cfg::UPS > 3 && ph == 3) issue_step<Cfg, PT, (Cfg::UPS > 3 ? 3 : 0)>(leader, p, tmem, bdesc0, buf, st, s == 0);
-        tc::mma_commit_if(leader, &sh.a_empty[buf]);
-      }
+      ok = __all_sync(0xffffffffu, tc::mbar_wait(&sh.full[st], (g / NSB) & 1));
+      // a producer that gave up also stops arriving, so the wait above ends
+      // the loop anyway; the flag only shortens that, and is read rarely
+      // because every cycle of this loop delays the next MMA
+      if ((g & 7) == 0) ok = ok && !read_abort(&sh.abort_flag);
       if (!ok) break;
-      tc::mma_commit_if(leader, &sh.b_empty[st]);
+      tc::fence_after_sync();
+      issue_step<Cfg, PT>(leader, p, tmem, bdesc0, g & 1, st, s == 0);
+      tc::mma_commit_if(leader, &sh.empty[st]);
       if (s == nsub - 1) tc::mma_commit_if(leader, &sh.acc_full);
     }
     if (!ok && lane == 0) {
