@@ -1,18 +1,24 @@
 // CurveFP block-scaled quantization and dequantization (Sec. 3.1, Eq. 1).
 //
-// Quantizer: one HBM streaming pass.  Each block of G values is read with
-// 16-byte vector loads by a group of lanes, reduced to max|x| with warp
-// shuffles, turned into the ceil-absmax scale a_b by integer exponent and
-// mantissa arithmetic, and every element is encoded without a search loop:
-//   t  = bits(|x|) - a_b * 2^23           (exponent subtraction = x * 2^{-a_b})
-//   j  = number of midpoints (2^{k/K} + 2^{(k+1)/K})/2 below the mantissa,
-//        from a 256-entry LUT on the top mantissa bits plus one compare
-//   m  = K * (exponent of t) + j + bias   (nearest lattice point, as a rank)
-//   m  = 0 below L_nmin/2, >= 1 otherwise; code = sign << 7 | m.
-// All thresholds are irrational, so no FP32 input ties.  Blocks containing
-// NaN, Inf or values that need subnormal care take an exact slow path.
+// Quantizer: one HBM streaming pass.  Each block of G values is reduced to
+// max|x| (16-bit SIMD max for BF16, warp shuffles across the lanes that share
+// the block), the ceil-absmax scale a_b comes from the max's exponent and one
+// mantissa compare (App. A.2), and every element is encoded without a search:
+// its scaled magnitude |x| 2^{-a_b} is a binade offset from the zero boundary
+// F_z plus a mantissa, and an exact rank table indexed by (binade offset, top
+// 7 mantissa bits) gives the nearest level's rank (BF16: the whole decision,
+// its mantissa has 7 bits; FP32: plus one compare against the bucket's
+// threshold).  m = 0 below L_nmin/2; code = sign << 7 | m, zero always 0x00.
+// All thresholds are irrational, so no input ties; the tables are generated
+// in exact integer arithmetic.  Blocks containing NaN, Inf or values that
+// need subnormal care take an exact slow path.
+//
+// Dense rows with G = 32 (the common case) are fed by bulk (TMA) copies into a
+// shared-memory ring; other shapes use a register-fed kernel of the same
+// arithmetic.
 #include "cfp_common.cuh"
 #include "kernels.cuh"
+#include "tc_ptx.cuh"
 
 namespace cfp {
 
@@ -325,6 +331,196 @@ __global__ void __launch_bounds__(256) quantize_rows_kernel(const T* __restrict_
 }
 
 // ---------------------------------------------------------------------------
+// block_axis 0, dense rows, G = 32: the same encoder fed by bulk (TMA) copies.
+// One producer lane streams 16 KB chunks of the input into a ring of NST
+// shared-memory stages (completion counted in mbarrier transaction bytes);
+// 16 consumer warps each take 1 KB of every chunk with conflict-free 16-byte
+// shared loads, release the stage at once, encode, and write codes and scales
+// straight to global memory.  The input stream never waits on the encoder's
+// arithmetic, which the register-fed kernel above cannot avoid.
+constexpr int QB_CHUNK = 16384;  // bytes per stage
+constexpr int QB_NCW = 16;       // consumer warps, 1 KB of each chunk each
+
+template <int FMT, typename T>
+struct BulkQ {
+  static constexpr int NTAB = RankTab<FMT>::NBIN * 128;
+  static constexpr bool BF16 = sizeof(T) == 2;
+  static constexpr size_t smem(int nst) {
+    return (size_t)nst * QB_CHUNK + 256 * 4 + (size_t)NTAB * (BF16 ? 1 : 4) + (size_t)2 * nst * 8;
+  }
+};
+
+#ifndef CFP_QB_NST
+#define CFP_QB_NST 3  // stages of the bulk-fed quantizer
+#endif
+#ifndef CFP_QB_CTAS
+#define CFP_QB_CTAS 2  // its resident CTAs per SM (at most)
+#endif
+
+template <int FMT, typename T, int NST>
+__global__ void __launch_bounds__((QB_NCW + 1) * 32, CFP_QB_CTAS) quantize_rows_bulk_kernel(const T* __restrict__ x, int64_t nblk,
+                                                                              uint8_t* __restrict__ codes,
+                                                                              int8_t* __restrict__ scales,
+                                                                              uint32_t* status) {
+  using F = Fmt<FMT>;
+  constexpr int G = 32;
+  constexpr bool BF16 = sizeof(T) == 2;
+  constexpr int VEC = 16 / (int)sizeof(T);  // elements per 16-byte vector
+  constexpr int TPB = G / VEC;              // lanes per block: 4 (BF16) or 8 (FP32)
+  constexpr int BLK_BYTES = G * (int)sizeof(T);
+  constexpr int CH_BLK = QB_CHUNK / BLK_BYTES;  // blocks per chunk
+  constexpr int NTAB = BulkQ<FMT, T>::NTAB;
+  extern __shared__ __align__(128) uint8_t qsm[];
+  uint8_t* ring = qsm;
+  uint32_t* lut = reinterpret_cast<uint32_t*>(qsm + (size_t)NST * QB_CHUNK);
+  uint32_t* tab = lut + 256;  // FP32: full entries; BF16: rank bytes (tab8)
+  uint8_t* tab8 = reinterpret_cast<uint8_t*>(tab);
+  uint64_t* full = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(tab) + (size_t)NTAB * (BF16 ? 1 : 4));
+  uint64_t* empty = full + NST;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int i = threadIdx.x; i < 256; i += blockDim.x) lut[i] = __ldg(lut_src<F::K>() + i);
+  for (int i = threadIdx.x; i < NTAB; i += blockDim.x) {
+    const uint32_t e = __ldg(RankTab<FMT>::src() + i);
+    if (BF16)
+      tab8[i] = (uint8_t)(e & 0xFFu);
+    else
+      tab[i] = e;
+  }
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < NST; ++i) {
+      tc::mbar_init(&full[i], 1);
+      tc::mbar_init(&empty[i], QB_NCW);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+
+  const int64_t nchunks = (nblk + CH_BLK - 1) / CH_BLK;
+  if (warp == QB_NCW) {
+    // ------------------------------ producer ---------------------------------
+    if (lane == 0) {
+      int issued = 0;
+      bool ok = true;
+      for (int64_t c = blockIdx.x; c < nchunks; c += gridDim.x, ++issued) {
+        const int st = issued % NST;
+        if (issued >= NST && !tc::mbar_wait(&empty[st], ((issued / NST) - 1) & 1)) {
+          ok = false;
+          break;
+        }
+        const int64_t b0 = c * CH_BLK;
+        const int64_t left = nblk - b0;
+        const uint32_t bytes = (uint32_t)(left < CH_BLK ? left : CH_BLK) * BLK_BYTES;
+        tc::mbar_arrive_expect_tx(&full[st], bytes);
+        tc::bulk_g2s(ring + (size_t)st * QB_CHUNK, reinterpret_cast<const uint8_t*>(x) + b0 * BLK_BYTES, bytes,
+                     &full[st]);
+      }
+      if (!ok) {
+        if (status) atomicOr(status, CURVEFP_DEV_TIMEOUT);
+        // the copies already issued land before the CTA may exit
+        for (int j = issued - NST < 0 ? 0 : issued - NST; j < issued; ++j) tc::mbar_wait(&full[j % NST], (j / NST) & 1);
+      }
+    }
+    return;
+  }
+
+  // ------------------------------ consumers ----------------------------------
+  bool saw_nan = false;
+  const int sub = lane % TPB;
+  int it = 0;
+  for (int64_t c = blockIdx.x; c < nchunks; c += gridDim.x, ++it) {
+    const int st = it % NST;
+    if (!__all_sync(0xffffffffu, tc::mbar_wait(&full[st], (it / NST) & 1))) {
+      if (lane == 0 && status) atomicOr(status, CURVEFP_DEV_TIMEOUT);
+      break;
+    }
+    const uint4* src = reinterpret_cast<const uint4*>(ring + (size_t)st * QB_CHUNK + warp * 1024);
+    uint4 v[2];
+    v[0] = src[lane];
+    v[1] = src[32 + lane];
+    __syncwarp();
+    if (lane == 0) tc::mbar_arrive(&empty[st]);  // the data is in registers: refill the stage now
+    const int64_t b0 = c * CH_BLK;
+    const int64_t left = nblk - b0;
+    const int nb = (int)(left < CH_BLK ? left : CH_BLK);
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      const int lb = (warp * 64 + q * 32 + lane) / TPB;  // block within the chunk
+      const uint32_t w[4] = {v[q].x, v[q].y, v[q].z, v[q].w};
+      uint32_t mx = 0u;
+      if (BF16) {
+        uint32_t m2 = 0u;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) m2 = max_u16x2(m2, w[i] & 0x7FFF7FFFu);
+        mx = max(m2 & 0xFFFFu, m2 >> 16) << 16;
+      } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) mx = max(mx, w[i] & 0x7FFFFFFFu);
+      }
+#pragma unroll
+      for (int o = TPB / 2; o > 0; o >>= 1) mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      int a = block_scale<FMT>(mx);
+      const bool fast = mx < 0x7F800000u && a >= -100;
+      if (__any_sync(0xffffffffu, !fast)) {  // rare: NaN / Inf / subnormal-scale blocks
+        uint32_t mx2 = 0u;
+#pragma unroll
+        for (int i = 0; i < VEC; ++i) {
+          const uint32_t b = Elem<T>::bits(v[q], i) & 0x7FFFFFFFu;
+          mx2 = max(mx2, b > 0x7F800000u ? 0u : b);
+        }
+#pragma unroll
+        for (int o = TPB / 2; o > 0; o >>= 1) mx2 = max(mx2, __shfl_xor_sync(0xffffffffu, mx2, o));
+        if (!fast) a = block_scale<FMT>(mx2);
+      }
+      if (lb >= nb) continue;
+      const int64_t blk = b0 + lb;
+      if (sub == 0) scales[blk] = (int8_t)a;
+      uint8_t* d = codes + blk * G + sub * VEC;
+      const int kb = (127 + a + ZeroBoundary<FMT>::FZ) << 7;
+      if (fast) {
+        if (BF16) {
+          const uint32_t kb2 = (uint32_t)kb * 0x00010001u;
+          uint32_t out[2];
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const uint32_t w0 = w[2 * h], w1 = w[2 * h + 1];
+            const uint32_t k0 = max_u16x2(w0 & 0x7FFF7FFFu, kb2) - kb2;
+            const uint32_t k1 = max_u16x2(w1 & 0x7FFF7FFFu, kb2) - kb2;
+            const uint32_t r0 = tab8[k0 & 0xFFFFu], r1 = tab8[k0 >> 16];
+            const uint32_t r2 = tab8[k1 & 0xFFFFu], r3 = tab8[k1 >> 16];
+            const uint32_t r4 = __byte_perm(__byte_perm(r0, r1, 0x0040), __byte_perm(r2, r3, 0x0040), 0x5410);
+            out[h] = merge_signs(r4, __byte_perm(w0, w1, 0x7531));
+          }
+          *reinterpret_cast<uint2*>(d) = make_uint2(out[0], out[1]);
+        } else {
+          uint32_t r[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const uint32_t ab = w[i] & 0x7FFFFFFFu;
+            const uint32_t e = tab[max(ab >> 16, (uint32_t)kb) - (uint32_t)kb];
+            r[i] = ((ab & 0xFFFFu) >= (e >> 16)) ? ((e >> 8) & 0xFFu) : (e & 0xFFu);
+          }
+          const uint32_t r4 = r[0] | (r[1] << 8) | (r[2] << 16) | (r[3] << 24);
+          const uint32_t s4 = __byte_perm(__byte_perm(w[0], w[1], 0x0073), __byte_perm(w[2], w[3], 0x7300), 0x7610);
+          *reinterpret_cast<uint32_t*>(d) = merge_signs(r4, s4);
+        }
+      } else {
+        uint32_t cc[VEC];
+#pragma unroll
+        for (int i = 0; i < VEC; ++i) cc[i] = encode_slow<FMT>(lut, Elem<T>::bits(v[q], i), a, saw_nan);
+        if constexpr (VEC == 4) {
+          *reinterpret_cast<uint32_t*>(d) = cc[0] | (cc[1] << 8) | (cc[2] << 16) | (cc[3] << 24);
+        } else {
+          *reinterpret_cast<uint2*>(d) = make_uint2(cc[0] | (cc[1] << 8) | (cc[2] << 16) | (cc[3] << 24),
+                                                    cc[4] | (cc[5] << 8) | (cc[6] << 16) | (cc[7] << 24));
+        }
+      }
+    }
+  }
+  if (saw_nan && status) atomicOr(status, CURVEFP_DEV_NAN);
+}
+
+// ---------------------------------------------------------------------------
 // block_axis 1: blocks of G consecutive rows of one column; the output is the
 // transposed operand (codes [cols x rows]).  One lane owns one column and one
 // row-block: its loads are coalesced across the warp (consecutive columns),
@@ -445,9 +641,35 @@ __global__ void __launch_bounds__(256) dequantize_kernel(const uint8_t* __restri
 // ---------------------------------------------------------------------------
 // Host-side launchers (called by the C ABI after argument validation).
 
+template <int FMT, typename T>
+static cudaError_t launch_q_bulk(const void* x, int64_t nblk, uint8_t* codes, int8_t* scales, uint32_t* status,
+                                 cudaStream_t st, int sms) {
+  constexpr int NST = CFP_QB_NST;
+  const size_t smem = BulkQ<FMT, T>::smem(NST);
+  auto kern = quantize_rows_bulk_kernel<FMT, T, NST>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  const int64_t ch_blk = QB_CHUNK / (32 * (int64_t)sizeof(T));
+  const int64_t nchunks = (nblk + ch_blk - 1) / ch_blk;
+  // persistent CTAs take chunks round-robin, so the grid must be resident at once
+  int per_sm = 0;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, (QB_NCW + 1) * 32, smem);
+  if (e != cudaSuccess) return e;
+  if (per_sm > CFP_QB_CTAS) per_sm = CFP_QB_CTAS;
+  if (per_sm < 1) per_sm = 1;
+  int64_t grid = (int64_t)sms * per_sm;
+  if (grid > nchunks) grid = nchunks;
+  kern<<<(unsigned)grid, (QB_NCW + 1) * 32, smem, st>>>(static_cast<const T*>(x), nblk, codes, scales, status);
+  return cudaGetLastError();
+}
+
 template <int FMT, typename T, int G>
 static cudaError_t launch_q(const void* x, int64_t rows, int64_t cols, int64_t ld, int axis, uint8_t* codes,
                             int8_t* scales, uint32_t* status, cudaStream_t st, int sms) {
+  // dense rows of 32-element blocks: the bulk-fed kernel (16-byte aligned
+  // input is checked by the caller for block_axis 0)
+  if (axis == 0 && G == 32 && ld == cols)
+    return launch_q_bulk<FMT, T>(x, rows * (cols / G), codes, scales, status, st, sms);
   if (axis == 0) {
     constexpr int VEC = Elem<T>::VEC;
     constexpr int TPB = (sizeof(T) == 2 && G == 32) ? 2 : ((G / VEC) < 8 ? (G / VEC) : 8);

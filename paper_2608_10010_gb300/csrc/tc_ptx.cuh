@@ -1,6 +1,6 @@
-// Inline-PTX wrappers for the sm_103a tensor-core path: tcgen05 (TMEM
-// allocation, loads/stores, MMA, commit), mbarriers with bounded waits, and
-// the shared-memory / instruction descriptors of tcgen05.mma.
+// Inline-PTX wrappers for sm_103a: mbarriers with bounded waits, bulk (TMA)
+// copies, tcgen05 (TMEM allocation, loads/stores, MMA, commit) and the
+// shared-memory / instruction descriptors of tcgen05.mma.
 #pragma once
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -50,6 +50,21 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
   while (!mbar_try_wait_hint(bar, parity, 100000u))
     if (clock64() - t0 > (1ll << 31)) return false;
   return true;
+}
+
+// ---- bulk copies (the TMA unit's 1D form) ------------------------------------
+// Arrive on a barrier and add `bytes` to the transaction count it waits for.
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+// Global -> shared copy of `bytes` (a multiple of 16; both addresses 16-byte
+// aligned); completion is counted on `bar` as transaction bytes.
+__device__ __forceinline__ void bulk_g2s(void* dst_smem, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_u32(dst_smem)),
+               "l"(src), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
 }
 
 __device__ __forceinline__ void fence_proxy_async_smem() {

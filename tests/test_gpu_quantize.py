@@ -57,6 +57,17 @@ def test_formats_blocks_dtypes(torch, fmt, dtype, block):
     check_q(torch, y, fmt, block, 1, dtype)
 
 
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("shape", [(1, 32), (3, 96), (1000, 4160), (257, 8192)])
+def test_chunk_boundaries(torch, dtype, shape):
+    """Dense rows of 32-element blocks are streamed in 16 KB chunks (256 BF16 or
+    128 FP32 blocks) by persistent CTAs: a single block, less than one chunk,
+    a ragged last chunk, and more chunks than resident CTAs."""
+    x = inputs.elementwise_outliers(shape, 70 + shape[0])
+    for fmt in FORMATS:
+        check_q(torch, x, fmt, 32, 0, dtype)
+
+
 @pytest.mark.parametrize("fmt", FORMATS)
 def test_binade_exhaustive(torch, fmt):
     """All 2^23 FP32 mantissas of the binade [1, 2) under a fixed block scale."""
