@@ -127,6 +127,81 @@ def aggregate(per_rank_seconds, per_rank_units):
     return sum(per_rank_units) / t, t
 
 
+# ------------------------------------------------------------ other workloads
+def _time_ms(torch, stream, fn, flush_l2, reps=5, warm=2):
+    """Median CUDA-event time of fn() on `stream`, L2 flushed before each run."""
+    out = []
+    for i in range(warm + reps):
+        flush_l2()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        fn()
+        e1.record(stream)
+        e1.synchronize()
+        if i >= warm:
+            out.append(e0.elapsed_time(e1))
+    return statistics.median(out)
+
+
+def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
+    """The remaining workloads, reported beside the headline line: the
+    quantize-only bandwidth sweep (BF16, 2^20..2^30 elements, three formats)
+    and the tensor-core GEMM on the training triplet and the FFN sweep."""
+    res = {"quantize_sweep": [], "gemm_shapes": []}
+    for lg in (20, 22, 24, 26, 28, 30):
+        n = 1 << lg
+        x = inputs.bandwidth_tensor_cuda(n, 4096 if n >= 4096 * 64 else 1024, 3)
+        codes = torch.empty(x.shape, dtype=torch.uint8, device=x.device)
+        sc = torch.empty((x.shape[0], x.shape[1] // G), dtype=torch.int8, device=x.device)
+        for fmt in ("E3C3", "E4C3", "E5C2"):
+            ms = _time_ms(torch, stream, lambda: cfp.quantize(x, fmt, G, 0, codes=codes, scales=sc, stream=stream),
+                          flush_l2)
+            gbs = n * (2 + 1 + 1 / G) / (ms / 1e3) / 1e9
+            res["quantize_sweep"].append({"n": f"2^{lg}", "format": fmt, "ms": round(ms, 4), "gbs": round(gbs, 1),
+                                          "frac_of_8TBps": round(gbs / 8000, 4),
+                                          "frac_of_measured_copy": round(gbs / hbm, 4)})
+        del x, codes, sc
+    torch.cuda.empty_cache()
+
+    def q(t, fmt, axis):
+        return cfp.quantize(t, fmt, G, axis, stream=stream)
+
+    def gemm_case(name, A, fa, B, fb, planes, hbm_bound=False):
+        a, sa = A
+        b, sb = B
+        Mx, Kx = a.shape
+        Nx = b.shape[0]
+        out = torch.empty((Mx, Nx), dtype=torch.float32, device=a.device)
+        ms = _time_ms(torch, stream, lambda: cfp.gemm(a, sa, b, sb, fa, fb, G, "tensor", out=out, stream=stream),
+                      flush_l2)
+        tops = 2.0 * Mx * Nx * Kx / (ms / 1e3) / 1e12
+        r = {"case": name, "M": Mx, "N": Nx, "K": Kx, "formats": f"{fa}x{fb}", "ms": round(ms, 4),
+             "tops": round(tops, 3), "tensor_work_frac": round(tops * planes / fp8_peak, 4)}
+        if hbm_bound:
+            wbytes = Nx * Kx + Nx * Kx // G
+            r["weight_code_gbs"] = round(wbytes / (ms / 1e3) / 1e9, 1)
+            r["frac_of_measured_copy"] = round(wbytes / (ms / 1e3) / 1e9 / hbm, 4)
+        res["gemm_shapes"].append(r)
+        del out
+
+    # training triplet, E4C3 weights/activations, E5C2 gradients
+    X, Wt, dY = inputs.training_triplet_cuda()
+    gemm_case("fwd X.W", q(X, "E4C3", 0), "E4C3", q(Wt, "E4C3", 1), "E4C3", 64)
+    gemm_case("dgrad dY.W^T", q(dY, "E5C2", 0), "E5C2", q(Wt, "E4C3", 0), "E4C3", 32)
+    gemm_case("wgrad dY^T.X", q(dY, "E5C2", 1), "E5C2", q(X, "E4C3", 1), "E4C3", 32)
+    del X, Wt, dY
+    torch.cuda.empty_cache()
+    # FFN sweep, E3C3, N = 14336
+    for Kf in (4096, 3584):
+        for Mf in (1, 16, 128, 4096):
+            Xf, Wf = inputs.ffn_cuda(Mf, Kf)
+            gemm_case(f"ffn M={Mf} K={Kf}", q(Xf, "E3C3", 0), "E3C3", q(Wf, "E3C3", 1), "E3C3", 64,
+                      hbm_bound=Mf <= 128)
+            del Xf, Wf
+    torch.cuda.empty_cache()
+    return res
+
+
 # ---------------------------------------------------------------------------- ours
 def run_ours(args):
     import torch
@@ -287,6 +362,11 @@ def run_ours(args):
     torch.cuda.synchronize()
     assert int(status.item()) == 0, f"device status {int(status.item())}"
 
+    extra = None
+    if not args.no_sweep and rank == 0:
+        extra = other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, 2.0 * bf16)
+        torch.cuda.synchronize()
+
     if rank != 0:
         if ws > 1:
             torch.distributed.destroy_process_group()
@@ -331,6 +411,8 @@ def run_ours(args):
         "clocks": clk.summary(),
         "wall_s_timed_region": round(wall, 4),
     }
+    if extra:
+        out.update(extra)
     if not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(ORACLE_SAMPLE_ROWS)
     if ws > 1:
@@ -428,6 +510,7 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--only", choices=["gemm", "quantize"], default=None)
+    ap.add_argument("--no-sweep", action="store_true", help="skip the other workloads (quantize sweep, GEMM shapes)")
     args = ap.parse_args()
     if args.only:
         run_only(args)

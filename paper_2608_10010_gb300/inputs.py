@@ -105,3 +105,34 @@ def bandwidth_tensor_cuda(n: int, cols: int = 4096, seed: int = 3):
     x = torch.where(mask, x * 100.0, x)
     del mask
     return x.to(torch.bfloat16)
+
+
+def training_triplet_cuda(tokens: int = 4096, d_in: int = 4096, d_out: int = 11008, seed: int = 3):
+    """Device-side draw of the training-GEMM tensors (same distributions as
+    ``training_triplet``, torch's CUDA generator): X[tokens x d_in] ~ N(0,1),
+    W[d_in x d_out] ~ N(0, 0.02^2), dY[tokens x d_out] = 1e-3 * t_3 with
+    t_3 = Z / sqrt(chi^2_3 / 3)."""
+    import torch
+
+    g = torch.Generator(device="cuda").manual_seed(seed)
+    x = torch.randn((tokens, d_in), device="cuda", generator=g)
+    w = torch.randn((d_in, d_out), device="cuda", generator=g) * 0.02
+    z = torch.randn((tokens, d_out), device="cuda", generator=g)
+    chi2 = torch.zeros_like(z)
+    for _ in range(3):
+        chi2 += torch.randn((tokens, d_out), device="cuda", generator=g) ** 2
+    dy = 1e-3 * z / torch.sqrt(chi2 / 3.0)
+    return x, w, dy
+
+
+def ffn_cuda(M: int, K: int = 4096, N: int = 14336, seed: int = 3):
+    """Device-side draw of an FFN-sweep case (same distributions as
+    ``ffn_sweep``): X[M x K] = Z diag(s), s_c ~ LogNormal(0, 1.5);
+    W[K x N] ~ N(0, 0.02^2)."""
+    import torch
+
+    g = torch.Generator(device="cuda").manual_seed(seed)
+    z = torch.randn((M, K), device="cuda", generator=g)
+    s = torch.exp(1.5 * torch.randn((K,), device="cuda", generator=g))
+    w = torch.randn((K, N), device="cuda", generator=g) * 0.02
+    return z * s[None, :], w
