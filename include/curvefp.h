@@ -57,8 +57,15 @@ typedef enum {
 
 /* GEMM kernels.  EXACT: integer-ALU kernel whose per-phase sums are exact
  * integers (bit-identical to the definition).  TENSOR: tcgen05 tensor-core
- * kernel over power-of-two phase planes with FP32 per-phase accumulation. */
-typedef enum { CURVEFP_GEMM_EXACT = 0, CURVEFP_GEMM_TENSOR = 1 } curvefp_gemm_algo_t;
+ * kernel over power-of-two phase planes with FP32 per-phase accumulation, one
+ * plane pair per dense MMA.  TENSOR_SPARSE: the same method with two plane
+ * pairs per 2:4-sparse MMA (half the tensor work, more producer arithmetic;
+ * code tiles streamed by TMA). */
+typedef enum {
+  CURVEFP_GEMM_EXACT = 0,
+  CURVEFP_GEMM_TENSOR = 1,
+  CURVEFP_GEMM_TENSOR_SPARSE = 2
+} curvefp_gemm_algo_t;
 
 /* Bits of the device status word. */
 #define CURVEFP_DEV_NAN 1u     /* quantize: a NaN input was encoded as 0x00        */
@@ -103,7 +110,10 @@ curvefp_status_t curvefp_dequantize(curvefp_format_t fmt, int block, const uint8
  * Requirements: K % block == 0; a, b 16-byte aligned.
  * EXACT: S_h exact, combine in FP64, one FP32 rounding; outputs whose scale
  *   spread leaves the int128 window raise CURVEFP_DEV_RANGE (values undefined).
- * TENSOR: S_h accumulated in FP32 on the tensor cores, combine in FP32. */
+ * TENSOR, TENSOR_SPARSE: S_h accumulated in FP32 on the tensor cores, combine
+ *   in FP32; plane values below 2^-14 of a row's largest block scale flush.
+ *   Format pairs: E3C3 x E3C3, E4C3 x E4C3, E5C2 x E4C3, E4C3 x E5C2,
+ *   E5C2 x E5C2 (others return CURVEFP_ERR_UNSUPPORTED). */
 curvefp_status_t curvefp_gemm(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, curvefp_format_t fmt_b, int block,
                               const uint8_t* a, const int8_t* sa, const uint8_t* b, const int8_t* sb, int64_t M,
                               int64_t N, int64_t K, float* c, uint32_t* device_status, void* stream);

@@ -14,7 +14,7 @@ from . import _build
 
 FORMATS = {"E3C3": 0, "E4C3": 1, "E5C2": 2}
 DTYPES = {"f32": 0, "bf16": 1}
-ALGOS = {"exact": 0, "tensor": 1}
+ALGOS = {"exact": 0, "tensor": 1, "tensor_sparse": 2}
 STATUS_BITS = {"nan": 1, "range": 2, "timeout": 4}
 
 _lib = None

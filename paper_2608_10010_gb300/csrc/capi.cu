@@ -76,8 +76,10 @@ curvefp_status_t curvefp_gemm(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, 
   if (algo == CURVEFP_GEMM_EXACT)
     return from_cuda(cfp::launch_gemm_exact(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, nullptr, nullptr,
                                             device_status, st));
-  if (algo == CURVEFP_GEMM_TENSOR) {
+  if (algo == CURVEFP_GEMM_TENSOR || algo == CURVEFP_GEMM_TENSOR_SPARSE) {
     if (!cfp::gemm_tensor_supported(fmt_a, fmt_b)) return CURVEFP_ERR_UNSUPPORTED;
+    if (algo == CURVEFP_GEMM_TENSOR_SPARSE)
+      return from_cuda(cfp::launch_gemm_tensor_sparse(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, device_status, st));
     return from_cuda(cfp::launch_gemm_tensor(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, device_status, st,
                                              sm_count()));
   }

@@ -16,6 +16,9 @@ cudaError_t launch_gemm_exact(int fa, int fb, int G, const uint8_t* a, const int
 cudaError_t launch_gemm_tensor(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
                                const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, uint32_t* status,
                                cudaStream_t st, int sms);
+cudaError_t launch_gemm_tensor_sparse(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
+                                      const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, uint32_t* status,
+                                      cudaStream_t st);
 bool gemm_tensor_supported(int fa, int fb);
 
 }  // namespace cfp

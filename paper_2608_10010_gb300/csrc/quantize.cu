@@ -438,8 +438,12 @@ __global__ void __launch_bounds__((QB_NCW + 1) * 32, CFP_QB_CTAS) quantize_rows_
     uint4 v[2];
     v[0] = src[lane];
     v[1] = src[32 + lane];
-    __syncwarp();
-    if (lane == 0) tc::mbar_arrive(&empty[st]);  // the data is in registers: refill the stage now
+    // refill the stage as soon as every lane's loads have returned: a shuffle
+    // consumes a word of each load and the arrival depends on its result (an
+    // arrival right after the loads could let the next bulk copy overwrite
+    // the stage while a load is still in flight)
+    const uint32_t dep = __shfl_xor_sync(0xffffffffu, v[0].x ^ v[1].x, 1);
+    if (lane == 0) tc::mbar_arrive_after(&empty[st], dep);
     const int64_t b0 = c * CH_BLK;
     const int64_t left = nblk - b0;
     const int nb = (int)(left < CH_BLK ? left : CH_BLK);

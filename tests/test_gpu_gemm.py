@@ -78,8 +78,8 @@ def check_exact(torch, a, sa, b, sb, fa, fb, block, rows=None):
     return c, ref
 
 
-def check_tensor(torch, a, sa, b, sb, fa, fb, block, rows=None):
-    c, st = gpu_gemm(torch, a, sa, b, sb, fa, fb, block, "tensor")
+def check_tensor(torch, a, sa, b, sb, fa, fb, block, rows=None, algo="tensor"):
+    c, st = gpu_gemm(torch, a, sa, b, sb, fa, fb, block, algo)
     assert st == 0
     ra = a if rows is None else a[rows]
     rsa = sa if rows is None else sa[rows]
@@ -149,24 +149,41 @@ def test_exact_zero_and_extreme_operands(torch):
 
 # ---- tensor kernel ------------------------------------------------------------------
 
+@pytest.mark.parametrize("algo", ["tensor", "tensor_sparse"])
 @pytest.mark.parametrize("fa,fb", TC_PAIRS)
-def test_tensor_pairs_ragged(torch, fa, fb):
+def test_tensor_pairs_ragged(torch, fa, fb, algo):
     rng = np.random.default_rng(99 + hash((fa, fb)) % 1000)
     for (M, N, K, block) in [(1, 1, 32, 32), (3, 17, 64, 32), (130, 33, 160, 32), (257, 70, 1024, 64), (128, 32, 512, 512)]:
         x = inputs.normal((M, K), int(rng.integers(1 << 30)))
         w = inputs.normal((N, K), int(rng.integers(1 << 30)), 0.02)
         a, sa = quantized(x, fa, block)
         b, sb = quantized(w, fb, block)
-        check_tensor(torch, a, sa, b, sb, fa, fb, block)
+        check_tensor(torch, a, sa, b, sb, fa, fb, block, algo=algo)
 
 
+@pytest.mark.parametrize("algo", ["tensor", "tensor_sparse"])
 @pytest.mark.parametrize("fa,fb", TC_PAIRS)
-def test_tensor_full_code_space(torch, fa, fb):
+def test_tensor_full_code_space(torch, fa, fb, algo):
     """Uniformly random codes (every level, both signs, zeros) and scale spread."""
     rng = np.random.default_rng(5)
     a, sa = rand_operand(rng, fa, 200, 256, 32, spread=6)
     b, sb = rand_operand(rng, fb, 100, 256, 32, spread=6)
-    check_tensor(torch, a, sa, b, sb, fa, fb, 32)
+    check_tensor(torch, a, sa, b, sb, fa, fb, 32, algo=algo)
+
+
+@pytest.mark.parametrize("fa,fb", TC_PAIRS)
+def test_tensor_sparse_matches_dense(torch, fa, fb):
+    """Two plane pairs per 2:4-sparse MMA against one per dense MMA: the same
+    exact products, summed in a different order in FP32."""
+    rng = np.random.default_rng(11)
+    a, sa = rand_operand(rng, fa, 300, 1024, 32, spread=4)
+    b, sb = rand_operand(rng, fb, 200, 1024, 32, spread=4)
+    cs, st = gpu_gemm(torch, a, sa, b, sb, fa, fb, 32, "tensor_sparse")
+    cd, st2 = gpu_gemm(torch, a, sa, b, sb, fa, fb, 32, "tensor")
+    assert st == 0 and st2 == 0
+    na = oracle.row_norms(a, sa, fa)
+    nb = oracle.row_norms(b, sb, fb)
+    assert normalised_error(cs, cd.astype(np.float64), na, nb) <= TOL
 
 
 def test_tensor_matches_exact_kernel(torch):
@@ -210,6 +227,7 @@ def test_llama7b_linear_full_size(torch):
     rows = _sample(2048)
     check_exact(torch, ra, rsa, rb, rsb, "E3C3", "E3C3", 32, rows=rows)
     check_tensor(torch, ra, rsa, rb, rsb, "E3C3", "E3C3", 32, rows=rows)
+    check_tensor(torch, ra, rsa, rb, rsb, "E3C3", "E3C3", 32, rows=rows, algo="tensor_sparse")
 
 
 @pytest.mark.parametrize("which", ["fwd", "dgrad", "wgrad"])
