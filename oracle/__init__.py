@@ -37,7 +37,7 @@ def build(force: bool = False) -> str:
     if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
         tmp = _LIB + f".tmp{os.getpid()}"
         subprocess.check_call(
-            ["gcc", "-O2", "-std=gnu11", "-fopenmp", "-fPIC", "-shared", _SRC, "-o", tmp, "-lm"]
+            ["gcc", "-O2", "-std=gnu11", "-ffp-contract=off", "-fopenmp", "-fPIC", "-shared", _SRC, "-o", tmp, "-lm"]
         )
         os.replace(tmp, _LIB)
     return _LIB
@@ -60,6 +60,7 @@ def _load():
             lib.oracle_quantize.argtypes = [i32, i32, P, i64, i64, i64, i32, P, P]
             lib.oracle_decode.argtypes = [i32, i32, P, P, i64, i64, P]
             lib.oracle_encode.argtypes = [i32, i32, P, i64, i64, P, P]
+            lib.oracle_quantize_static.argtypes = [i32, i32, P, i64, i64, i32, i32, P, P]
             lib.oracle_dequantize.argtypes = [i32, i32, P, P, i64, i64, P]
             lib.oracle_closed_product.argtypes = [i32, i32, ctypes.c_uint8, ctypes.c_uint8, P, P, P]
             lib.oracle_pair_info.argtypes = [i32, i32, P, P, P]
@@ -137,6 +138,25 @@ def quantize(x: np.ndarray, fmt, block: int = 32, block_axis: int = 0):
     )
     if flags < 0:
         raise ValueError(fmt)
+    return codes, scales, bool(flags & 1)
+
+
+GRANULARITY = {"block": 0, "row": 1, "tensor": 2}
+SCALE_RULE = {"ceil": 0, "mse": 1}
+
+
+def quantize_static(x: np.ndarray, fmt, block: int = 32, granularity: str = "block", rule: str = "mse"):
+    """Q(X) with a scale per block / row / tensor (R11) chosen by ceil-absmax
+    or by reconstruction-MSE search (R12).  x [rows x cols] FP32, blocks along
+    columns.  Returns (codes, scales [rows x cols/block], nan_flag)."""
+    x = np.ascontiguousarray(x, np.float32)
+    rows, cols = x.shape
+    codes = np.empty((rows, cols), np.uint8)
+    scales = np.empty((rows, cols // block), np.int8)
+    flags = _load().oracle_quantize_static(_fid(fmt), block, _ptr(x), rows, cols, GRANULARITY[granularity],
+                                           SCALE_RULE[rule], _ptr(codes), _ptr(scales))
+    if flags < 0:
+        raise ValueError("bad arguments")
     return codes, scales, bool(flags & 1)
 
 

@@ -35,6 +35,7 @@
  *      n_b L/K_b, h = u mod L, t = floor(u / L), H = L phases.
  *   R6 exported per-phase sums are integers S_h at the per-output LSB
  *      lambda = min_b(sa_b + sb_b) + t_min.
+ *   R11, R12 static-operand scale groups and MSE-search scales (below).
  */
 #include <math.h>
 #include <stdint.h>
@@ -210,6 +211,102 @@ int oracle_encode(int id, int G, const float* x, int64_t R, int64_t Cc, const in
       }
       codes[r * Cc + c] = code;
     }
+  return flags;
+}
+
+/* ---- Static operands: scale granularity and MSE-search scales ----------
+ * Sec. 3.1: "static operands choose a representable power-of-two scale by
+ * reconstruction-MSE search; dynamic training operands use ceil-absmax";
+ * Sec. 4.2 evaluates tensorwise, rowwise and fixed-size block scaling.
+ * Readings (listed with the others):
+ *   R11 a scale group is a block of G elements of a row, a whole row, or the
+ *       whole tensor; scales are stored per block of G ([rows x cols/G]),
+ *       every block of a group holding the group's scale.
+ *   R12 MSE search: candidates a in [a_c - 3, a_c + 1] (clamped to int8),
+ *       a_c the group's ceil-absmax scale; each element is encoded at scale a
+ *       (nearest level, R3, saturating) and reconstructed as in R4; the
+ *       criterion is D(a) = sum_i floor((x_i - xhat_i)^2 * 2^{60 - 2 a_c}),
+ *       an exact integer (every squared FP32 reconstruction error on a grid
+ *       of 2^{2 a_c - 60}); the smallest D wins, ties go to the larger a.
+ *       NaN elements are left out; groups with Inf, or with amax = 0, keep
+ *       a_c. */
+
+/* Reading R4 for one code under scale a (0.0f for the zero code). */
+static float odequant_one(const ofmt* f, uint8_t code, int a) {
+  int s, n;
+  if (!odecode(f, code, &s, &n)) return 0.0f;
+  int e = floordiv(n, f->K), k = floormod(n, f->K);
+  float ck = (float)exp2((double)k / f->K);
+  double exact = ldexp((double)ck, a + e);
+  return (float)(s ? -exact : exact);
+}
+
+static uint8_t oencode_one(const ofmt* f, float xv, int a) {
+  if (isnan(xv)) return 0;
+  int m = onearest_rank(f, ldexp(fabs((double)xv), -a));
+  return m ? (uint8_t)(((signbit(xv) ? 1 : 0) << 7) | m) : 0;
+}
+
+/* floor((x - xhat)^2 * 2^{60 - 2 ac}), exact.  x - xhat is exact in fp64
+ * (both FP32, within a factor 16 of each other unless xhat = 0), so
+ * e = M 2^{E-53} with an integer M < 2^53 and e^2 = M^2 2^{2E-106}. */
+static unsigned __int128 osq_term(float x, float xhat, int ac) {
+  double e = fabs((double)x - (double)xhat);
+  if (e == 0.0) return 0;
+  int E;
+  double fr = frexp(e, &E);                   /* e = fr 2^E, fr in [0.5, 1) */
+  unsigned long long M = (unsigned long long)ldexp(fr, 53);
+  unsigned __int128 sq = (unsigned __int128)M * M;
+  int sh = 2 * E - 106 + 60 - 2 * ac;          /* term = sq * 2^sh */
+  if (sh >= 0) return sh >= 128 ? 0 : sq << sh; /* (never taken: |e| < 2^{ac+18}) */
+  return sh <= -128 ? 0 : sq >> (-sh);
+}
+
+/* Quantize with a scale per group (R11) chosen by ceil-absmax (rule 0) or by
+ * MSE search (rule 1, R12).  granularity: 0 block of G, 1 row, 2 tensor.
+ * x [rows x cols] (ld = cols), blocks along columns (cols % G == 0); codes
+ * [rows x cols], scales [rows x cols/G].  Returns the NaN flag. */
+int oracle_quantize_static(int id, int G, const float* x, int64_t rows, int64_t cols, int granularity, int rule,
+                           uint8_t* codes, int8_t* scales) {
+  ofmt f;
+  if (ofmt_get(id, &f) || G <= 0 || cols % G) return -1;
+  int64_t nb = cols / G;
+  int64_t glen = granularity == 0 ? G : (granularity == 1 ? cols : rows * cols);
+  int64_t ngroups = (rows * cols) / glen;
+  int flags = 0;
+#pragma omp parallel for schedule(dynamic) reduction(| : flags)
+  for (int64_t g = 0; g < ngroups; ++g) {
+    /* group g covers flat elements [g glen, (g + 1) glen) of the row-major tensor */
+    const int64_t i0 = g * glen;
+    double amax = 0.0;
+    int has_inf = 0;
+    for (int64_t i = i0; i < i0 + glen; ++i) {
+      float xv = x[i];
+      if (isnan(xv)) { flags |= 1; continue; }
+      if (isinf(xv)) has_inf = 1;
+      double av = fabs((double)xv);
+      if (av > amax) amax = av;
+    }
+    int ac = oracle_block_scale(id, amax);
+    int best = ac;
+    if (rule == 1 && !has_inf && amax != 0.0) {
+      unsigned __int128 bestD = 0;
+      int first = 1;
+      for (int a = ac - 3; a <= ac + 1; ++a) {
+        if (a < -128 || a > 127) continue;
+        unsigned __int128 D = 0;
+        for (int64_t i = i0; i < i0 + glen; ++i) {
+          float xv = x[i];
+          if (isnan(xv)) continue;
+          D += osq_term(xv, odequant_one(&f, oencode_one(&f, xv, a), a), ac);
+        }
+        if (first || D <= bestD) { bestD = D; best = a; first = 0; } /* ties: the larger a */
+      }
+    }
+    for (int64_t i = i0; i < i0 + glen; ++i) codes[i] = oencode_one(&f, x[i], best);
+    for (int64_t i = i0; i < i0 + glen; i += G) scales[i / G] = (int8_t)best;
+  }
+  (void)nb;
   return flags;
 }
 
