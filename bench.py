@@ -184,6 +184,18 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
         res["gemm_shapes"].append(r)
         del out
 
+    # static-operand quantization of the Llama-7B-like weight (E3C3, block 32):
+    # scale groups and rules (MSE search is a one-off, compute-bound pass)
+    res["quantize_static"] = []
+    Wt32 = torch.randn((4096, 4096), device="cuda", generator=torch.Generator(device="cuda").manual_seed(4)) * 0.02
+    for group in ("block", "row", "tensor"):
+        for rule in ("ceil", "mse"):
+            ms = _time_ms(torch, stream, lambda: cfp.quantize_static(Wt32, "E3C3", G, group, rule, stream=stream),
+                          flush_l2, reps=3, warm=1)
+            gbs = Wt32.numel() * (4 + 1 + 1 / G) / (ms / 1e3) / 1e9
+            res["quantize_static"].append({"workload": "E3C3 W[4096x4096] ~ N(0, 0.02^2) fp32", "group": group,
+                                           "rule": rule, "ms": round(ms, 4), "gbs": round(gbs, 1)})
+    del Wt32
     # training triplet, E4C3 weights/activations, E5C2 gradients
     X, Wt, dY = inputs.training_triplet_cuda()
     gemm_case("fwd X.W", q(X, "E4C3", 0), "E4C3", q(Wt, "E4C3", 1), "E4C3", 64)

@@ -36,6 +36,7 @@
 #ifndef CURVEFP_H
 #define CURVEFP_H
 
+#include <stddef.h>
 #include <stdint.h>
 
 #ifdef __cplusplus
@@ -89,6 +90,38 @@ typedef enum {
 curvefp_status_t curvefp_quantize(curvefp_format_t fmt, int block, const void* x, curvefp_dtype_t dtype,
                                   int64_t rows, int64_t cols, int64_t ld, int block_axis, uint8_t* codes,
                                   int8_t* scales, uint32_t* device_status, void* stream);
+
+/* Static operands (Sec. 3.1: "static operands choose a representable
+ * power-of-two scale by reconstruction-MSE search"; Sec. 4.2 evaluates
+ * tensorwise, rowwise and block scaling).  A scale group is a block of
+ * `block` elements of a row, a whole row, or the whole tensor. */
+typedef enum { CURVEFP_SCALE_BLOCK = 0, CURVEFP_SCALE_ROW = 1, CURVEFP_SCALE_TENSOR = 2 } curvefp_scale_group_t;
+/* CEIL_ABSMAX: the group's ceil-absmax scale a_c (as curvefp_quantize).
+ * MSE: the candidate a in [a_c - 3, a_c + 1] (clamped to int8) with the
+ *   smallest D(a) = sum_i floor((x_i - xhat_i)^2 * 2^{60 - 2 a_c}), xhat_i the
+ *   FP32 reconstruction (as curvefp_dequantize) of x_i encoded at scale a;
+ *   D is an exact integer, so the choice is independent of summation order;
+ *   ties go to the larger a.  NaN elements are left out of D; groups with an
+ *   Inf element or an all-zero max keep a_c. */
+typedef enum { CURVEFP_SCALE_CEIL_ABSMAX = 0, CURVEFP_SCALE_MSE = 1 } curvefp_scale_rule_t;
+
+/* Bytes of device workspace curvefp_quantize_static needs (0 for block
+ * groups; a few bytes per group for rows and the tensor); 0 for bad arguments. */
+size_t curvefp_quantize_static_workspace(int64_t rows, int64_t cols, int block, curvefp_scale_group_t group);
+
+/* Quantize a static operand with one scale per group.
+ *   x      : [rows x cols] FP32 or BF16, dense (ld = cols), aligned to its element.
+ *   codes  : [rows x cols]; scales: [rows x cols/block], every block of a group
+ *            holding the group's scale (the layout every GEMM call takes).
+ *   workspace : device memory of at least curvefp_quantize_static_workspace()
+ *            bytes, 16-byte aligned, owned by the caller (contents clobbered);
+ *            may be NULL when that size is 0.
+ * Requirements: cols % block == 0.  NaN inputs encode as 0x00 and raise
+ * CURVEFP_DEV_NAN.  The library allocates nothing. */
+curvefp_status_t curvefp_quantize_static(curvefp_format_t fmt, int block, curvefp_scale_group_t group,
+                                         curvefp_scale_rule_t rule, const void* x, curvefp_dtype_t dtype, int64_t rows,
+                                         int64_t cols, uint8_t* codes, int8_t* scales, void* workspace,
+                                         size_t workspace_bytes, uint32_t* device_status, void* stream);
 
 /* Dequantization to FP32 (Eq. 1): out = RN32( RN32(2^{k/K}) * 2^{a_b + e} ) with
  * the sign applied; zero codes give +0.0.

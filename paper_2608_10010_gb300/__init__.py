@@ -43,10 +43,14 @@ def load(build_if_missing: bool = False):
         lib.curvefp_gemm.argtypes = [I, I, I, I, P, P, P, P, L, L, L, P, P, P]
         lib.curvefp_gemm_phases.argtypes = [I, I, I, P, P, P, P, L, L, L, P, P, P, P, P]
         lib.curvefp_phase_count.argtypes = [I, I]
+        lib.curvefp_quantize_static_workspace.argtypes = [L, L, I, I]
+        lib.curvefp_quantize_static_workspace.restype = ctypes.c_size_t
+        lib.curvefp_quantize_static.argtypes = [I, I, I, I, P, I, L, L, P, P, P, ctypes.c_size_t, P, P]
         lib.curvefp_status_string.argtypes = [I]
         lib.curvefp_status_string.restype = ctypes.c_char_p
         lib.curvefp_version.restype = ctypes.c_char_p
-        for f in ("curvefp_quantize", "curvefp_dequantize", "curvefp_gemm", "curvefp_gemm_phases"):
+        for f in ("curvefp_quantize", "curvefp_quantize_static", "curvefp_dequantize", "curvefp_gemm",
+                  "curvefp_gemm_phases"):
             getattr(lib, f).restype = I
         _lib = lib
     return _lib
@@ -91,6 +95,32 @@ def quantize(x, fmt, block: int = 32, block_axis: int = 0, codes=None, scales=No
     dt = {torch.float32: 0, torch.bfloat16: 1}[x.dtype]
     _check(load().curvefp_quantize(_fmt(fmt), block, _p(x), dt, rows, cols, x.stride(0), block_axis,
                                    _p(codes), _p(scales), _p(status), _stream(stream)))
+    return codes, scales
+
+
+SCALE_GROUPS = {"block": 0, "row": 1, "tensor": 2}
+SCALE_RULES = {"ceil": 0, "mse": 1}
+
+
+def quantize_static(x, fmt, block: int = 32, group: str = "block", rule: str = "mse", codes=None, scales=None,
+                    status=None, stream=None):
+    """Static-operand Q(X): one scale per block / row / tensor, chosen by
+    ceil-absmax or reconstruction-MSE search.  x [rows x cols] dense FP32/BF16
+    CUDA tensor; returns (codes [rows x cols], scales [rows x cols/block])."""
+    import torch
+
+    assert x.dim() == 2 and x.is_cuda and x.is_contiguous()
+    rows, cols = x.shape
+    if codes is None:
+        codes = torch.empty((rows, cols), dtype=torch.uint8, device=x.device)
+    if scales is None:
+        scales = torch.empty((rows, cols // block), dtype=torch.int8, device=x.device)
+    lib = load()
+    nws = lib.curvefp_quantize_static_workspace(rows, cols, block, SCALE_GROUPS[group])
+    ws = torch.empty(max(int(nws), 16), dtype=torch.uint8, device=x.device) if nws else None
+    dt = {torch.float32: 0, torch.bfloat16: 1}[x.dtype]
+    _check(lib.curvefp_quantize_static(_fmt(fmt), block, SCALE_GROUPS[group], SCALE_RULES[rule], _p(x), dt, rows, cols,
+                                       _p(codes), _p(scales), _p(ws), int(nws), _p(status), _stream(stream)))
     return codes, scales
 
 

@@ -48,6 +48,31 @@ curvefp_status_t curvefp_quantize(curvefp_format_t fmt, int block, const void* x
                                         device_status, static_cast<cudaStream_t>(stream), sm_count()));
 }
 
+size_t curvefp_quantize_static_workspace(int64_t rows, int64_t cols, int block, curvefp_scale_group_t group) {
+  if (rows <= 0 || cols <= 0 || !block_ok(block) || group < CURVEFP_SCALE_BLOCK || group > CURVEFP_SCALE_TENSOR) return 0;
+  return cfp::quantize_static_workspace(rows, cols, block, group);
+}
+
+curvefp_status_t curvefp_quantize_static(curvefp_format_t fmt, int block, curvefp_scale_group_t group,
+                                         curvefp_scale_rule_t rule, const void* x, curvefp_dtype_t dtype, int64_t rows,
+                                         int64_t cols, uint8_t* codes, int8_t* scales, void* workspace,
+                                         size_t workspace_bytes, uint32_t* device_status, void* stream) {
+  if (!fmt_ok(fmt) || !block_ok(block) || (dtype != CURVEFP_F32 && dtype != CURVEFP_BF16)) return CURVEFP_ERR_INVALID_ARG;
+  if (group < CURVEFP_SCALE_BLOCK || group > CURVEFP_SCALE_TENSOR) return CURVEFP_ERR_INVALID_ARG;
+  if (rule != CURVEFP_SCALE_CEIL_ABSMAX && rule != CURVEFP_SCALE_MSE) return CURVEFP_ERR_INVALID_ARG;
+  if (rows < 0 || cols < 0) return CURVEFP_ERR_INVALID_ARG;
+  if (rows == 0 || cols == 0) return CURVEFP_OK;
+  if (!x || !codes || !scales || cols % block != 0) return CURVEFP_ERR_INVALID_ARG;
+  const int64_t esz = dtype == CURVEFP_F32 ? 4 : 2;
+  if ((reinterpret_cast<uintptr_t>(x) % esz) != 0) return CURVEFP_ERR_INVALID_ARG;
+  const size_t need = cfp::quantize_static_workspace(rows, cols, block, group);
+  if (need && (!workspace || workspace_bytes < need || (reinterpret_cast<uintptr_t>(workspace) & 15) != 0))
+    return CURVEFP_ERR_INVALID_ARG;
+  if (rows * cols > (int64_t)1 << 40) return CURVEFP_ERR_UNSUPPORTED;
+  return from_cuda(cfp::launch_quantize_static(fmt, block, group, rule, x, dtype, rows, cols, codes, scales, workspace,
+                                               device_status, static_cast<cudaStream_t>(stream), sm_count()));
+}
+
 curvefp_status_t curvefp_dequantize(curvefp_format_t fmt, int block, const uint8_t* codes, const int8_t* scales,
                                     int64_t rows, int64_t cols, float* out, void* stream) {
   if (!fmt_ok(fmt) || !block_ok(block) || rows < 0 || cols < 0) return CURVEFP_ERR_INVALID_ARG;

@@ -8,6 +8,10 @@ namespace cfp {
 
 cudaError_t launch_quantize(int fmt, int G, const void* x, int dtype, int64_t rows, int64_t cols, int64_t ld,
                             int axis, uint8_t* codes, int8_t* scales, uint32_t* status, cudaStream_t st, int sms);
+size_t quantize_static_workspace(int64_t rows, int64_t cols, int G, int group);
+cudaError_t launch_quantize_static(int fmt, int G, int group, int rule, const void* x, int dtype, int64_t rows,
+                                   int64_t cols, uint8_t* codes, int8_t* scales, void* ws, uint32_t* status,
+                                   cudaStream_t st, int sms);
 cudaError_t launch_dequantize(int fmt, int G, const uint8_t* codes, const int8_t* scales, int64_t n, float* out,
                               cudaStream_t st, int sms);
 cudaError_t launch_gemm_exact(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,

@@ -643,6 +643,221 @@ __global__ void __launch_bounds__(256) dequantize_kernel(const uint8_t* __restri
 }
 
 // ---------------------------------------------------------------------------
+// Static operands (Sec. 3.1: "static operands choose a representable
+// power-of-two scale by reconstruction-MSE search"; Sec. 4.2: tensorwise,
+// rowwise and block scaling).  A scale group is a block of G elements, a row
+// or the whole tensor; its scale is the ceil-absmax scale a_c, or, for the MSE
+// rule, the candidate a in [a_c - 3, a_c + 1] with the smallest
+//   D(a) = sum_i floor((x_i - xhat_i)^2 2^{60 - 2 a_c}),
+// xhat_i the FP32 reconstruction (Eq. 1, RN32(RN32(2^{k/K}) 2^{a+e})) of the
+// element's nearest level at scale a; an exact integer, so the choice does
+// not depend on the order of the sum; ties go to the larger a.  NaN elements
+// are left out; groups with Inf or an all-zero max keep a_c.
+
+template <typename T>
+__device__ __forceinline__ uint32_t load_bits(const T* x, int64_t i) {
+  if constexpr (sizeof(T) == 2)
+    return (uint32_t)__ldg(reinterpret_cast<const uint16_t*>(x) + i) << 16;
+  else
+    return __float_as_uint(__ldg(reinterpret_cast<const float*>(x) + i));
+}
+
+// Eq. 1 reconstruction in FP32 of a code at scale a: one rounding of the
+// exact product RN32(2^{k/K}) 2^{a+e}.
+template <int FMT>
+__device__ __forceinline__ float recon_f32(uint32_t code, int a) {
+  using F = Fmt<FMT>;
+  const uint32_t m = code & 0x7Fu;
+  if (m == 0u) return 0.0f;
+  const int n = (int)m - F::B;
+  const int e = n >= 0 ? n / F::K : -((-n + F::K - 1) / F::K);
+  const int k = n - e * F::K;
+  const float ck = __uint_as_float(F::K == 8 ? CFP_CK_F32_K8_DEV[k] : CFP_CK_F32_K4_DEV[k]);
+  const float v = __double2float_rn(ldexp((double)ck, a + e));
+  return (code & 0x80u) ? -v : v;
+}
+
+// floor((x - xhat)^2 2^{60 - 2 ac}) exactly: x - xhat is exact in FP64 (both
+// FP32, within a factor 16 unless xhat = 0), e = M 2^{E-53}, e^2 = M^2 2^{2E-106}.
+__device__ __forceinline__ unsigned __int128 sq_term(float x, float xhat, int ac) {
+  const double e = fabs((double)x - (double)xhat);
+  if (e == 0.0) return 0;
+  int E;
+  const double fr = frexp(e, &E);
+  const unsigned long long M = (unsigned long long)ldexp(fr, 53);
+  const unsigned __int128 sq = (unsigned __int128)M * M;
+  const int sh = 2 * E - 106 + 60 - 2 * ac;
+  if (sh >= 0) return sh >= 128 ? (unsigned __int128)0 : sq << sh;
+  return sh <= -128 ? (unsigned __int128)0 : sq >> (-sh);
+}
+
+// Exact 128-bit accumulation into global memory ([lo, hi] words).
+__device__ __forceinline__ void atomic_add_u128(unsigned long long* p, unsigned __int128 v) {
+  const unsigned long long lo = (unsigned long long)v, hi = (unsigned long long)(v >> 64);
+  const unsigned long long old = atomicAdd(p, lo);
+  const unsigned long long carry = (old + lo < old) ? 1ull : 0ull;
+  if (hi + carry) atomicAdd(p + 1, hi + carry);
+}
+
+// Group statistics: max |x| as an FP32 bit pattern (NaN left out; Inf =
+// 0x7F800000), one atomic max per group and thread run.
+template <typename T>
+__global__ void __launch_bounds__(256) qs_stats_kernel(const T* __restrict__ x, int64_t n, int64_t glen,
+                                                       uint32_t* amax, uint32_t* status) {
+  bool nan = false;
+  uint32_t run = 0u;
+  int64_t run_g = -1;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t g = i / glen;
+    if (g != run_g) {
+      if (run_g >= 0 && run) atomicMax(&amax[run_g], run);
+      run_g = g;
+      run = 0u;
+    }
+    const uint32_t b = load_bits(x, i) & 0x7FFFFFFFu;
+    if (b > 0x7F800000u) nan = true;
+    else run = max(run, b);
+  }
+  if (run_g >= 0 && run) atomicMax(&amax[run_g], run);
+  if (nan && status) atomicOr(status, CURVEFP_DEV_NAN);
+}
+
+// Per group and candidate: D(a) over this thread's elements, flushed with one
+// exact 128-bit atomic add per candidate and group run.
+template <int FMT, typename T>
+__global__ void __launch_bounds__(256) qs_mse_kernel(const T* __restrict__ x, int64_t n, int64_t glen,
+                                                     const uint32_t* __restrict__ amax, unsigned long long* D) {
+  __shared__ uint32_t lut[256];
+  for (int i = threadIdx.x; i < 256; i += blockDim.x) lut[i] = __ldg(lut_src<Fmt<FMT>::K>() + i);
+  __syncthreads();
+  // each thread takes a contiguous run of elements (fewer group changes)
+  const int64_t nthreads = (int64_t)gridDim.x * blockDim.x;
+  const int64_t tid = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  const int64_t per = (n + nthreads - 1) / nthreads;
+  const int64_t i0 = tid * per, i1 = min(n, i0 + per);
+  unsigned __int128 acc[5];
+  int64_t run_g = -1;
+  int ac = 0;
+  bool search = false;
+  auto flush = [&]() {
+    if (run_g >= 0 && search)
+      for (int c = 0; c < 5; ++c)
+        if (acc[c]) atomic_add_u128(D + (run_g * 5 + c) * 2, acc[c]);
+  };
+  bool dummy = false;
+  for (int64_t i = i0; i < i1; ++i) {
+    const int64_t g = i / glen;
+    if (g != run_g) {
+      flush();
+      run_g = g;
+      const uint32_t am = amax[g];
+      ac = block_scale<FMT>(am);
+      search = am != 0u && am < 0x7F800000u;
+      for (int c = 0; c < 5; ++c) acc[c] = 0;
+    }
+    if (!search) continue;
+    const uint32_t b = load_bits(x, i);
+    if ((b & 0x7FFFFFFFu) > 0x7F800000u) continue;  // NaN: left out
+    const float xv = __uint_as_float(b);
+    for (int c = 0; c < 5; ++c) {
+      const int a = ac - 3 + c;
+      if (a < -128 || a > 127) continue;
+      const uint32_t code = encode_slow<FMT>(lut, b, a, dummy);
+      acc[c] += sq_term(xv, recon_f32<FMT>(code, a), ac);
+    }
+  }
+  flush();
+}
+
+// The group's scale: a_c, or the MSE candidate with the smallest D (ties: the
+// larger a).
+template <int FMT>
+__device__ __forceinline__ int choose_scale(uint32_t am, const unsigned long long* Dg, int rule) {
+  const int ac = block_scale<FMT>(am);
+  if (rule == 0 || am == 0u || am >= 0x7F800000u) return ac;
+  int best = ac;
+  unsigned __int128 bestD = 0;
+  bool first = true;
+  for (int c = 0; c < 5; ++c) {
+    const int a = ac - 3 + c;
+    if (a < -128 || a > 127) continue;
+    const unsigned __int128 d = ((unsigned __int128)Dg[2 * c + 1] << 64) | Dg[2 * c];
+    if (first || d <= bestD) {
+      bestD = d;
+      best = a;
+      first = false;
+    }
+  }
+  return best;
+}
+
+// Encode every element under its group's scale; scales stored per block of G.
+template <int FMT, typename T>
+__global__ void __launch_bounds__(256) qs_encode_kernel(const T* __restrict__ x, int64_t n, int64_t glen, int G,
+                                                        int rule, const uint32_t* __restrict__ amax,
+                                                        const unsigned long long* __restrict__ D, uint8_t* codes,
+                                                        int8_t* scales, uint32_t* status) {
+  __shared__ uint32_t lut[256];
+  for (int i = threadIdx.x; i < 256; i += blockDim.x) lut[i] = __ldg(lut_src<Fmt<FMT>::K>() + i);
+  __syncthreads();
+  bool nan = false;
+  int64_t run_g = -1;
+  int a = 0;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t g = i / glen;
+    if (g != run_g) {
+      run_g = g;
+      a = choose_scale<FMT>(amax[g], D ? D + g * 10 : nullptr, D ? rule : 0);
+    }
+    codes[i] = (uint8_t)encode_slow<FMT>(lut, load_bits(x, i), a, nan);
+    if (i % G == 0) scales[i / G] = (int8_t)a;
+  }
+  if (nan && status) atomicOr(status, CURVEFP_DEV_NAN);
+}
+
+// Block groups: one thread per block of G elements does everything in
+// registers (no workspace).
+template <int FMT, typename T>
+__global__ void __launch_bounds__(256) qs_block_kernel(const T* __restrict__ x, int64_t nblk, int G, int rule,
+                                                       uint8_t* codes, int8_t* scales, uint32_t* status) {
+  __shared__ uint32_t lut[256];
+  for (int i = threadIdx.x; i < 256; i += blockDim.x) lut[i] = __ldg(lut_src<Fmt<FMT>::K>() + i);
+  __syncthreads();
+  bool nan = false, dummy = false;
+  for (int64_t blk = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; blk < nblk;
+       blk += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t i0 = blk * G;
+    uint32_t am = 0u;
+    for (int i = 0; i < G; ++i) {
+      const uint32_t b = load_bits(x, i0 + i) & 0x7FFFFFFFu;
+      if (b > 0x7F800000u) nan = true;
+      else am = max(am, b);
+    }
+    unsigned long long Dg[10];
+    const bool search = rule == 1 && am != 0u && am < 0x7F800000u;
+    if (search) {
+      const int ac = block_scale<FMT>(am);
+      for (int c = 0; c < 5; ++c) {
+        const int a = ac - 3 + c;
+        unsigned __int128 d = 0;
+        if (a >= -128 && a <= 127)
+          for (int i = 0; i < G; ++i) {
+            const uint32_t b = load_bits(x, i0 + i);
+            if ((b & 0x7FFFFFFFu) > 0x7F800000u) continue;
+            d += sq_term(__uint_as_float(b), recon_f32<FMT>(encode_slow<FMT>(lut, b, a, dummy), a), ac);
+          }
+        Dg[2 * c] = (unsigned long long)d;
+        Dg[2 * c + 1] = (unsigned long long)(d >> 64);
+      }
+    }
+    const int a = choose_scale<FMT>(am, Dg, search ? 1 : 0);
+    scales[blk] = (int8_t)a;
+    for (int i = 0; i < G; ++i) codes[i0 + i] = (uint8_t)encode_slow<FMT>(lut, load_bits(x, i0 + i), a, dummy);
+  }
+  if (nan && status) atomicOr(status, CURVEFP_DEV_NAN);
+}
+
+// ---------------------------------------------------------------------------
 // Host-side launchers (called by the C ABI after argument validation).
 
 template <int FMT, typename T>
@@ -720,6 +935,56 @@ cudaError_t launch_quantize(int fmt, int G, const void* x, int dtype, int64_t ro
     case CURVEFP_E5C2: CFP_Q(CURVEFP_E5C2)
   }
 #undef CFP_Q
+  return cudaErrorInvalidValue;
+}
+
+size_t quantize_static_workspace(int64_t rows, int64_t cols, int G, int group) {
+  if (group == 0) return 0;
+  const int64_t ngroups = group == 1 ? rows : 1;
+  return (size_t)((ngroups * 4 + 15) / 16 * 16) + (size_t)ngroups * 80;
+}
+
+template <int FMT, typename T>
+static cudaError_t launch_qs_t(int G, int group, int rule, const void* xv, int64_t rows, int64_t cols, uint8_t* codes,
+                               int8_t* scales, void* ws, uint32_t* status, cudaStream_t st, int sms) {
+  const T* x = static_cast<const T*>(xv);
+  const int64_t n = rows * cols;
+  if (group == 0) {
+    const int64_t nblk = n / G;
+    int64_t grid = (nblk + 255) / 256;
+    if (grid > (int64_t)sms * 8) grid = (int64_t)sms * 8;
+    qs_block_kernel<FMT, T><<<(unsigned)(grid < 1 ? 1 : grid), 256, 0, st>>>(x, nblk, G, rule, codes, scales, status);
+    return cudaGetLastError();
+  }
+  const int64_t glen = group == 1 ? cols : n;
+  const int64_t ngroups = n / glen;
+  uint32_t* amax = static_cast<uint32_t*>(ws);
+  unsigned long long* D = reinterpret_cast<unsigned long long*>(static_cast<uint8_t*>(ws) + (ngroups * 4 + 15) / 16 * 16);
+  cudaError_t e = cudaMemsetAsync(ws, 0, quantize_static_workspace(rows, cols, G, group), st);
+  if (e != cudaSuccess) return e;
+  int64_t grid = (n + 255) / 256;
+  if (grid > (int64_t)sms * 8) grid = (int64_t)sms * 8;
+  const unsigned g = (unsigned)(grid < 1 ? 1 : grid);
+  qs_stats_kernel<T><<<g, 256, 0, st>>>(x, n, glen, amax, status);
+  if (rule == 1) qs_mse_kernel<FMT, T><<<g, 256, 0, st>>>(x, n, glen, amax, D);
+  qs_encode_kernel<FMT, T><<<g, 256, 0, st>>>(x, n, glen, G, rule, amax, rule == 1 ? D : nullptr, codes, scales,
+                                               status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_quantize_static(int fmt, int G, int group, int rule, const void* x, int dtype, int64_t rows,
+                                   int64_t cols, uint8_t* codes, int8_t* scales, void* ws, uint32_t* status,
+                                   cudaStream_t st, int sms) {
+#define CFP_QS(FMT)                                                                                            \
+  return dtype == CURVEFP_F32                                                                                  \
+             ? launch_qs_t<FMT, float>(G, group, rule, x, rows, cols, codes, scales, ws, status, st, sms)      \
+             : launch_qs_t<FMT, uint16_t>(G, group, rule, x, rows, cols, codes, scales, ws, status, st, sms);
+  switch (fmt) {
+    case CURVEFP_E3C3: CFP_QS(CURVEFP_E3C3)
+    case CURVEFP_E4C3: CFP_QS(CURVEFP_E4C3)
+    case CURVEFP_E5C2: CFP_QS(CURVEFP_E5C2)
+  }
+#undef CFP_QS
   return cudaErrorInvalidValue;
 }
 

@@ -72,6 +72,17 @@ def test_host_side_validation(lib):
     assert lib.curvefp_gemm(0, 1, 1, 32, dummy, dummy, dummy, dummy, 0, 4, 64, dummy, None, None) == INVALID
     assert lib.curvefp_gemm(7, 1, 1, 32, dummy, dummy, dummy, dummy, 4, 4, 64, dummy, None, None) == INVALID
     assert lib.curvefp_gemm_phases(1, 1, 32, dummy, dummy, dummy, dummy, 4, 4, 64, None, None, dummy, None, None) == INVALID
+    # static quantization: bad group / rule, cols not a multiple of the block,
+    # missing or short workspace for row groups; block groups need none
+    ws = lib.curvefp_quantize_static_workspace
+    assert ws(4, 64, 32, 0) == 0 and ws(4, 64, 32, 1) > 0 and ws(4, 64, 32, 2) > 0 and ws(4, 64, 32, 3) == 0
+    qs = lib.curvefp_quantize_static
+    assert qs(1, 32, 3, 1, dummy, 0, 4, 64, dummy, dummy, None, 0, None, None) == INVALID
+    assert qs(1, 32, 0, 2, dummy, 0, 4, 64, dummy, dummy, None, 0, None, None) == INVALID
+    assert qs(1, 32, 0, 1, dummy, 0, 4, 48, dummy, dummy, None, 0, None, None) == INVALID
+    assert qs(1, 32, 1, 1, dummy, 0, 4, 64, dummy, dummy, None, 0, None, None) == INVALID
+    assert qs(1, 32, 1, 1, dummy, 0, 4, 64, dummy, dummy, dummy, 8, None, None) == INVALID
+    assert qs(1, 32, 2, 1, None, 0, 0, 64, None, None, None, 0, None, None) == 0
 
 
 def test_product_path_does_not_touch_the_oracle():
