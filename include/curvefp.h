@@ -123,6 +123,24 @@ curvefp_status_t curvefp_quantize_static(curvefp_format_t fmt, int block, curvef
                                          int64_t cols, uint8_t* codes, int8_t* scales, void* workspace,
                                          size_t workspace_bytes, uint32_t* device_status, void* stream);
 
+/* curvefp_quantize_static without a workspace argument: the scratch lives
+ * in a fixed device array inside the library (CURVEFP_NOALLOC_SCRATCH_BYTES,
+ * enough for row groups of up to ~100,000 rows; tensor and block groups need
+ * almost none), so the call allocates nothing and takes nothing from the
+ * caller.  Not from the paper: an interface variant of the static quantizer.
+ *   Returns CURVEFP_ERR_UNSUPPORTED when the groups need more scratch than the
+ *   array holds.  The array is shared by every call on a device: calls must
+ *   not overlap (one stream at a time, or ordered by events).  The first call
+ *   on a device looks the array up (cudaGetSymbolAddress) and so must not be
+ *   the first call made inside a CUDA-graph capture; later calls are
+ *   capturable (one memset and three kernels).  Other arguments, results and
+ *   errors as curvefp_quantize_static. */
+#define CURVEFP_NOALLOC_SCRATCH_BYTES (8u << 20)
+curvefp_status_t curvefp_quantize_static_noalloc(curvefp_format_t fmt, int block, curvefp_scale_group_t group,
+                                                 curvefp_scale_rule_t rule, const void* x, curvefp_dtype_t dtype,
+                                                 int64_t rows, int64_t cols, uint8_t* codes, int8_t* scales,
+                                                 uint32_t* device_status, void* stream);
+
 /* Dequantization to FP32 (Eq. 1): out = RN32( RN32(2^{k/K}) * 2^{a_b + e} ) with
  * the sign applied; zero codes give +0.0.
  *   codes [rows x cols] (16-byte aligned, cols % block == 0), scales

@@ -46,11 +46,12 @@ def load(build_if_missing: bool = False):
         lib.curvefp_quantize_static_workspace.argtypes = [L, L, I, I]
         lib.curvefp_quantize_static_workspace.restype = ctypes.c_size_t
         lib.curvefp_quantize_static.argtypes = [I, I, I, I, P, I, L, L, P, P, P, ctypes.c_size_t, P, P]
+        lib.curvefp_quantize_static_noalloc.argtypes = [I, I, I, I, P, I, L, L, P, P, P, P]
         lib.curvefp_status_string.argtypes = [I]
         lib.curvefp_status_string.restype = ctypes.c_char_p
         lib.curvefp_version.restype = ctypes.c_char_p
-        for f in ("curvefp_quantize", "curvefp_quantize_static", "curvefp_dequantize", "curvefp_gemm",
-                  "curvefp_gemm_phases"):
+        for f in ("curvefp_quantize", "curvefp_quantize_static", "curvefp_quantize_static_noalloc",
+                  "curvefp_dequantize", "curvefp_gemm", "curvefp_gemm_phases"):
             getattr(lib, f).restype = I
         _lib = lib
     return _lib
@@ -121,6 +122,24 @@ def quantize_static(x, fmt, block: int = 32, group: str = "block", rule: str = "
     dt = {torch.float32: 0, torch.bfloat16: 1}[x.dtype]
     _check(lib.curvefp_quantize_static(_fmt(fmt), block, SCALE_GROUPS[group], SCALE_RULES[rule], _p(x), dt, rows, cols,
                                        _p(codes), _p(scales), _p(ws), int(nws), _p(status), _stream(stream)))
+    return codes, scales
+
+
+def quantize_static_noalloc(x, fmt, block: int = 32, group: str = "block", rule: str = "mse", codes=None,
+                            scales=None, status=None, stream=None):
+    """quantize_static through the entry point that takes no workspace (its
+    scratch is a fixed device array inside the library)."""
+    import torch
+
+    assert x.dim() == 2 and x.is_cuda and x.is_contiguous()
+    rows, cols = x.shape
+    if codes is None:
+        codes = torch.empty((rows, cols), dtype=torch.uint8, device=x.device)
+    if scales is None:
+        scales = torch.empty((rows, cols // block), dtype=torch.int8, device=x.device)
+    dt = {torch.float32: 0, torch.bfloat16: 1}[x.dtype]
+    _check(load().curvefp_quantize_static_noalloc(_fmt(fmt), block, SCALE_GROUPS[group], SCALE_RULES[rule], _p(x), dt,
+                                                  rows, cols, _p(codes), _p(scales), _p(status), _stream(stream)))
     return codes, scales
 
 

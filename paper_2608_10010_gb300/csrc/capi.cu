@@ -73,6 +73,32 @@ curvefp_status_t curvefp_quantize_static(curvefp_format_t fmt, int block, curvef
                                                device_status, static_cast<cudaStream_t>(stream), sm_count()));
 }
 
+/* Scratch for curvefp_quantize_static_noalloc: a file-scope device array
+ * (reserved when the library's module loads, never allocated by a call). */
+static __device__ __align__(256) unsigned char g_static_scratch[CURVEFP_NOALLOC_SCRATCH_BYTES];
+
+curvefp_status_t curvefp_quantize_static_noalloc(curvefp_format_t fmt, int block, curvefp_scale_group_t group,
+                                                 curvefp_scale_rule_t rule, const void* x, curvefp_dtype_t dtype,
+                                                 int64_t rows, int64_t cols, uint8_t* codes, int8_t* scales,
+                                                 uint32_t* device_status, void* stream) {
+  if (rows < 0 || cols < 0) return CURVEFP_ERR_INVALID_ARG;
+  if (rows == 0 || cols == 0) return CURVEFP_OK;
+  if (!block_ok(block) || group < CURVEFP_SCALE_BLOCK || group > CURVEFP_SCALE_TENSOR) return CURVEFP_ERR_INVALID_ARG;
+  const size_t need = cfp::quantize_static_workspace(rows, cols, block, group);
+  if (need > CURVEFP_NOALLOC_SCRATCH_BYTES) return CURVEFP_ERR_UNSUPPORTED;
+  void* scratch = nullptr;
+  if (need) {
+    // this device's copy of the array, looked up once per device
+    static void* addr[64] = {nullptr};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return CURVEFP_ERR_CUDA;
+    if (!addr[dev] && cudaGetSymbolAddress(&addr[dev], g_static_scratch) != cudaSuccess) return CURVEFP_ERR_CUDA;
+    scratch = addr[dev];
+  }
+  return curvefp_quantize_static(fmt, block, group, rule, x, dtype, rows, cols, codes, scales, scratch, need,
+                                 device_status, stream);
+}
+
 curvefp_status_t curvefp_dequantize(curvefp_format_t fmt, int block, const uint8_t* codes, const int8_t* scales,
                                     int64_t rows, int64_t cols, float* out, void* stream) {
   if (!fmt_ok(fmt) || !block_ok(block) || rows < 0 || cols < 0) return CURVEFP_ERR_INVALID_ARG;
