@@ -196,6 +196,16 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
             res["quantize_static"].append({"workload": "E3C3 W[4096x4096] ~ N(0, 0.02^2) fp32", "group": group,
                                            "rule": rule, "ms": round(ms, 4), "gbs": round(gbs, 1)})
     del Wt32
+    # the tile's Q32 integer semantics (a validation GEMM on integer ALUs)
+    Xq = torch.randn((1024, 4096), device="cuda", generator=torch.Generator(device="cuda").manual_seed(3))
+    Wq = torch.randn((1024, 4096), device="cuda", generator=torch.Generator(device="cuda").manual_seed(4)) * 0.02
+    (aq, saq), (bq, sbq) = q(Xq, "E4C3", 0), q(Wq, "E4C3", 0)
+    outq = torch.empty((1024, 1024), dtype=torch.int64, device="cuda")
+    ms = _time_ms(torch, stream, lambda: cfp.gemm_q32(aq, saq, bq, sbq, "E4C3", "E4C3", G, out=outq, stream=stream),
+                  flush_l2, reps=3, warm=1)
+    res["gemm_q32"] = {"workload": "E4C3 1024x1024x4096", "ms": round(ms, 4),
+                       "gmac_per_s": round(1024 * 1024 * 4096 / (ms / 1e3) / 1e9, 1)}
+    del Xq, Wq, aq, saq, bq, sbq, outq
     # training triplet, E4C3 weights/activations, E5C2 gradients
     X, Wt, dY = inputs.training_triplet_cuda()
     gemm_case("fwd X.W", q(X, "E4C3", 0), "E4C3", q(Wt, "E4C3", 1), "E4C3", 64)

@@ -184,6 +184,20 @@ curvefp_status_t curvefp_gemm_phases(curvefp_format_t fmt_a, curvefp_format_t fm
                                      int64_t K, float* c, int64_t* phase_sums, int32_t* phase_lsb,
                                      uint32_t* device_status, void* stream);
 
+/* The spatial tile's integer semantics as a second bit-exact GEMM (App. C.1,
+ * C.2): every nonzero product, with lattice exponent u = L e + k (as in
+ * curvefp_gemm), adds (-1)^{s_a xor s_b} round(2^{k/L} 2^16) 2^{16+e+sa+sb} to a
+ * signed 64-bit Q32 accumulator (value = acc * 2^-32), with no intermediate
+ * rounding; for E4C3 x E4C3 this is the tile's Q16 coefficient select on
+ * q_p = m_a + m_b - 128 = 8e + k followed by the shift into Q32.
+ *   acc : [M x N] int64, row-major.
+ * A product needing a shift below 0 or above 45, or an accumulator outside
+ * int64, raises CURVEFP_DEV_RANGE (that output's value is undefined).
+ * Operands, layouts and format pairs as curvefp_gemm with algo TENSOR. */
+curvefp_status_t curvefp_gemm_q32(curvefp_format_t fmt_a, curvefp_format_t fmt_b, int block, const uint8_t* a,
+                                  const int8_t* sa, const uint8_t* b, const int8_t* sb, int64_t M, int64_t N, int64_t K,
+                                  int64_t* acc, uint32_t* device_status, void* stream);
+
 /* Number of phases H of a format pair (Eq. 4 with binary radix, on the shared
  * lattice L = max(K_a, K_b)); -1 for an unknown format. */
 int curvefp_phase_count(curvefp_format_t fmt_a, curvefp_format_t fmt_b);

@@ -47,11 +47,12 @@ def load(build_if_missing: bool = False):
         lib.curvefp_quantize_static_workspace.restype = ctypes.c_size_t
         lib.curvefp_quantize_static.argtypes = [I, I, I, I, P, I, L, L, P, P, P, ctypes.c_size_t, P, P]
         lib.curvefp_quantize_static_noalloc.argtypes = [I, I, I, I, P, I, L, L, P, P, P, P]
+        lib.curvefp_gemm_q32.argtypes = [I, I, I, P, P, P, P, L, L, L, P, P, P]
         lib.curvefp_status_string.argtypes = [I]
         lib.curvefp_status_string.restype = ctypes.c_char_p
         lib.curvefp_version.restype = ctypes.c_char_p
         for f in ("curvefp_quantize", "curvefp_quantize_static", "curvefp_quantize_static_noalloc",
-                  "curvefp_dequantize", "curvefp_gemm", "curvefp_gemm_phases"):
+                  "curvefp_dequantize", "curvefp_gemm", "curvefp_gemm_phases", "curvefp_gemm_q32"):
             getattr(lib, f).restype = I
         _lib = lib
     return _lib
@@ -163,6 +164,19 @@ def gemm(a, sa, b, sb, fmt_a, fmt_b, block: int = 32, algo: str = "tensor", out=
         out = torch.empty((M, N), dtype=torch.float32, device=a.device)
     _check(load().curvefp_gemm(ALGOS[algo], _fmt(fmt_a), _fmt(fmt_b), block, _p(a), _p(sa), _p(b), _p(sb),
                                M, N, K, _p(out), _p(status), _stream(stream)))
+    return out
+
+
+def gemm_q32(a, sa, b, sb, fmt_a, fmt_b, block: int = 32, out=None, status=None, stream=None):
+    """The tile's Q32 integer accumulators [M x N] int64 (value = acc 2^-32)."""
+    import torch
+
+    M, K = a.shape
+    N = b.shape[0]
+    if out is None:
+        out = torch.empty((M, N), dtype=torch.int64, device=a.device)
+    _check(load().curvefp_gemm_q32(_fmt(fmt_a), _fmt(fmt_b), block, _p(a), _p(sa), _p(b), _p(sb), M, N, K, _p(out),
+                                   _p(status), _stream(stream)))
     return out
 
 

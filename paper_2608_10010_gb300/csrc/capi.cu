@@ -148,6 +148,18 @@ curvefp_status_t curvefp_gemm_phases(curvefp_format_t fmt_a, curvefp_format_t fm
                                           device_status, static_cast<cudaStream_t>(stream)));
 }
 
+curvefp_status_t curvefp_gemm_q32(curvefp_format_t fmt_a, curvefp_format_t fmt_b, int block, const uint8_t* a,
+                                  const int8_t* sa, const uint8_t* b, const int8_t* sb, int64_t M, int64_t N, int64_t K,
+                                  int64_t* acc, uint32_t* device_status, void* stream) {
+  curvefp_status_t r = gemm_args(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K);
+  if (r != CURVEFP_OK) return r;
+  if (!acc) return CURVEFP_ERR_INVALID_ARG;
+  if (!cfp::gemm_tensor_supported(fmt_a, fmt_b)) return CURVEFP_ERR_UNSUPPORTED;  // same format pairs
+  if ((M + 15) / 16 > 65535) return CURVEFP_ERR_UNSUPPORTED;
+  return from_cuda(cfp::launch_gemm_q32(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, acc, device_status,
+                                        static_cast<cudaStream_t>(stream)));
+}
+
 int curvefp_phase_count(curvefp_format_t fmt_a, curvefp_format_t fmt_b) {
   if (!fmt_ok(fmt_a) || !fmt_ok(fmt_b)) return -1;
   const int ka = fmt_k(fmt_a), kb = fmt_k(fmt_b);

@@ -14,6 +14,7 @@ Constants (binary radix, K in {4, 8}):
   * MU_SAT: 1 + mant/2^23 > 2^{(K-1)/K} iff mant >= MU_SAT (block scale).
   * MU_Z:   1 + mant/2^23 > 2^{1/K}    iff mant >= MU_Z   (zero boundary).
   * C_K[k]: FP32 bits of RN32(2^{k/K}) (dequantization).
+  * Q16_K[k]: round(2^{k/K} 2^16), the tile's integer coefficients (App. C.1).
   * phase constants 2^{h/L} for L in {4, 8}, as FP32 and FP64 bits.
 
 Run:  python gen_constants.py > curvefp_constants.h
@@ -58,6 +59,17 @@ def mant_threshold_fix(x_fix: int, exact: bool) -> int:
     q, r = divmod(frac, 1 << shift)
     assert 2 < r < (1 << shift) - 2, "threshold too close to an FP32 mantissa"
     return q + 1
+
+
+def q16_coeff(k: int, K: int) -> int:
+    """App. C.1 tile coefficient round(2^{k/K} 2^16) (never a tie: irrational
+    for 0 < k < K)."""
+    x = fix_pow2(k, K)
+    shift = P - 16
+    q, r = divmod(x, 1 << shift)
+    if k:
+        assert 2 < abs(r - (1 << (shift - 1))), "coefficient too close to a half"
+    return q + (1 if r >= (1 << (shift - 1)) else 0)
 
 
 def midpoint_threshold(k: int, K: int) -> int:
@@ -168,7 +180,8 @@ def main(out=sys.stdout):
         for i in range(0, 256, 8):
             w("  " + ", ".join(f"0x{v:08x}u" for v in lut[i:i + 8]) + ", \\\n")
         w("}\n")
-        w(f"#define CFP_CK_F32_K{K}_INIT {{" + ", ".join(f"0x{f32_bits_pow2(k, K):08x}u" for k in range(K)) + "}\n\n")
+        w(f"#define CFP_CK_F32_K{K}_INIT {{" + ", ".join(f"0x{f32_bits_pow2(k, K):08x}u" for k in range(K)) + "}\n")
+        w(f"#define CFP_Q16_K{K}_INIT {{" + ", ".join(f"{q16_coeff(k, K)}u" for k in range(K)) + "}\n\n")
     for name, (E, C) in FORMATS.items():
         nbin, tab = rank_table(E, C)
         w(f"#define CFP_RANK_{name}_NBIN {nbin}\n")

@@ -24,5 +24,8 @@ cudaError_t launch_gemm_tensor_sparse(int fa, int fb, int G, const uint8_t* a, c
                                       const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, uint32_t* status,
                                       cudaStream_t st);
 bool gemm_tensor_supported(int fa, int fb);
+cudaError_t launch_gemm_q32(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
+                            const int8_t* sb, int64_t M, int64_t N, int64_t K, int64_t* out, uint32_t* status,
+                            cudaStream_t s);
 
 }  // namespace cfp
