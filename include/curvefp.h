@@ -184,6 +184,21 @@ curvefp_status_t curvefp_gemm_phases(curvefp_format_t fmt_a, curvefp_format_t fm
                                      int64_t K, float* c, int64_t* phase_sums, int32_t* phase_lsb,
                                      uint32_t* device_status, void* stream);
 
+/* GEMM followed by output requantization (Sec. 3.2: closure holds on the
+ * widened product coordinates; the explicit requantization to an E-bit
+ * destination comes after the phase combine): C = A_hat B_hat^T as
+ * curvefp_gemm, then Q(C) as curvefp_quantize with blocks of block_c along N
+ * (the layout of the next layer's activation operand).
+ *   c        : [M x N] FP32 (16-byte aligned), written; the requantizer reads it
+ *              back (one extra HBM round trip of 4 M N bytes).
+ *   codes_c  : [M x N] codes of fmt_c; scales_c: [M x N/block_c].
+ * Requirements: those of both calls, and N % block_c == 0. */
+curvefp_status_t curvefp_gemm_requant(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, curvefp_format_t fmt_b,
+                                      int block, const uint8_t* a, const int8_t* sa, const uint8_t* b,
+                                      const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c,
+                                      curvefp_format_t fmt_c, int block_c, uint8_t* codes_c, int8_t* scales_c,
+                                      uint32_t* device_status, void* stream);
+
 /* The spatial tile's integer semantics as a second bit-exact GEMM (App. C.1,
  * C.2): every nonzero product, with lattice exponent u = L e + k (as in
  * curvefp_gemm), adds (-1)^{s_a xor s_b} round(2^{k/L} 2^16) 2^{16+e+sa+sb} to a

@@ -48,11 +48,13 @@ def load(build_if_missing: bool = False):
         lib.curvefp_quantize_static.argtypes = [I, I, I, I, P, I, L, L, P, P, P, ctypes.c_size_t, P, P]
         lib.curvefp_quantize_static_noalloc.argtypes = [I, I, I, I, P, I, L, L, P, P, P, P]
         lib.curvefp_gemm_q32.argtypes = [I, I, I, P, P, P, P, L, L, L, P, P, P]
+        lib.curvefp_gemm_requant.argtypes = [I, I, I, I, P, P, P, P, L, L, L, P, I, I, P, P, P, P]
         lib.curvefp_status_string.argtypes = [I]
         lib.curvefp_status_string.restype = ctypes.c_char_p
         lib.curvefp_version.restype = ctypes.c_char_p
         for f in ("curvefp_quantize", "curvefp_quantize_static", "curvefp_quantize_static_noalloc",
-                  "curvefp_dequantize", "curvefp_gemm", "curvefp_gemm_phases", "curvefp_gemm_q32"):
+                  "curvefp_dequantize", "curvefp_gemm", "curvefp_gemm_phases", "curvefp_gemm_q32",
+                  "curvefp_gemm_requant"):
             getattr(lib, f).restype = I
         _lib = lib
     return _lib
@@ -165,6 +167,26 @@ def gemm(a, sa, b, sb, fmt_a, fmt_b, block: int = 32, algo: str = "tensor", out=
     _check(load().curvefp_gemm(ALGOS[algo], _fmt(fmt_a), _fmt(fmt_b), block, _p(a), _p(sa), _p(b), _p(sb),
                                M, N, K, _p(out), _p(status), _stream(stream)))
     return out
+
+
+def gemm_requant(a, sa, b, sb, fmt_a, fmt_b, fmt_c, block: int = 32, block_c: int = 32, algo: str = "tensor",
+                 c=None, codes_c=None, scales_c=None, status=None, stream=None):
+    """C = A_hat B_hat^T and its requantization Q(C) (blocks along N).
+    Returns (c [M x N] fp32, codes_c, scales_c)."""
+    import torch
+
+    M, K = a.shape
+    N = b.shape[0]
+    if c is None:
+        c = torch.empty((M, N), dtype=torch.float32, device=a.device)
+    if codes_c is None:
+        codes_c = torch.empty((M, N), dtype=torch.uint8, device=a.device)
+    if scales_c is None:
+        scales_c = torch.empty((M, N // block_c), dtype=torch.int8, device=a.device)
+    _check(load().curvefp_gemm_requant(ALGOS[algo], _fmt(fmt_a), _fmt(fmt_b), block, _p(a), _p(sa), _p(b), _p(sb), M,
+                                       N, K, _p(c), _fmt(fmt_c), block_c, _p(codes_c), _p(scales_c), _p(status),
+                                       _stream(stream)))
+    return c, codes_c, scales_c
 
 
 def gemm_q32(a, sa, b, sb, fmt_a, fmt_b, block: int = 32, out=None, status=None, stream=None):

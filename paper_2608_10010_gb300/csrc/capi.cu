@@ -148,6 +148,18 @@ curvefp_status_t curvefp_gemm_phases(curvefp_format_t fmt_a, curvefp_format_t fm
                                           device_status, static_cast<cudaStream_t>(stream)));
 }
 
+curvefp_status_t curvefp_gemm_requant(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, curvefp_format_t fmt_b,
+                                      int block, const uint8_t* a, const int8_t* sa, const uint8_t* b,
+                                      const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c,
+                                      curvefp_format_t fmt_c, int block_c, uint8_t* codes_c, int8_t* scales_c,
+                                      uint32_t* device_status, void* stream) {
+  if (!fmt_ok(fmt_c) || !block_ok(block_c) || N % block_c != 0 || !c || !codes_c || !scales_c || !al16(c))
+    return CURVEFP_ERR_INVALID_ARG;
+  curvefp_status_t r = curvefp_gemm(algo, fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, device_status, stream);
+  if (r != CURVEFP_OK) return r;
+  return curvefp_quantize(fmt_c, block_c, c, CURVEFP_F32, M, N, N, 0, codes_c, scales_c, device_status, stream);
+}
+
 curvefp_status_t curvefp_gemm_q32(curvefp_format_t fmt_a, curvefp_format_t fmt_b, int block, const uint8_t* a,
                                   const int8_t* sa, const uint8_t* b, const int8_t* sb, int64_t M, int64_t N, int64_t K,
                                   int64_t* acc, uint32_t* device_status, void* stream) {

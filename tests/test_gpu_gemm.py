@@ -262,3 +262,29 @@ def test_ffn_sweep_small_m(torch, M):
     bs, sbs = b[cols], sb[cols]
     check_exact(torch, a, sa, bs, sbs, "E3C3", "E3C3", 32)
     check_tensor(torch, a, sa, bs, sbs, "E3C3", "E3C3", 32)
+
+
+# ---- output requantization ------------------------------------------------------
+
+@pytest.mark.parametrize("algo", ["tensor", "exact"])
+@pytest.mark.parametrize("fa,fb,fc", [("E3C3", "E3C3", "E3C3"), ("E4C3", "E4C3", "E4C3"), ("E5C2", "E4C3", "E5C2")])
+def test_gemm_requant(torch, algo, fa, fb, fc):
+    """C within tolerance of the oracle, and its requantized codes/scales
+    bit-exact with the oracle's quantization of that same FP32 C."""
+    import paper_2608_10010_gb300 as cfp
+
+    x = inputs.outlier_channels((200, 512), 3)
+    w = inputs.normal((96 * 3, 512), 4, 0.02)
+    a, sa = quantized(x, fa)
+    b, sb = quantized(w, fb)
+    st = new_status(torch)
+    c, codes, scales = cfp.gemm_requant(to_dev(torch, a), to_dev(torch, sa), to_dev(torch, b), to_dev(torch, sb),
+                                        fa, fb, fc, 32, 32, algo, status=st)
+    torch.cuda.synchronize()
+    assert status_bits(st) == 0
+    c = c.cpu().numpy()
+    ref = oracle.gemm(a, sa, b, sb, fa, fb, 32, phases=False)
+    na, nb = oracle.row_norms(a, sa, fa), oracle.row_norms(b, sb, fb)
+    assert normalised_error(c, ref["C"], na, nb) <= TOL
+    rc, rs, _ = oracle.quantize(c, fc, 32, 0)
+    assert np.array_equal(codes.cpu().numpy(), rc) and np.array_equal(scales.cpu().numpy(), rs)
