@@ -66,6 +66,8 @@ def _load():
             lib.oracle_pair_info.argtypes = [i32, i32, P, P, P]
             lib.oracle_gemm.argtypes = [i32, i32, i32, P, P, P, P, i64, i64, i64, P, P, P, P]
             lib.oracle_gemm.restype = i64
+            lib.oracle_gemm_elem.argtypes = [i32, i32, P, P, P, P, i64, i64, i64, P, P, P, P]
+            lib.oracle_gemm_elem.restype = i64
             lib.oracle_histogram.argtypes = [i32, i32, i32, P, P, P, P, i64, i32, i32, P]
             lib.oracle_row_norms.argtypes = [i32, i32, P, P, i64, i64, P]
             lib.oracle_num_threads.argtypes = []
@@ -229,6 +231,57 @@ def gemm(a, sa, b, sb, fmt_a, fmt_b, block: int = 32, phases: bool = True):
     if phases:
         out["S_raw"] = S  # int128 as (lo, hi) int64 pairs
     return out
+
+
+def operand_view(codes, scales, block: int, layout: str = "rows"):
+    """A GEMM operand with one scale per element (R13).
+
+    layout "rows": codes [R x K], scales [R x K/block] (blocked along the
+    GEMM's K).  layout "cols": codes [K x R], scales [K x R/block], a matrix
+    quantized along R and used transposed (the reused operand of a backward
+    GEMM).  Returns (codes [R x K], per-element scales [R x K])."""
+    codes = np.asarray(codes, np.uint8)
+    scales = np.asarray(scales, np.int8)
+    if layout == "rows":
+        return np.ascontiguousarray(codes), np.ascontiguousarray(np.repeat(scales, block, axis=1))
+    if layout == "cols":
+        return np.ascontiguousarray(codes.T), np.ascontiguousarray(np.repeat(scales, block, axis=1).T)
+    raise ValueError(layout)
+
+
+def gemm_elem(a, ea, b, eb, fmt_a, fmt_b, phases: bool = True):
+    """Closed-product GEMM with per-element scales (Eq. 5, R13).
+
+    a: [M x K] codes with scales ea [M x K]; b: [N x K] with eb [N x K].
+    Returns the same dict as ``gemm``."""
+    a = np.ascontiguousarray(a, np.uint8)
+    b = np.ascontiguousarray(b, np.uint8)
+    ea = np.ascontiguousarray(ea, np.int8)
+    eb = np.ascontiguousarray(eb, np.int8)
+    M, K = a.shape
+    N = b.shape[0]
+    if ea.shape != a.shape or eb.shape != b.shape or b.shape[1] != K:
+        raise ValueError("shape mismatch")
+    L = pair_info(fmt_a, fmt_b)[0]
+    C = np.empty((M, N), np.float64)
+    S = np.empty((M, N, L, 2), np.int64) if phases else None
+    lsb = np.empty((M, N), np.int32)
+    rng = np.empty((M, N), np.uint8)
+    _load().oracle_gemm_elem(
+        _fid(fmt_a), _fid(fmt_b), _ptr(a), _ptr(ea), _ptr(b), _ptr(eb), M, N, K,
+        _ptr(C), _ptr(S) if phases else None, _ptr(lsb), _ptr(rng),
+    )
+    out = {"C": C, "lsb": lsb, "range": rng.astype(bool)}
+    if phases:
+        out["S_raw"] = S
+    return out
+
+
+def gemm_oriented(a, sa, layout_a, b, sb, layout_b, fmt_a, fmt_b, block: int = 32, phases: bool = True):
+    """GEMM of two operands in either layout (see ``operand_view``)."""
+    ca, ea = operand_view(a, sa, block, layout_a)
+    cb, eb = operand_view(b, sb, block, layout_b)
+    return gemm_elem(ca, ea, cb, eb, fmt_a, fmt_b, phases)
 
 
 def int128_to_int(raw: np.ndarray) -> np.ndarray:

@@ -36,6 +36,11 @@
  *   R6 exported per-phase sums are integers S_h at the per-output LSB
  *      lambda = min_b(sa_b + sb_b) + t_min.
  *   R11, R12 static-operand scale groups and MSE-search scales (below).
+ *   R13 reused operands (Sec. 4, training GEMMs: the backward GEMMs take the
+ *      forward pass's quantized operands, one of them transposed) keep each
+ *      element's own code and block scale, so a GEMM operand may carry a
+ *      scale per element; the accumulation is Eq. 5 with per-element scales
+ *      (oracle_gemm_elem below).
  */
 #include <math.h>
 #include <stdint.h>
@@ -440,6 +445,66 @@ int64_t oracle_gemm(int ida, int idb, int G, const uint8_t* A, const int8_t* sA,
           int u = n1 * l.wa + n2 * l.wb;
           int h = floormod(u, l.L);
           int t = floordiv(u, l.L) + sA[i * nb + d / G] + sB[j * nb + d / G];
+          i128 term = (i128)1 << (t - lambda);
+          acc[h] += (s1 ^ s2) ? -term : term;
+        }
+      }
+      double c = 0.0;
+      for (int h = 0; h < l.L; ++h)
+        c += exp2((double)h / l.L) * ldexp((double)acc[h], lambda);
+      if (out_of_range) { c = NAN; bad++; }
+      C[i * N + j] = c;
+      if (S)
+        for (int h = 0; h < l.L; ++h) {
+          S[((i * N + j) * l.L + h) * 2 + 0] = (int64_t)(uint64_t)((unsigned __int128)acc[h]);
+          S[((i * N + j) * l.L + h) * 2 + 1] = (int64_t)(acc[h] >> 64);
+        }
+      if (lsb) lsb[i * N + j] = lambda;
+      if (rflag) rflag[i * N + j] = (uint8_t)out_of_range;
+    }
+  }
+  return bad;
+}
+
+/* ---- Per-element scales (R13) ----------------------------------------
+ * As oracle_gemm, with a scale per operand element: ea [M x K], eb [N x K]
+ * (int8, K contiguous).  For output (i, j) and index d:
+ *   t      = floor(u / L) + ea[i,d] + eb[j,d]
+ *   lambda = min_d (ea[i,d] + eb[j,d]) + t_min
+ * and the int128 window check takes spread = max_d - min_d of the same sum.
+ * With block scales broadcast to every element of their block this is
+ * oracle_gemm's definition (the min and max over d run over the same set of
+ * values as over blocks). */
+int64_t oracle_gemm_elem(int ida, int idb, const uint8_t* A, const int8_t* eA, const uint8_t* B,
+                         const int8_t* eB, int64_t M, int64_t N, int64_t K, double* C, int64_t* S,
+                         int32_t* lsb, uint8_t* rflag) {
+  ofmt fa, fb;
+  if (ofmt_get(ida, &fa) || ofmt_get(idb, &fb)) return -1;
+  olattice l = olattice_of(&fa, &fb);
+  int tmin, tmax;
+  otrange(&fa, &fb, &tmin, &tmax);
+  int64_t bad = 0;
+#pragma omp parallel for schedule(dynamic, 1) reduction(+ : bad)
+  for (int64_t i = 0; i < M; ++i) {
+    i128 acc[8];
+    for (int64_t j = 0; j < N; ++j) {
+      int smin = 1 << 20, smax = -(1 << 20);
+      for (int64_t d = 0; d < K; ++d) {
+        int s = eA[i * K + d] + eB[j * K + d];
+        if (s < smin) smin = s;
+        if (s > smax) smax = s;
+      }
+      int lambda = smin + tmin;
+      int out_of_range = obitlen(K) + (smax - smin) + (tmax - tmin) > 127;
+      for (int h = 0; h < l.L; ++h) acc[h] = 0;
+      if (!out_of_range) {
+        for (int64_t d = 0; d < K; ++d) {
+          int s1, n1, s2, n2;
+          if (!odecode(&fa, A[i * K + d], &s1, &n1)) continue;
+          if (!odecode(&fb, B[j * K + d], &s2, &n2)) continue;
+          int u = n1 * l.wa + n2 * l.wb;
+          int h = floormod(u, l.L);
+          int t = floordiv(u, l.L) + eA[i * K + d] + eB[j * K + d];
           i128 term = (i128)1 << (t - lambda);
           acc[h] += (s1 ^ s2) ? -term : term;
         }
