@@ -211,7 +211,25 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
     gemm_case("fwd X.W", q(X, "E4C3", 0), "E4C3", q(Wt, "E4C3", 1), "E4C3", 64)
     gemm_case("dgrad dY.W^T", q(dY, "E5C2", 0), "E5C2", q(Wt, "E4C3", 0), "E4C3", 32)
     gemm_case("wgrad dY^T.X", q(dY, "E5C2", 1), "E5C2", q(X, "E4C3", 1), "E4C3", 32)
-    del X, Wt, dY
+    # the same triplet on operands quantized once and reused (the backward
+    # GEMMs read W, X and dY in the forward pass's block orientation; the
+    # timed region includes the operand preparation kernels)
+    (qx, sx), (qw, sw), (qg, sg) = q(X, "E4C3", 0), q(Wt, "E4C3", 1), q(dY, "E5C2", 0)
+    T, din = X.shape
+    dout = Wt.shape[1]
+    for name, A, la, fa, B, lb, fb, Mx, Nx, Kx, planes in (
+            ("dgrad dY.W (reused W)", (qg, sg), "rows", "E5C2", (qw, sw), "cols", "E4C3", T, din, dout, 32),
+            ("wgrad dY^T.X (reused dY, X)", (qg, sg), "cols", "E5C2", (qx, sx), "cols", "E4C3", dout, din, T, 32)):
+        ws = torch.empty(cfp.gemm_oriented_workspace_bytes(la, lb, Mx, Nx, Kx), dtype=torch.uint8, device="cuda")
+        out = torch.empty((Mx, Nx), dtype=torch.float32, device="cuda")
+        ms = _time_ms(torch, stream, lambda: cfp.gemm_oriented(A[0], A[1], la, B[0], B[1], lb, fa, fb, G, "tensor",
+                                                               out=out, workspace=ws, stream=stream), flush_l2)
+        tops = 2.0 * Mx * Nx * Kx / (ms / 1e3) / 1e12
+        res["gemm_shapes"].append({"case": name, "M": Mx, "N": Nx, "K": Kx, "formats": f"{fa}x{fb}",
+                                   "layouts": f"{la}x{lb}", "ms": round(ms, 4), "tops": round(tops, 3),
+                                   "tensor_work_frac": round(tops * planes / fp8_peak, 4)})
+        del ws, out
+    del X, Wt, dY, qx, sx, qw, sw, qg, sg
     torch.cuda.empty_cache()
     # FFN sweep, E3C3, N = 14336
     for Kf in (4096, 3584):

@@ -184,6 +184,48 @@ curvefp_status_t curvefp_gemm_phases(curvefp_format_t fmt_a, curvefp_format_t fm
                                      int64_t K, float* c, int64_t* phase_sums, int32_t* phase_lsb,
                                      uint32_t* device_status, void* stream);
 
+/* Operand layouts of curvefp_gemm_oriented (Sec. 4, training GEMMs: the
+ * backward pass reuses the forward pass's quantized operands, one of them
+ * transposed: dgrad = Q(dY) Q(W), wgrad = Q(dY)^T Q(X)).  For an operand with
+ * R GEMM rows (R = M for A, N for B):
+ *   ROWS: codes [R x K] (K contiguous), scales [R x K/block]: quantized along
+ *         the GEMM's K, as curvefp_gemm takes it.  K % block == 0.
+ *   COLS: codes [K x R] (R contiguous), scales [K x R/block]: a matrix
+ *         quantized along R (curvefp_quantize with block_axis 0 on a [K x R]
+ *         matrix) and used transposed.  Every element keeps its own block
+ *         scale, so along a GEMM row the scale changes with k.  R % block == 0. */
+typedef enum { CURVEFP_LAYOUT_ROWS = 0, CURVEFP_LAYOUT_COLS = 1 } curvefp_layout_t;
+
+/* Bytes of device workspace curvefp_gemm_oriented needs (0 for EXACT and for
+ * ROWS x ROWS); for TENSOR with a COLS operand:
+ *   sum over operands of [R K (COLS only)] + R K + 4 R, each rounded up to 256. */
+size_t curvefp_gemm_oriented_workspace_bytes(curvefp_gemm_algo_t algo, curvefp_layout_t layout_a,
+                                             curvefp_layout_t layout_b, int64_t M, int64_t N, int64_t K);
+
+/* C = A_hat B_hat^T with each operand in either layout; every product is the
+ * closed product of Eq. 2 with both elements' own scales, accumulated per
+ * phase (Eq. 5 with per-element scales: lambda = min_k(a(i,k) + b(j,k)) +
+ * t_min, the window check on the spread of the same sums).
+ *   EXACT : integer ALUs, phase sums bit-identical to the definition;
+ *           phase_sums / phase_lsb as curvefp_gemm_phases (both or neither);
+ *           c may be NULL when phase_sums is given.  No workspace.
+ *   TENSOR: the tensor-core kernel with per-element scales (tolerance and
+ *           flush rule as curvefp_gemm TENSOR, the reference exponent of a
+ *           row being its largest element scale); phase_sums and phase_lsb
+ *           must be NULL; K % 32 == 0; workspace (256-byte aligned, at least
+ *           curvefp_gemm_oriented_workspace_bytes) receives the transposed
+ *           codes of COLS operands and a relative-scale byte per element,
+ *           written by preparation kernels on the same stream.  ROWS x ROWS
+ *           is curvefp_gemm (no workspace).
+ *   TENSOR_SPARSE: ROWS x ROWS only (CURVEFP_ERR_UNSUPPORTED otherwise).
+ * Codes pointers 16-byte aligned; M, N, K > 0. */
+curvefp_status_t curvefp_gemm_oriented(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, curvefp_format_t fmt_b,
+                                       int block, const uint8_t* a, const int8_t* sa, curvefp_layout_t layout_a,
+                                       const uint8_t* b, const int8_t* sb, curvefp_layout_t layout_b, int64_t M,
+                                       int64_t N, int64_t K, float* c, int64_t* phase_sums, int32_t* phase_lsb,
+                                       void* workspace, size_t workspace_bytes, uint32_t* device_status,
+                                       void* stream);
+
 /* GEMM followed by output requantization (Sec. 3.2: closure holds on the
  * widened product coordinates; the explicit requantization to an E-bit
  * destination comes after the phase combine): C = A_hat B_hat^T as

@@ -49,12 +49,16 @@ def load(build_if_missing: bool = False):
         lib.curvefp_quantize_static_noalloc.argtypes = [I, I, I, I, P, I, L, L, P, P, P, P]
         lib.curvefp_gemm_q32.argtypes = [I, I, I, P, P, P, P, L, L, L, P, P, P]
         lib.curvefp_gemm_requant.argtypes = [I, I, I, I, P, P, P, P, L, L, L, P, I, I, P, P, P, P]
+        lib.curvefp_gemm_oriented_workspace_bytes.argtypes = [I, I, I, L, L, L]
+        lib.curvefp_gemm_oriented_workspace_bytes.restype = ctypes.c_size_t
+        lib.curvefp_gemm_oriented.argtypes = [I, I, I, I, P, P, I, P, P, I, L, L, L, P, P, P, P, ctypes.c_size_t,
+                                              P, P]
         lib.curvefp_status_string.argtypes = [I]
         lib.curvefp_status_string.restype = ctypes.c_char_p
         lib.curvefp_version.restype = ctypes.c_char_p
         for f in ("curvefp_quantize", "curvefp_quantize_static", "curvefp_quantize_static_noalloc",
                   "curvefp_dequantize", "curvefp_gemm", "curvefp_gemm_phases", "curvefp_gemm_q32",
-                  "curvefp_gemm_requant"):
+                  "curvefp_gemm_requant", "curvefp_gemm_oriented"):
             getattr(lib, f).restype = I
         _lib = lib
     return _lib
@@ -167,6 +171,46 @@ def gemm(a, sa, b, sb, fmt_a, fmt_b, block: int = 32, algo: str = "tensor", out=
     _check(load().curvefp_gemm(ALGOS[algo], _fmt(fmt_a), _fmt(fmt_b), block, _p(a), _p(sa), _p(b), _p(sb),
                                M, N, K, _p(out), _p(status), _stream(stream)))
     return out
+
+
+LAYOUTS = {"rows": 0, "cols": 1}
+
+
+def _rows_of(x, layout):
+    """GEMM rows of an operand's code matrix, and its K."""
+    return (x.shape[0], x.shape[1]) if layout == "rows" else (x.shape[1], x.shape[0])
+
+
+def gemm_oriented_workspace_bytes(layout_a, layout_b, M, N, K, algo: str = "tensor") -> int:
+    return int(load().curvefp_gemm_oriented_workspace_bytes(ALGOS[algo], LAYOUTS[layout_a], LAYOUTS[layout_b], M, N,
+                                                            K))
+
+
+def gemm_oriented(a, sa, layout_a, b, sb, layout_b, fmt_a, fmt_b, block: int = 32, algo: str = "tensor", out=None,
+                  phases: bool = False, workspace=None, status=None, stream=None):
+    """C = A_hat B_hat^T with operands in either layout ("rows": codes [R x K]
+    blocked along K; "cols": codes [K x R] blocked along R, used transposed).
+    Returns C, or (C, phase_sums, phase_lsb) with phases=True (exact only)."""
+    import torch
+
+    M, K = _rows_of(a, layout_a)
+    N, Kb = _rows_of(b, layout_b)
+    if Kb != K:
+        raise CurveFPError("operand K mismatch")
+    c = out if out is not None else torch.empty((M, N), dtype=torch.float32, device=a.device)
+    ps = pl = None
+    if phases:
+        H = phase_count(fmt_a, fmt_b)
+        ps = torch.empty((M, N, H, 2), dtype=torch.int64, device=a.device)
+        pl = torch.empty((M, N), dtype=torch.int32, device=a.device)
+    need = gemm_oriented_workspace_bytes(layout_a, layout_b, M, N, K, algo)
+    if workspace is None and need:
+        workspace = torch.empty(need, dtype=torch.uint8, device=a.device)
+    wsb = workspace.numel() if workspace is not None else 0
+    _check(load().curvefp_gemm_oriented(ALGOS[algo], _fmt(fmt_a), _fmt(fmt_b), block, _p(a), _p(sa),
+                                        LAYOUTS[layout_a], _p(b), _p(sb), LAYOUTS[layout_b], M, N, K, _p(c), _p(ps),
+                                        _p(pl), _p(workspace), wsb, _p(status), _stream(stream)))
+    return (c, ps, pl) if phases else c
 
 
 def gemm_requant(a, sa, b, sb, fmt_a, fmt_b, fmt_c, block: int = 32, block_c: int = 32, algo: str = "tensor",

@@ -148,6 +148,57 @@ curvefp_status_t curvefp_gemm_phases(curvefp_format_t fmt_a, curvefp_format_t fm
                                           device_status, static_cast<cudaStream_t>(stream)));
 }
 
+static bool layout_ok(int l) { return l == CURVEFP_LAYOUT_ROWS || l == CURVEFP_LAYOUT_COLS; }
+
+static curvefp_status_t oriented_args(int fa, int fb, int block, const uint8_t* a, const int8_t* sa, int la,
+                                      const uint8_t* b, const int8_t* sb, int lb, int64_t M, int64_t N, int64_t K) {
+  if (!fmt_ok(fa) || !fmt_ok(fb) || !block_ok(block) || !layout_ok(la) || !layout_ok(lb))
+    return CURVEFP_ERR_INVALID_ARG;
+  if (M <= 0 || N <= 0 || K <= 0) return CURVEFP_ERR_INVALID_ARG;
+  // the blocked extent of each operand: K for ROWS, its own row count for COLS
+  if ((la == CURVEFP_LAYOUT_ROWS ? K : M) % block != 0 || (lb == CURVEFP_LAYOUT_ROWS ? K : N) % block != 0)
+    return CURVEFP_ERR_INVALID_ARG;
+  if (!a || !sa || !b || !sb || !al16(a) || !al16(b)) return CURVEFP_ERR_INVALID_ARG;
+  if (M > INT32_MAX || N > INT32_MAX || K > INT32_MAX) return CURVEFP_ERR_UNSUPPORTED;
+  return CURVEFP_OK;
+}
+
+size_t curvefp_gemm_oriented_workspace_bytes(curvefp_gemm_algo_t algo, curvefp_layout_t layout_a,
+                                             curvefp_layout_t layout_b, int64_t M, int64_t N, int64_t K) {
+  if (algo != CURVEFP_GEMM_TENSOR || !layout_ok(layout_a) || !layout_ok(layout_b) || M <= 0 || N <= 0 || K <= 0)
+    return 0;
+  return cfp::gemm_reuse_workspace(layout_a, layout_b, M, N, K);
+}
+
+curvefp_status_t curvefp_gemm_oriented(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, curvefp_format_t fmt_b,
+                                       int block, const uint8_t* a, const int8_t* sa, curvefp_layout_t layout_a,
+                                       const uint8_t* b, const int8_t* sb, curvefp_layout_t layout_b, int64_t M,
+                                       int64_t N, int64_t K, float* c, int64_t* phase_sums, int32_t* phase_lsb,
+                                       void* workspace, size_t workspace_bytes, uint32_t* device_status,
+                                       void* stream) {
+  curvefp_status_t r = oriented_args(fmt_a, fmt_b, block, a, sa, layout_a, b, sb, layout_b, M, N, K);
+  if (r != CURVEFP_OK) return r;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (algo == CURVEFP_GEMM_EXACT) {
+    if (!c && !phase_sums) return CURVEFP_ERR_INVALID_ARG;
+    if (!phase_sums != !phase_lsb) return CURVEFP_ERR_INVALID_ARG;
+    return from_cuda(cfp::launch_gemm_exact_oriented(fmt_a, fmt_b, block, a, sa, layout_a, b, sb, layout_b, M, N, K,
+                                                     c, phase_sums, phase_lsb, device_status, st));
+  }
+  if (phase_sums || phase_lsb || !c) return CURVEFP_ERR_INVALID_ARG;
+  if (layout_a == CURVEFP_LAYOUT_ROWS && layout_b == CURVEFP_LAYOUT_ROWS)
+    return curvefp_gemm(algo, fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, device_status, stream);
+  if (algo == CURVEFP_GEMM_TENSOR_SPARSE) return CURVEFP_ERR_UNSUPPORTED;
+  if (algo != CURVEFP_GEMM_TENSOR) return CURVEFP_ERR_INVALID_ARG;
+  if (!cfp::gemm_tensor_supported(fmt_a, fmt_b)) return CURVEFP_ERR_UNSUPPORTED;
+  if (K % 32 != 0) return CURVEFP_ERR_INVALID_ARG;
+  const size_t need = cfp::gemm_reuse_workspace(layout_a, layout_b, M, N, K);
+  if (!workspace || workspace_bytes < need || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
+    return CURVEFP_ERR_INVALID_ARG;
+  return from_cuda(cfp::launch_gemm_tensor_reuse(fmt_a, fmt_b, block, a, sa, layout_a, b, sb, layout_b, M, N, K, c,
+                                                 workspace, device_status, st));
+}
+
 curvefp_status_t curvefp_gemm_requant(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, curvefp_format_t fmt_b,
                                       int block, const uint8_t* a, const int8_t* sa, const uint8_t* b,
                                       const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c,

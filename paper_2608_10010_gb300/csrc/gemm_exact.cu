@@ -156,6 +156,150 @@ __global__ void __launch_bounds__(NT) gemm_exact_kernel(const uint8_t* __restric
   if (phase_lsb) phase_lsb[o] = lambda;
 }
 
+// ---------------------------------------------------------------------------
+// Operands with a scale per element (reused operands of the training GEMMs):
+// element (r, k) of an operand view is code c[r cr + k ck] with scale
+// s[(r >> rsh) sr + (k >> ksh) sk]; ROWS and COLS layouts are two settings of
+// the strides.  Every product adds delta 2^{t - lambda} (t includes both
+// element scales) to an exact int128 phase sum in shared memory; lambda =
+// min_k (a(i,k) + b(j,k)) + t_min as for block scales.
+struct OpView {
+  const uint8_t* c;
+  int64_t cr, ck;
+  const int8_t* s;
+  int64_t sr, sk;
+  int rsh, ksh;
+  __device__ __forceinline__ uint8_t code(int64_t r, int64_t k) const { return __ldg(c + r * cr + k * ck); }
+  __device__ __forceinline__ int scale(int64_t r, int64_t k) const {
+    return (int)__ldg(s + (r >> rsh) * sr + (k >> ksh) * sk);
+  }
+};
+
+template <int FA, int FB>
+__global__ void __launch_bounds__(NT) gemm_exact_view_kernel(const OpView va, const OpView vb, int M, int N, int K,
+                                                             float* __restrict__ C, int64_t* __restrict__ phase_sums,
+                                                             int32_t* __restrict__ phase_lsb, uint32_t* status) {
+  using P = Pair<FA, FB>;
+  constexpr int L = P::L;
+  constexpr int DT = P::TMAX - P::TMIN;
+  constexpr uint32_t MA = Fmt<FA>::MMASK, MB = Fmt<FB>::MMASK;
+  __shared__ uint8_t Ac[TM][KC], Bc[TN][KC];
+  __shared__ int8_t As[TM][KC], Bs[TN][KC];
+  __shared__ __int128 acc[L][NT];
+
+  const int tid = threadIdx.x;
+  const int ty = tid / TN, tx = tid % TN;
+  const int i = blockIdx.y * TM + ty, j = blockIdx.x * TN + tx;
+  const bool live = i < M && j < N;
+
+  // stage a 16 x 32 tile of codes and scales of each operand; the index
+  // order follows the contiguous direction of the layout
+  auto stage = [&](int k0, bool codes) {
+    for (int e = tid; e < 2 * TM * KC; e += NT) {
+      const bool is_b = e >= TM * KC;
+      const int f = e - (is_b ? TM * KC : 0);
+      const OpView& v = is_b ? vb : va;
+      const int rr = v.ck == 1 ? f / KC : f % TM, kk = v.ck == 1 ? f % KC : f / TM;
+      const int64_t r = (int64_t)(is_b ? blockIdx.x * TN : blockIdx.y * TM) + rr;
+      const bool in = r < (is_b ? N : M) && k0 + kk < K;
+      if (codes) (is_b ? Bc : Ac)[rr][kk] = in ? v.code(r, k0 + kk) : (uint8_t)0;
+      (is_b ? Bs : As)[rr][kk] = in ? (int8_t)v.scale(r, k0 + kk) : (int8_t)0;
+    }
+  };
+
+  int smin = 1 << 20, smax = -(1 << 20);
+  for (int k0 = 0; k0 < K; k0 += KC) {
+    __syncthreads();
+    stage(k0, false);
+    __syncthreads();
+    if (live)
+      for (int kk = 0; kk < KC && k0 + kk < K; ++kk) {
+        const int s = (int)As[ty][kk] + (int)Bs[tx][kk];
+        smin = min(smin, s);
+        smax = max(smax, s);
+      }
+  }
+  const bool in_range = live && i128_bitlen_ok(smax - smin, DT, K);
+  if (live && !in_range && status) atomicOr(status, CURVEFP_DEV_RANGE);
+#pragma unroll
+  for (int h = 0; h < L; ++h) acc[h][tid] = 0;
+
+  for (int k0 = 0; k0 < K; k0 += KC) {
+    __syncthreads();
+    stage(k0, true);
+    __syncthreads();
+    if (!in_range) continue;
+    for (int kk = 0; kk < KC && k0 + kk < K; ++kk) {
+      const uint32_t ca = Ac[ty][kk], cb = Bc[tx][kk];
+      const uint32_t ma = ca & MA, mb = cb & MB;
+      if (ma == 0u || mb == 0u) continue;
+      const uint32_t u = ma * P::WA + mb * P::WB;
+      const int sh = (int)(u >> P::LOG2L) + (int)As[ty][kk] + (int)Bs[tx][kk] - smin;
+      const __int128 term = (__int128)1 << sh;
+      acc[u & (L - 1)][tid] += ((ca ^ cb) & 0x80u) ? -term : term;
+    }
+  }
+
+  if (!live) return;
+  const int lambda = smin + P::TMIN;
+  const int64_t o = (int64_t)i * N + j;
+  if (C) {
+    float out;
+    if (in_range) {
+      double c = 0.0;
+#pragma unroll
+      for (int h = 0; h < L; ++h) {
+        const double sd = i128_to_double(acc[h][tid]);
+        const uint64_t cb = L == 8 ? CFP_PHASE_F64_L8_DEV[h] : CFP_PHASE_F64_L4_DEV[h];
+        c = fma(__longlong_as_double((long long)cb), sd, c);
+      }
+      out = (float)scalbn(c, lambda);
+    } else {
+      out = __int_as_float(0x7fc00000);
+    }
+    C[o] = out;
+  }
+  if (phase_sums) {
+#pragma unroll
+    for (int h = 0; h < L; ++h) {
+      const __int128 v = acc[h][tid];
+      phase_sums[(o * L + h) * 2 + 0] = (int64_t)(uint64_t)v;
+      phase_sums[(o * L + h) * 2 + 1] = (int64_t)(v >> 64);
+    }
+  }
+  if (phase_lsb) phase_lsb[o] = lambda;
+}
+
+static OpView view_of(int layout, const uint8_t* c, const int8_t* s, int64_t R, int64_t K, int G) {
+  int g = 0;
+  while ((1 << g) < G) ++g;
+  if (layout == CURVEFP_LAYOUT_ROWS) return OpView{c, K, 1, s, K >> g, 1, 0, g};
+  return OpView{c, 1, R, s, 1, R >> g, g, 0};
+}
+
+cudaError_t launch_gemm_exact_oriented(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, int la,
+                                       const uint8_t* b, const int8_t* sb, int lb, int64_t M, int64_t N, int64_t K,
+                                       float* c, int64_t* ps, int32_t* pl, uint32_t* st, cudaStream_t s) {
+  const OpView va = view_of(la, a, sa, M, K, G), vb = view_of(lb, b, sb, N, K, G);
+  dim3 grid((unsigned)((N + TN - 1) / TN), (unsigned)((M + TM - 1) / TM));
+#define CFP_V(X, Y)                                                                                        \
+  if (fa == X && fb == Y) {                                                                                \
+    gemm_exact_view_kernel<X, Y><<<grid, NT, 0, s>>>(va, vb, (int)M, (int)N, (int)K, c, ps, pl, st);       \
+    return cudaGetLastError();                                                                             \
+  }
+  CFP_V(CURVEFP_E3C3, CURVEFP_E3C3)
+  CFP_V(CURVEFP_E3C3, CURVEFP_E4C3)
+  CFP_V(CURVEFP_E3C3, CURVEFP_E5C2)
+  CFP_V(CURVEFP_E4C3, CURVEFP_E3C3)
+  CFP_V(CURVEFP_E4C3, CURVEFP_E4C3)
+  CFP_V(CURVEFP_E4C3, CURVEFP_E5C2)
+  CFP_V(CURVEFP_E5C2, CURVEFP_E3C3)
+  CFP_V(CURVEFP_E5C2, CURVEFP_E4C3)
+  CFP_V(CURVEFP_E5C2, CURVEFP_E5C2)
+#undef CFP_V
+  return cudaErrorInvalidValue;
+}
+
 template <int FA, int FB>
 static cudaError_t launch_exact_t(int G, const uint8_t* a, const int8_t* sa, const uint8_t* b, const int8_t* sb,
                                   int64_t M, int64_t N, int64_t K, float* c, int64_t* ps, int32_t* pl, uint32_t* st,

@@ -1,0 +1,481 @@
+// Tensor-core closed-product GEMM (tcgen05, sm_103a): phase-plane
+// decomposition with per-phase FP32 accumulation in TMEM and the phase
+// combine fused into the epilogue (Sec. 3.2, Eq. 2, Eq. 5).
+//
+// Decomposition.  Write every decoded operand element as
+//   x = 2^{k/K} * X_k,   X_k = +-2^{a_b - ref + e}  (an exact power of two),
+// i.e. split each operand into K "curve planes" that hold the element in the
+// plane of its curve index k and zero elsewhere.  Plane k1 of A times plane k2
+// of B lands on the single phase h = (k1 WA + k2 WB) mod L with carry
+// c = floor((k1 WA + k2 WB) / L) (Eq. 2 on the shared lattice L), so
+//   S_h = sum_{k1,k2 : phase h} 2^c  A_{k1} B_{k2}^T,
+// a sum of dense products of power-of-two matrices, which the tensor cores
+// multiply without rounding; only the FP32 accumulation in TMEM rounds.  Block
+// scales enter the plane values as 2^{a_b - ref} (ref = largest block scale of
+// the row) and 2^{ref_i + ref_j} is applied in the epilogue.  Plane values are
+// BF16 or FP8 E5M2 (every power of two in [2^-16, 2^15] is exact in E5M2; E5C2
+// planes are stored one binade low so that the carry still fits).
+//
+// Shape.  A CTA owns a 128 x 96 tile of C.  A 128 x 96 x 32 FP8 MMA runs at
+// the full tensor rate (the per-instruction floor is ~45 cycles, this shape
+// takes 48); TMEM (512 columns) holds four 96-column phase accumulators plus
+// two steps of A planes, so the L phases are processed in passes of PP = 4
+// phases over the whole K; each pass adds its part of sum_h 2^{h/L} S_h to C.
+//
+// Roles (480 threads):
+//   warps 0-7   A producers (two threads per row, 16 codes each per step):
+//               codes -> planes in registers -> TMEM (tcgen05.st); A is the
+//               TMEM operand of the MMA and costs no shared-memory bandwidth.
+//               At the end of each pass they run the epilogue.
+//   warps 8-13  B producers (two threads per row): codes -> the planes (and
+//               x2 carry planes) that the current pass needs -> shared memory,
+//               K-major core-matrix layout.
+//   warp 14     TMEM allocation and MMA issue (one elected lane of the
+//               converged warp).
+// One mbarrier hand-off per pipeline step and operand: every wait and commit
+// sits on the path between two MMAs, so the stages are whole steps.  Every
+// wait is bounded.
+#pragma once
+#include "cfp_common.cuh"
+#include "kernels.cuh"
+#include "tc_planes.cuh"
+#include "tc_ptx.cuh"
+
+#ifndef CFP_TC_ATPR
+#define CFP_TC_ATPR 2  // A producer threads per row (2 or 4)
+#endif
+
+#ifndef CFP_TC_PLANE
+#define CFP_TC_PLANE 1  // 0: BF16 planes (K = 16 per MMA), 1: E5M2 planes (K = 32 per MMA)
+#endif
+
+namespace cfp {
+
+namespace {
+
+template <int FA, int FB, int PT>
+struct TcCfg {
+  using P = Pair<FA, FB>;
+  static constexpr int KA = Fmt<FA>::K, KB = Fmt<FB>::K, L = P::L, WA = P::WA, WB = P::WB, LOG2L = P::LOG2L;
+  static constexpr int FA_ = FA, FB_ = FB;
+  static constexpr int BM = 128;
+  static constexpr int KS = PT == PLANE_BF16 ? 16 : 32;  // K per MMA = K per pipeline step (32 bytes per row)
+  // Columns per CTA (= MMA N) and phases per pass: 4 accumulators of 96
+  // columns leave 128 TMEM columns for A; N = 96 still runs the MMA at full
+  // rate (the per-instruction floor is ~45 cycles, a 128x96x32 FP8 MMA is 48).
+  static constexpr int BN = 96;
+  static constexpr int PP = 4;                            // phases per pass
+  static constexpr int NP = (L + PP - 1) / PP;            // passes
+  static constexpr int ACC_COLS = PP * BN;
+  // A planes of a step occupy AU_COLS TMEM columns (8 per plane); two steps
+  // rotate (NAU units).
+  static constexpr int AU_COLS = KA * 8;
+  static constexpr int NAU = 2;
+  static constexpr int ACOL0 = ACC_COLS;
+  static_assert(ACC_COLS + NAU * AU_COLS <= 512, "TMEM budget");
+  static constexpr int PLANE_BYTES = BN * 32;             // 128 rows x 32 bytes
+  static constexpr int NSB = 4;                           // B stages
+  static constexpr int PBA = FA == CURVEFP_E5C2 ? 1 : 0;  // plane exponent bias
+  static constexpr int PBB = FB == CURVEFP_E5C2 ? 1 : 0;
+  static constexpr int ATPR = CFP_TC_ATPR;                // A producer threads per row
+  static constexpr int NAW = 4 * ATPR;                    // A producer warps (4 TMEM lane groups)
+  static constexpr int NWA = 8 / ATPR;                    // TMEM columns per A thread and plane
+  static constexpr int NBT = 2 * BN;                      // B producer threads (two per row)
+  static constexpr int THREADS = NAW * 32 + NBT + 32;     // A producers, B producers, MMA warp
+  static constexpr int MMA_WARP = (NAW * 32 + NBT) / 32;
+  static_assert(NBT % 32 == 0 && BN % (8 * ATPR) == 0 && 8 % ATPR == 0, "producer warps");
+  // D = F32, A = B = BF16 (kind::f16) or E5M2 (kind::f8f6f4): same bit pattern
+  static constexpr uint32_t IDESC = tc::idesc_bf16_f32(BM, BN);
+
+  __host__ __device__ static constexpr int phase(int k1, int k2) { return (k1 * WA + k2 * WB) & (L - 1); }
+  __host__ __device__ static constexpr int carry(int k1, int k2) { return (k1 * WA + k2 * WB) >> LOG2L; }
+  // Does pass p need B plane (k2, c)?
+  __host__ __device__ static constexpr bool needed(int p, int c, int k2) {
+    for (int k1 = 0; k1 < KA; ++k1)
+      if (carry(k1, k2) == c && phase(k1, k2) / PP == p) return true;
+    return false;
+  }
+  // Shared-memory slot of B plane (k2, c) in pass p (-1 if unused).
+  __host__ __device__ static constexpr int slot(int p, int c, int k2) {
+    int s = 0;
+    for (int cc = 0; cc < 2; ++cc)
+      for (int k = 0; k < KB; ++k) {
+        const bool need = needed(p, cc, k);
+        if (cc == c && k == k2) return need ? s : -1;
+        if (need) ++s;
+      }
+    return -1;
+  }
+  __host__ __device__ static constexpr int nslots(int p) {
+    int s = 0;
+    for (int cc = 0; cc < 2; ++cc)
+      for (int k = 0; k < KB; ++k) s += needed(p, cc, k) ? 1 : 0;
+    return s;
+  }
+  __host__ __device__ static constexpr int maxslots() {
+    int m = 0;
+    for (int p = 0; p < NP; ++p) m = nslots(p) > m ? nslots(p) : m;
+    return m;
+  }
+  // Is (k1, k2) the first pair of the issue order that lands on its phase?
+  __host__ __device__ static constexpr bool first_of_phase(int k1, int k2) {
+    for (int a = 0; a < KA; ++a)
+      for (int b = 0; b < KB; ++b)
+        if (phase(a, b) == phase(k1, k2)) return a == k1 && b == k2;
+    return false;
+  }
+  static constexpr int MAXS = maxslots();
+  static constexpr int BSTAGE = MAXS * PLANE_BYTES;
+  static constexpr size_t SMEM = (size_t)NSB * BSTAGE + 2048;
+};
+
+// One 16-byte core-matrix row (chunk kc of the run) of every B plane the pass needs.
+template <class Cfg, int PT, int PASS>
+__device__ __forceinline__ void write_b_planes(uint8_t* stage, int row, int kc, const uint32_t (&v)[4],
+                                               const uint32_t (&vc)[4], const uint32_t (&mk)[4][3]) {
+  constexpr int KBITS = Fmt<Cfg::FB_>::C;
+  const uint32_t core = (uint32_t)((row >> 3) * 256 + kc * 128 + (row & 7) * 16);
+#pragma unroll
+  for (int c = 0; c < 2; ++c) {
+    bool any = false;
+#pragma unroll
+    for (int k2 = 0; k2 < Cfg::KB; ++k2) any = any || Cfg::slot(PASS, c, k2) >= 0;
+    if (!any) continue;
+    uint32_t pw[4][8];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) planes_of<KBITS>(c ? vc[q] : v[q], mk[q], pw[q]);
+#pragma unroll
+    for (int k2 = 0; k2 < Cfg::KB; ++k2) {
+      const int sl = Cfg::slot(PASS, c, k2);
+      if (sl < 0) continue;
+      *reinterpret_cast<uint4*>(stage + (size_t)sl * Cfg::PLANE_BYTES + core) =
+          make_uint4(pw[0][k2], pw[1][k2], pw[2][k2], pw[3][k2]);
+    }
+  }
+}
+
+template <class Cfg, int PT, int PASS>
+__device__ __forceinline__ void issue_pass(uint32_t leader, uint32_t tmem, uint64_t bdesc0, int abuf, int bstage,
+                                           bool first_step) {
+#pragma unroll
+  for (int k1 = 0; k1 < Cfg::KA; ++k1)
+#pragma unroll
+    for (int k2 = 0; k2 < Cfg::KB; ++k2) {
+      const int h = Cfg::phase(k1, k2);
+      if (h / Cfg::PP != PASS) continue;
+      const int sl = Cfg::slot(PASS, Cfg::carry(k1, k2), k2);
+      const uint32_t a_t = tmem + Cfg::ACOL0 + abuf * Cfg::AU_COLS + k1 * 8;
+      const uint64_t bd = bdesc0 + (uint64_t)((bstage * Cfg::BSTAGE + sl * Cfg::PLANE_BYTES) >> 4);
+      const uint32_t d_t = tmem + (h - PASS * Cfg::PP) * Cfg::BN;
+      const uint32_t accum = (first_step && Cfg::first_of_phase(k1, k2)) ? 0u : 1u;
+      if (PT == PLANE_BF16)
+        tc::mma_f16_ts_if(leader, d_t, a_t, bd, Cfg::IDESC, accum);
+      else
+        tc::mma_f8_ts_if(leader, d_t, a_t, bd, Cfg::IDESC, accum);
+    }
+}
+
+template <class Cfg, int PT>
+__device__ __forceinline__ void issue_step(uint32_t leader, int p, uint32_t tmem, uint64_t bdesc0, int abuf,
+                                           int bstage, bool first_step) {
+  if (p == 0) issue_pass<Cfg, PT, 0>(leader, tmem, bdesc0, abuf, bstage, first_step);
+  if (Cfg::NP > 1 && p == 1) issue_pass<Cfg, PT, (Cfg::NP > 1 ? 1 : 0)>(leader, tmem, bdesc0, abuf, bstage, first_step);
+  if (Cfg::NP > 2 && p == 2) issue_pass<Cfg, PT, (Cfg::NP > 2 ? 2 : 0)>(leader, tmem, bdesc0, abuf, bstage, first_step);
+}
+
+}  // namespace
+
+// Per-element scales of both operands (PES = true; reused operands of the
+// training GEMMs): dp[r][k] = max(a(r,k) - ref, -64) + 64 beside the codes,
+// and the row reference ref = max_k a(r,k) read as refs[r >> rsh].
+struct PesOperands {
+  const uint8_t* dA;
+  const uint8_t* dB;
+  const int* refA;
+  const int* refB;
+  int rshA, rshB;
+};
+
+// Thread layout: warps 0 .. NAW-1 produce A (warp w: TMEM lane group w & 3,
+// share w >> 2 of each 32-byte run: NWA columns per plane) and run the
+// epilogue (columns [BN/ATPR share, BN/ATPR (share + 1))); the next 2 BN
+// threads produce B (thread 32 NAW + t: row t % BN, half t / BN); the last
+// warp allocates TMEM and issues the MMAs.
+template <int FA, int FB, int PT, bool PES>
+__global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(const uint8_t* __restrict__ A, const int8_t* __restrict__ sA,
+                                                         const uint8_t* __restrict__ B, const int8_t* __restrict__ sB,
+                                                         int M, int N, int K, int G, int gshift,
+                                                         float* __restrict__ C, uint32_t* status,
+                                                         const PesOperands pes) {
+  using Cfg = TcCfg<FA, FB, PT>;
+  constexpr int L = Cfg::L, PP = Cfg::PP, NP = Cfg::NP, BN = Cfg::BN, NSB = Cfg::NSB;
+  constexpr int NAW = Cfg::NAW, NWA = Cfg::NWA, ATPR = Cfg::ATPR;
+  constexpr int CB = PT == PLANE_E5M2 ? 4 : 2;  // code bytes per TMEM column / value word
+  static_assert(NP <= 3, "pass dispatch");
+  static_assert(NSB == TC_MAX_RING && Cfg::NAU == 2, "barrier rings");
+  extern __shared__ __align__(1024) uint8_t smem[];
+  uint8_t* bstage = smem;
+  TcShared& sh = *reinterpret_cast<TcShared*>(smem + (size_t)NSB * Cfg::BSTAGE);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int m0 = blockIdx.y * Cfg::BM, n0 = blockIdx.x * BN;
+  const int nb = K / G, nsub = K / Cfg::KS, total = NP * nsub;
+
+  if (tid == 0) {
+    for (int s = 0; s < NSB; ++s) {
+      tc::mbar_init(&sh.full[s], NAW + Cfg::NBT / 32);  // one arrival per producer warp
+      tc::mbar_init(&sh.empty[s], 1);
+    }
+    tc::mbar_init(&sh.acc_full, 1);
+    tc::mbar_init(&sh.drain, 1);
+    sh.abort_flag = 0;
+  }
+  if (warp == Cfg::MMA_WARP) {
+    tc::tmem_alloc(&sh.tmem_base, 512);
+    tc::tmem_relinquish();
+  }
+  // producer geometry and the row's reference exponent (largest block scale)
+  const bool is_a = warp < NAW;
+  const bool is_prod = warp < Cfg::MMA_WARP;
+  const int rloc = is_a ? ((warp & 3) * 32 + lane) : ((tid - NAW * 32) % BN);
+  const int part = is_a ? (warp >> 2) : ((tid - NAW * 32) / BN);  // share of the 32-byte run
+  const int r = (is_a ? m0 : n0) + rloc;
+  const bool rowok = is_prod && r < (is_a ? M : N);
+  int ref = -128;
+  if (PES) {
+    if (rowok) ref = __ldg(is_a ? pes.refA + (r >> pes.rshA) : pes.refB + (r >> pes.rshB));
+  } else if (rowok) {
+    const int8_t* s = (is_a ? sA : sB) + (int64_t)r * nb;
+    if ((nb & 15) == 0 && (reinterpret_cast<uintptr_t>(s) & 15) == 0) {
+      // 16 scales per load, all loads in flight at once, byte-wise signed max
+      uint32_t m4 = 0x80808080u;
+#pragma unroll 8
+      for (int b = 0; b < nb; b += 16) {
+        const uint4 q = __ldg(reinterpret_cast<const uint4*>(s + b));
+        m4 = __vmaxs4(m4, __vmaxs4(__vmaxs4(q.x, q.y), __vmaxs4(q.z, q.w)));
+      }
+      ref = max(max((int)(int8_t)(m4 & 0xFF), (int)(int8_t)((m4 >> 8) & 0xFF)),
+                max((int)(int8_t)((m4 >> 16) & 0xFF), (int)(int8_t)(m4 >> 24)));
+    } else {
+#pragma unroll 8
+      for (int b = 0; b < nb; ++b) ref = max(ref, (int)__ldg(s + b));
+    }
+  }
+  if (!is_a && is_prod && part == 0) sh.refB[rloc] = ref;
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = sh.tmem_base;
+
+  if (is_prod) {
+    // ------------------------------ producers ------------------------------
+    const uint8_t* src = (is_a ? A : B) + (int64_t)r * K + part * (is_a ? NWA : 4) * CB;
+    const uint8_t* dsrc = PES ? (is_a ? pes.dA : pes.dB) + (int64_t)r * K + part * (is_a ? NWA : 4) * CB : nullptr;
+    const int8_t* srow = (is_a ? sA : sB) + (int64_t)r * nb;
+    const int bias = is_a ? Cfg::PBA : Cfg::PBB;
+    auto pass_of = [&](int g) { return (NP > 1 && g >= nsub ? 1 : 0) + (NP > 2 && g >= 2 * nsub ? 1 : 0); };
+    auto load = [&](int g, uint4& cw, int& off, uint4& dw) {
+      cw = make_uint4(0, 0, 0, 0);
+      dw = make_uint4(0, 0, 0, 0);
+      off = 0;
+      if (rowok && g < total) {
+        const int s = g - pass_of(g) * nsub;
+        const uint8_t* p = src + (int64_t)s * Cfg::KS;
+        const int nbytes = (is_a ? NWA : 4) * CB;  // 16, 8 or 4
+        if (nbytes == 16) {
+          cw = __ldg(reinterpret_cast<const uint4*>(p));
+        } else if (nbytes == 8) {
+          const uint2 t = __ldg(reinterpret_cast<const uint2*>(p));
+          cw.x = t.x;
+          cw.y = t.y;
+        } else {
+          cw.x = __ldg(reinterpret_cast<const uint32_t*>(p));
+        }
+        if (PES)
+          dw = __ldg(reinterpret_cast<const uint4*>(dsrc + (int64_t)s * Cfg::KS));  // 16 relative scales
+        else
+          off = (int)__ldg(srow + (s >> gshift));  // raw scale: consumed two steps later
+      }
+    };
+    const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+    // One pipeline step of this producer thread; false ends the loop (abort).
+    auto step = [&](const int g, const uint4 cw, const int raw_scale, const uint4 dw) -> bool {
+      const int off = raw_scale - ref - bias;
+      const int p = pass_of(g), s = g - p * nsub;
+      if (is_a) {
+        uint32_t v[NWA], vc[NWA], mk[NWA][3];
+        if constexpr (PES)
+          decode_words_pes<FA, NWA>(cw, dw, bias, v, vc, mk, false);
+        else
+          decode_words<FA, PT, NWA>(cw, off, v, vc, mk, false);
+        uint32_t pl[NWA][8];
+#pragma unroll
+        for (int c = 0; c < NWA; ++c) planes_of<Fmt<FA>::C>(v[c], mk[c], pl[c]);
+        const int buf = g & 1;
+        if (g >= 2) {
+          // warp-uniform outcome: the TMEM stores below are warp-collective
+          const int gr = g - 2;
+          const bool ok = __all_sync(0xffffffffu, tc::mbar_wait(&sh.empty[gr % NSB], (gr / NSB) & 1));
+          tc::fence_after_sync();
+          if (!ok) {
+            if (lane == 0) raise_flag(status, CURVEFP_DEV_TIMEOUT);
+            sh.abort_flag = 1;
+            return false;
+          }
+        }
+        // plane k1 occupies 8 columns of the unit; this thread's share of
+        // the 32-byte run is columns NWA part .. NWA part + NWA - 1
+#pragma unroll
+        for (int j = 0; j < Cfg::KA; ++j) {
+          uint32_t reg[NWA];
+#pragma unroll
+          for (int c = 0; c < NWA; ++c) reg[c] = pl[c][j];
+          const uint32_t ta = lane_base + Cfg::ACOL0 + buf * Cfg::AU_COLS + j * 8 + part * NWA;
+          if constexpr (NWA == 2) tc::tmem_st2(ta, reg);
+          else tc::tmem_st4(ta, reg);
+        }
+        tc::tmem_wait_st();
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&sh.full[g % NSB]);
+
+        if (s == nsub - 1) {
+          // ---------------- epilogue of pass p -----------------------------
+          const bool ok = __all_sync(0xffffffffu, tc::mbar_wait(&sh.acc_full, p & 1));
+          if (!ok) {
+            raise_flag(status, CURVEFP_DEV_TIMEOUT);
+            sh.abort_flag = 1;
+          }
+          tc::fence_after_sync();
+#pragma unroll 1
+          for (int c0 = part * (BN / ATPR); c0 < (part + 1) * (BN / ATPR); c0 += 8) {
+            uint32_t acc[PP][8];
+#pragma unroll
+            for (int q = 0; q < PP; ++q)
+              if (p * PP + q < L) tc::tmem_ld8(lane_base + q * BN + c0, acc[q]);
+            tc::tmem_wait_ld();
+            if (rowok && ok) {
+              float y[8];
+#pragma unroll
+              for (int c = 0; c < 8; ++c) {
+                float t = 0.f;
+#pragma unroll
+                for (int q = 0; q < PP; ++q)
+                  if (p * PP + q < L) t = fmaf(phase_const(L, p * PP + q), __uint_as_float(acc[q][c]), t);
+                y[c] = scalbnf(t, ref + Cfg::PBA + sh.refB[c0 + c] + Cfg::PBB);
+              }
+              float* dst = C + (int64_t)r * N + n0 + c0;
+              const bool full8 = n0 + c0 + 8 <= N && ((reinterpret_cast<uintptr_t>(dst) & 15) == 0);
+              if (full8) {
+                float4* d4 = reinterpret_cast<float4*>(dst);
+                float4 a0 = make_float4(y[0], y[1], y[2], y[3]), a1 = make_float4(y[4], y[5], y[6], y[7]);
+                if (p > 0) {
+                  const float4 b0 = d4[0], b1 = d4[1];
+                  a0.x += b0.x; a0.y += b0.y; a0.z += b0.z; a0.w += b0.w;
+                  a1.x += b1.x; a1.y += b1.y; a1.z += b1.z; a1.w += b1.w;
+                }
+                d4[0] = a0;
+                d4[1] = a1;
+              } else {
+#pragma unroll
+                for (int c = 0; c < 8; ++c)
+                  if (n0 + c0 + c < N) dst[c] = p == 0 ? y[c] : dst[c] + y[c];
+              }
+            }
+          }
+          if (!ok) return false;
+        }
+      } else {
+        const int st = g % NSB;
+        bool fail = false;
+        if (g >= NSB) fail = !__all_sync(0xffffffffu, tc::mbar_wait(&sh.empty[st], ((g / NSB) - 1) & 1));
+        if (fail) {
+          if (lane == 0) raise_flag(status, CURVEFP_DEV_TIMEOUT);
+          sh.abort_flag = 1;
+          return false;
+        }
+        uint32_t v[4], vc[4], mk[4][3];
+        if constexpr (PES)
+          decode_words_pes<FB, 4>(cw, dw, bias, v, vc, mk, true);
+        else
+          decode_words<FB, PT, 4>(cw, off, v, vc, mk, true);
+        uint8_t* stg = bstage + (size_t)st * Cfg::BSTAGE;
+        if (p == 0) write_b_planes<Cfg, PT, 0>(stg, rloc, part, v, vc, mk);
+        if (NP > 1 && p == 1) write_b_planes<Cfg, PT, (NP > 1 ? 1 : 0)>(stg, rloc, part, v, vc, mk);
+        if (NP > 2 && p == 2) write_b_planes<Cfg, PT, (NP > 2 ? 2 : 0)>(stg, rloc, part, v, vc, mk);
+        tc::fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&sh.full[st]);
+      }
+      return true;
+    };
+    // Two register sets of codes, each loaded two steps before it is used and
+    // never copied, so that no register move waits on an in-flight load.
+    uint4 q0, q1, d0, d1;
+    int r0, r1;
+    load(0, q0, r0, d0);
+    load(1, q1, r1, d1);
+    for (int g = 0; g < total; g += 2) {
+      if (!step(g, q0, r0, d0)) break;
+      load(g + 2, q0, r0, d0);
+      if (g + 1 >= total) break;
+      if (!step(g + 1, q1, r1, d1)) break;
+      load(g + 3, q1, r1, d1);
+    }
+  } else {
+    // ------------------------------ MMA issuer -------------------------------
+    // The whole warp runs the loop; the elected lane issues MMAs and commits.
+    const uint32_t leader = tc::elect_one();
+    const uint64_t bdesc0 = tc::smem_desc(tc::smem_u32(bstage), 128, 256);
+    bool ok = true;
+    for (int g = 0; g < total && ok; ++g) {
+      const int p = (NP > 1 && g >= nsub ? 1 : 0) + (NP > 2 && g >= 2 * nsub ? 1 : 0), s = g - p * nsub;
+      const int st = g % NSB;
+      ok = __all_sync(0xffffffffu, tc::mbar_wait(&sh.full[st], (g / NSB) & 1));
+      // a producer that gave up also stops arriving, so the wait above ends
+      // the loop anyway; the flag only shortens that, and is read rarely
+      // because every cycle of this loop delays the next MMA
+      if ((g & 7) == 0) ok = ok && !read_abort(&sh.abort_flag);
+      if (!ok) break;
+      tc::fence_after_sync();
+      issue_step<Cfg, PT>(leader, p, tmem, bdesc0, g & 1, st, s == 0);
+      tc::mma_commit_if(leader, &sh.empty[st]);
+      if (s == nsub - 1) tc::mma_commit_if(leader, &sh.acc_full);
+    }
+    if (!ok && lane == 0) {
+      raise_flag(status, CURVEFP_DEV_TIMEOUT);
+      sh.abort_flag = 1;
+    }
+    // every issued MMA retires before TMEM is released (also on abort)
+    tc::mma_commit_if(leader, &sh.drain);
+    if (!tc::mbar_wait(&sh.drain, 0) && lane == 0) raise_flag(status, CURVEFP_DEV_TIMEOUT);
+    __syncwarp();
+  }
+
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == Cfg::MMA_WARP) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc(tmem, 512);
+  }
+}
+
+template <int FA, int FB, int PT, bool PES>
+static cudaError_t launch_tc_t(int G, const uint8_t* a, const int8_t* sa, const uint8_t* b, const int8_t* sb,
+                               int64_t M, int64_t N, int64_t K, float* c, uint32_t* st, cudaStream_t s,
+                               const PesOperands& pes) {
+  using Cfg = TcCfg<FA, FB, PT>;
+  static_assert(sizeof(TcShared) <= 2048, "shared tail");
+  static_assert(Cfg::SMEM <= 227 * 1024, "shared memory");
+  static_assert(!PES || (PT == PLANE_E5M2 && Cfg::NWA == 4), "per-element scales: E5M2 planes, 16-byte runs");
+  auto kern = gemm_tc_kernel<FA, FB, PT, PES>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg::SMEM);
+  if (e != cudaSuccess) return e;
+  dim3 grid((unsigned)((N + Cfg::BN - 1) / Cfg::BN), (unsigned)((M + Cfg::BM - 1) / Cfg::BM));
+  int gshift = 0;  // scale block of step s is s >> gshift (G / KS is a power of two)
+  while ((Cfg::KS << gshift) < G) ++gshift;
+  kern<<<grid, Cfg::THREADS, Cfg::SMEM, s>>>(a, sa, b, sb, (int)M, (int)N, (int)K, G, gshift, c, st, pes);
+  return cudaGetLastError();
+}
+
+}  // namespace cfp

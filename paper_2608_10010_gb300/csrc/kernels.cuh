@@ -24,6 +24,14 @@ cudaError_t launch_gemm_tensor_sparse(int fa, int fb, int G, const uint8_t* a, c
                                       const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, uint32_t* status,
                                       cudaStream_t st);
 bool gemm_tensor_supported(int fa, int fb);
+cudaError_t launch_gemm_exact_oriented(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, int la,
+                                       const uint8_t* b, const int8_t* sb, int lb, int64_t M, int64_t N, int64_t K,
+                                       float* c, int64_t* phase_sums, int32_t* phase_lsb, uint32_t* status,
+                                       cudaStream_t st);
+size_t gemm_reuse_workspace(int la, int lb, int64_t M, int64_t N, int64_t K);
+cudaError_t launch_gemm_tensor_reuse(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, int la,
+                                     const uint8_t* b, const int8_t* sb, int lb, int64_t M, int64_t N, int64_t K,
+                                     float* c, void* ws, uint32_t* status, cudaStream_t st);
 cudaError_t launch_gemm_q32(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
                             const int8_t* sb, int64_t M, int64_t N, int64_t K, int64_t* out, uint32_t* status,
                             cudaStream_t s);

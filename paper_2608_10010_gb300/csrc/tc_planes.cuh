@@ -171,6 +171,44 @@ __device__ __forceinline__ void decode_words(const uint4& cw, int off, uint32_t 
   }
 }
 
+// E5M2 plane bytes of four codes whose scales differ per element (reused
+// operands).  Byte i of dp holds d_i + 64, d_i = max(a_i - ref, -64) the
+// element's scale relative to the row reference, so the exponent field is
+//   e5_i = e_b + 15 - 2^{E-1} - bias + d_i
+// and the element is kept where e5_i >= 1 and m != 0 (as e5m2_word, which is
+// the case d_i = const).  Per lane u = e5 + 127 = e_b + dp + (78 - 2^{E-1} -
+// bias): every term is non-negative and u <= 2^E - 1 + 64 + 74 < 256, so no
+// lane carries into its neighbour; bit 7 of u is e5 >= 1, and where it is set
+// (u & 0x7F) + 1 = e5 <= 2^{E-1} + 14 - bias <= 30.
+template <int FMT>
+__device__ __forceinline__ uint32_t e5m2_word_pes(uint32_t w, uint32_t dp, uint32_t kc, uint32_t& keep) {
+  using F = Fmt<FMT>;
+  const uint32_t m4 = w & CodeBits<FMT>::MM;
+  const uint32_t eb = (w >> F::C) & (((1u << F::E) - 1u) * 0x01010101u);
+  const uint32_t u = eb + dp + kc;
+  keep = prmt_sign(u & (m4 + 0x7F7F7F7Fu) & 0x80808080u, 0xBA98u);
+  const uint32_t e5 = ((u & 0x7F7F7F7Fu) + 0x01010101u) & keep;
+  return (w & 0x80808080u & keep) | (e5 << 2);
+}
+
+// decode_words for E5M2 planes with per-element scales (dw: the d + 64 bytes
+// of the sixteen codes of cw).
+template <int FMT, int NW>
+__device__ __forceinline__ void decode_words_pes(const uint4& cw, const uint4& dw, int bias, uint32_t (&v)[NW],
+                                                 uint32_t (&vc)[NW], uint32_t (&mk)[NW][3], bool want_carry) {
+  constexpr int KBITS = Fmt<FMT>::C;
+  const uint32_t w[4] = {cw.x, cw.y, cw.z, cw.w};
+  const uint32_t d[4] = {dw.x, dw.y, dw.z, dw.w};
+  const uint32_t kc = (uint32_t)(78 - (1 << (Fmt<FMT>::E - 1)) - bias) * 0x01010101u;
+#pragma unroll
+  for (int i = 0; i < NW; ++i) {
+    uint32_t keep;
+    v[i] = e5m2_word_pes<FMT>(w[i], d[i], kc, keep);
+    vc[i] = want_carry ? v[i] + (keep & 0x04040404u) : 0u;  // exponent + 1
+    k_masks<PLANE_E5M2, KBITS>(w[i], mk[i]);
+  }
+}
+
 __device__ __forceinline__ float phase_const(int L, int h) {
   return __uint_as_float(L == 8 ? CFP_PHASE_F32_L8_DEV[h] : CFP_PHASE_F32_L4_DEV[h]);
 }

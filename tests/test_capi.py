@@ -85,6 +85,42 @@ def test_host_side_validation(lib):
     assert qs(1, 32, 2, 1, None, 0, 0, 64, None, None, None, 0, None, None) == 0
 
 
+def test_oriented_gemm_validation(lib):
+    """Layouts, blocked extents, workspace and algorithm rules of the oriented
+    GEMM, all decided on the host before any launch."""
+    import ctypes as C
+
+    P = C.c_void_p
+    d = P(4096)
+    INVALID, UNSUPPORTED = 1, 2
+    lib.curvefp_gemm_oriented_workspace_bytes.restype = C.c_size_t
+    lib.curvefp_gemm_oriented_workspace_bytes.argtypes = [C.c_int, C.c_int, C.c_int, C.c_int64, C.c_int64, C.c_int64]
+    wsb = lib.curvefp_gemm_oriented_workspace_bytes
+    al = lambda v: (v + 255) // 256 * 256  # noqa: E731
+    assert wsb(1, 0, 0, 256, 96, 64) == 0 and wsb(0, 1, 1, 256, 96, 64) == 0
+    assert wsb(1, 0, 1, 256, 96, 64) == al(256 * 64) + al(4 * 256) + 2 * al(96 * 64) + al(4 * 96)
+    assert wsb(1, 1, 1, 256, 96, 64) == 2 * al(256 * 64) + al(4 * 256) + 2 * al(96 * 64) + al(4 * 96)
+    go = lib.curvefp_gemm_oriented
+    go.argtypes = [C.c_int] * 4 + [P, P, C.c_int, P, P, C.c_int, C.c_int64, C.c_int64, C.c_int64, P, P, P, P,
+                                   C.c_size_t, P, P]
+
+    def call(algo=1, la=0, lb=1, M=64, N=64, K=64, c=d, ps=None, pl=None, ws=None, wsn=0, block=32):
+        return go(algo, 1, 1, block, d, d, la, d, d, lb, M, N, K, c, ps, pl, ws, wsn, None, None)
+
+    assert call(la=2) == INVALID                       # unknown layout
+    assert call(la=1, M=48) == INVALID                 # COLS rows not a multiple of the block
+    assert call(lb=0, K=48) == INVALID                 # ROWS K not a multiple of the block
+    assert call(lb=1, N=80) == INVALID
+    assert call() == INVALID                           # TENSOR with a COLS operand needs workspace
+    assert call(ws=P(4096 + 16), wsn=1 << 30) == INVALID  # workspace not 256-byte aligned
+    assert call(ws=d, wsn=16) == INVALID               # workspace too small
+    assert call(ps=d, pl=d, ws=d, wsn=1 << 30) == INVALID  # phase sums only from EXACT
+    assert call(algo=2, ws=d, wsn=1 << 30) == UNSUPPORTED  # sparse: ROWS x ROWS only
+    assert call(la=1, lb=1, K=48, ws=d, wsn=1 << 30) == INVALID  # tensor steps need K % 32
+    assert call(algo=0, c=None) == INVALID             # exact: nothing to write
+    assert call(algo=0, ps=d, pl=None) == INVALID      # exact: both phase arrays or neither
+
+
 def test_product_path_does_not_touch_the_oracle():
     """The CUDA library and its binding neither import nor link the oracle."""
     pkg = os.path.join(ROOT, "paper_2608_10010_gb300")
