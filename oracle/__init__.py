@@ -29,7 +29,8 @@ _LIB = os.path.join(_HERE, "liboracle.so")
 _lock = threading.Lock()
 _lib = None
 
-FORMATS = {"E3C3": 0, "E4C3": 1, "E5C2": 2}
+# 3, 4: E4C3 with the rational radices r = 2^{8/9} and r = 2^{3/4} (R14)
+FORMATS = {"E3C3": 0, "E4C3": 1, "E5C2": 2, "E4C3_R8_9": 3, "E4C3_R3_4": 4}
 
 
 def build(force: bool = False) -> str:
@@ -97,7 +98,7 @@ def format_params(fmt) -> dict:
 
 
 def levels(fmt) -> np.ndarray:
-    """All positive levels 2^{n/K}, n = -nmax..nmax (Eq. 1, binary radix)."""
+    """All positive levels r^{n/K} = 2^{p n/(qK)}, n = -nmax..nmax (Eq. 1)."""
     p = format_params(fmt)
     out = np.empty(2 * p["nmax"] + 1, np.float64)
     _load().oracle_levels(_fid(fmt), _ptr(out))
@@ -202,7 +203,8 @@ def closed_product(fmt_a, fmt_b, ca: int, cb: int):
 def pair_info(fmt_a, fmt_b):
     """(L, t_min, t_max): shared lattice size (= phase count H) and bin range."""
     L, lo, hi = ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
-    _load().oracle_pair_info(_fid(fmt_a), _fid(fmt_b), ctypes.byref(L), ctypes.byref(lo), ctypes.byref(hi))
+    if _load().oracle_pair_info(_fid(fmt_a), _fid(fmt_b), ctypes.byref(L), ctypes.byref(lo), ctypes.byref(hi)):
+        raise ValueError("format pair not supported (rational radices pair only with themselves)")
     return L.value, lo.value, hi.value
 
 

@@ -36,6 +36,16 @@
  *   R6 exported per-phase sums are integers S_h at the per-output LSB
  *      lambda = min_b(sa_b + sb_b) + t_min.
  *   R11, R12 static-operand scale groups and MSE-search scales (below).
+ *   R14 rational radix r = 2^{p/q} (Sec. 3.1, Eq. 4, Table 7's E4C3 points
+ *      r = 2^{8/9} and r = 2^{3/4}): the level of index n is 2^{p n/(qK)};
+ *      the closed product of two codes of the same format has
+ *      u = p (n_a + n_b), phase h = (u mod qK)/g and bin t = floor(u/qK)
+ *      (App. A.1), H = qK/g phases weighted 2^{h/H}; FP32 dequantization is
+ *      RN32(2^{j/(qK)}) 2^{a + floor(p n/(qK))}, j = p n mod qK (R4 with the
+ *      fractional exponent in place of k/K).  Only same-format pairs.  An
+ *      exact tie in the nearest-level search (possible only between zero and
+ *      L_nmin when L_nmin is a power of two, as for r = 2^{8/9}) goes to the
+ *      smaller magnitude.
  *   R13 reused operands (Sec. 4, training GEMMs: the backward GEMMs take the
  *      forward pass's quantized operands, one of them transposed) keep each
  *      element's own code and block scale, so a GEMM operand may carry a
@@ -59,6 +69,7 @@ typedef struct {
   int K;    /* curves per exponent, K = 2^C           */
   int B;    /* rank bias 2^{E+C-1}                    */
   int nmax; /* largest lattice index, nmin = -nmax    */
+  int p, q; /* radix r = 2^{p/q} (R14); 1, 1 = binary  */
 } ofmt;
 
 static int ofmt_get(int id, ofmt* f) {
@@ -66,8 +77,12 @@ static int ofmt_get(int id, ofmt* f) {
     case 0: f->E = 3; f->C = 3; break; /* E3C3 */
     case 1: f->E = 4; f->C = 3; break; /* E4C3 */
     case 2: f->E = 5; f->C = 2; break; /* E5C2 */
+    case 3: f->E = 4; f->C = 3; break; /* E4C3, r = 2^{8/9} (R14) */
+    case 4: f->E = 4; f->C = 3; break; /* E4C3, r = 2^{3/4} (R14) */
     default: return -1;
   }
+  f->p = id == 3 ? 8 : (id == 4 ? 3 : 1);
+  f->q = id == 3 ? 9 : (id == 4 ? 4 : 1);
   f->K = 1 << f->C;
   f->B = 1 << (f->E + f->C - 1);
   /* Sec. 3.1: exponents e in [-2^{E-1}, 2^{E-1}-1], k in [0, K-1]; the
@@ -80,10 +95,23 @@ static int ofmt_get(int id, ofmt* f) {
 static int floordiv(int a, int b) { int q = a / b; if ((a % b) && ((a < 0) != (b < 0))) q--; return q; }
 static int floormod(int a, int b) { int r = a % b; if (r && ((r < 0) != (b < 0))) r += b; return r; }
 
-/* ---- Element value, Eq. 1 (binary radix r = 2) ----------------------- */
+/* ---- Element value, Eq. 1 ------------------------------------------- */
 
-/* Unscaled level for lattice index n: 2^{n/K}. */
-static double olevel(const ofmt* f, int n) { return exp2((double)n / (double)f->K); }
+/* Unscaled level for lattice index n: r^{n/K} = 2^{p n/(q K)}, evaluated as
+ * 2^{j/(qK)} 2^e with e = floor(p n/(qK)), j = p n mod qK (the exponent's
+ * fractional part is then the only rounded input of exp2). */
+static double olevel(const ofmt* f, int n) {
+  int den = f->q * f->K;
+  return ldexp(exp2((double)floormod(f->p * n, den) / den), floordiv(f->p * n, den));
+}
+
+/* R4 (R14): RN32 of the fractional power times the integer power. */
+static double odequant_exact(const ofmt* f, int n, int a) {
+  int den = f->q * f->K;
+  int e = floordiv(f->p * n, den), j = floormod(f->p * n, den);
+  float cj = (float)exp2((double)j / den); /* RN32(2^{j/(qK)}) */
+  return ldexp((double)cj, a + e);        /* exact in fp64     */
+}
 
 int oracle_format(int id, int* E, int* C, int* K, int* B, int* nmax) {
   ofmt f;
@@ -240,9 +268,7 @@ int oracle_encode(int id, int G, const float* x, int64_t R, int64_t Cc, const in
 static float odequant_one(const ofmt* f, uint8_t code, int a) {
   int s, n;
   if (!odecode(f, code, &s, &n)) return 0.0f;
-  int e = floordiv(n, f->K), k = floormod(n, f->K);
-  float ck = (float)exp2((double)k / f->K);
-  double exact = ldexp((double)ck, a + e);
+  double exact = odequant_exact(f, n, a);
   return (float)(s ? -exact : exact);
 }
 
@@ -345,26 +371,46 @@ int oracle_dequantize(int id, int G, const uint8_t* codes, const int8_t* scales,
       int s, n;
       float v = 0.0f;
       if (odecode(&f, codes[r * Cc + c], &s, &n)) {
-        int e = floordiv(n, f.K), k = floormod(n, f.K);
-        float ck = (float)exp2((double)k / f.K);               /* RN32(2^{k/K})      */
-        double exact = ldexp((double)ck, scales[r * nb + c / G] + e); /* exact in fp64 */
-        v = (float)(s ? -exact : exact);                         /* one RN32 rounding  */
+        double exact = odequant_exact(&f, n, scales[r * nb + c / G]); /* exact in fp64 */
+        v = (float)(s ? -exact : exact);                               /* one RN32 rounding */
       }
       out[r * Cc + c] = v;
     }
   return 0;
 }
 
-/* ---- Closed product, Eq. 2 and App. A.1 (binary radix), reading R5 ---- */
-typedef struct { int La, wa, wb, L; } olattice;
+/* ---- Closed product, Eq. 2 and App. A.1, readings R5 and R14 ---------
+ * A product of lattice indices n_a, n_b sits at u = P (n_a wa + n_b wb) on a
+ * lattice of N steps per binade: phase h = (u mod N)/g, bin t = floor(u/N),
+ * L = N/g phases.  Binary radix (R5): N = max(K_a, K_b) (the lcm of two
+ * powers of two), wa = N/K_a, wb = N/K_b, P = g = 1.  Rational radix, same
+ * format on both sides (R14): N = qK, wa = wb = 1, P = p, g = gcd(p, qK). */
+typedef struct { int wa, wb, P, N, g, L, ok; } olattice;
 
 static olattice olattice_of(const ofmt* fa, const ofmt* fb) {
   olattice l;
-  l.L = fa->K > fb->K ? fa->K : fb->K; /* lcm of two powers of two */
-  l.wa = l.L / fa->K;
-  l.wb = l.L / fb->K;
-  l.La = 0;
+  if (fa->p == 1 && fa->q == 1 && fb->p == 1 && fb->q == 1) {
+    l.N = fa->K > fb->K ? fa->K : fb->K;
+    l.wa = l.N / fa->K;
+    l.wb = l.N / fb->K;
+    l.P = 1;
+    l.g = 1;
+    l.ok = 1;
+  } else {
+    l.ok = fa->p == fb->p && fa->q == fb->q && fa->K == fb->K;
+    l.N = fa->q * fa->K;
+    l.wa = l.wb = 1;
+    l.P = fa->p;
+    l.g = (int)gcdl(fa->p, l.N);
+  }
+  l.L = l.N / l.g;
   return l;
+}
+
+static void oaddr(const olattice* l, int na, int nb, int* h, int* t) {
+  int u = l->P * (na * l->wa + nb * l->wb);
+  *h = floormod(u, l->N) / l->g;
+  *t = floordiv(u, l->N);
 }
 
 /* Product of two codes: returns 0 if either is zero (no update), else sets
@@ -375,25 +421,33 @@ int oracle_closed_product(int ida, int idb, uint8_t ca, uint8_t cb, int* delta, 
   int sa, na, sb, nb;
   if (!odecode(&fa, ca, &sa, &na) || !odecode(&fb, cb, &sb, &nb)) return 0;
   olattice l = olattice_of(&fa, &fb);
-  int u = na * l.wa + nb * l.wb;
+  if (!l.ok) return -1;
   *delta = (sa ^ sb) ? -1 : 1;
-  *h = floormod(u, l.L);
-  *t = floordiv(u, l.L);
+  oaddr(&l, na, nb, h, t);
   return 1;
 }
 
-/* Smallest and largest bin offset t over nonzero products of a pair. */
+/* Smallest and largest bin offset t over nonzero products of a pair (every
+ * pair of lattice indices tried). */
 static void otrange(const ofmt* fa, const ofmt* fb, int* tmin, int* tmax) {
   olattice l = olattice_of(fa, fb);
-  int umax = fa->nmax * l.wa + fb->nmax * l.wb;
-  *tmin = floordiv(-umax, l.L);
-  *tmax = floordiv(umax, l.L);
+  *tmin = 1 << 20;
+  *tmax = -(1 << 20);
+  for (int na = -fa->nmax; na <= fa->nmax; ++na)
+    for (int nb = -fb->nmax; nb <= fb->nmax; ++nb) {
+      int h, t;
+      oaddr(&l, na, nb, &h, &t);
+      if (t < *tmin) *tmin = t;
+      if (t > *tmax) *tmax = t;
+    }
 }
 
 int oracle_pair_info(int ida, int idb, int* L, int* tmin, int* tmax) {
   ofmt fa, fb;
   if (ofmt_get(ida, &fa) || ofmt_get(idb, &fb)) return -1;
-  *L = olattice_of(&fa, &fb).L;
+  olattice l = olattice_of(&fa, &fb);
+  if (!l.ok) return -1;
+  *L = l.L;
   otrange(&fa, &fb, tmin, tmax);
   return 0;
 }
@@ -420,13 +474,14 @@ int64_t oracle_gemm(int ida, int idb, int G, const uint8_t* A, const int8_t* sA,
   ofmt fa, fb;
   if (ofmt_get(ida, &fa) || ofmt_get(idb, &fb)) return -1;
   olattice l = olattice_of(&fa, &fb);
+  if (!l.ok) return -1;
   int tmin, tmax;
   otrange(&fa, &fb, &tmin, &tmax);
   int64_t nb = K / G;
   int64_t bad = 0;
 #pragma omp parallel for schedule(dynamic, 1) reduction(+ : bad)
   for (int64_t i = 0; i < M; ++i) {
-    i128 acc[8];
+    i128 acc[32];
     for (int64_t j = 0; j < N; ++j) {
       int smin = 1 << 20, smax = -(1 << 20);
       for (int64_t b = 0; b < nb; ++b) {
@@ -442,9 +497,9 @@ int64_t oracle_gemm(int ida, int idb, int G, const uint8_t* A, const int8_t* sA,
           int s1, n1, s2, n2;
           if (!odecode(&fa, A[i * K + d], &s1, &n1)) continue;
           if (!odecode(&fb, B[j * K + d], &s2, &n2)) continue;
-          int u = n1 * l.wa + n2 * l.wb;
-          int h = floormod(u, l.L);
-          int t = floordiv(u, l.L) + sA[i * nb + d / G] + sB[j * nb + d / G];
+          int h, t;
+          oaddr(&l, n1, n2, &h, &t);
+          t += sA[i * nb + d / G] + sB[j * nb + d / G];
           i128 term = (i128)1 << (t - lambda);
           acc[h] += (s1 ^ s2) ? -term : term;
         }
@@ -481,12 +536,13 @@ int64_t oracle_gemm_elem(int ida, int idb, const uint8_t* A, const int8_t* eA, c
   ofmt fa, fb;
   if (ofmt_get(ida, &fa) || ofmt_get(idb, &fb)) return -1;
   olattice l = olattice_of(&fa, &fb);
+  if (!l.ok) return -1;
   int tmin, tmax;
   otrange(&fa, &fb, &tmin, &tmax);
   int64_t bad = 0;
 #pragma omp parallel for schedule(dynamic, 1) reduction(+ : bad)
   for (int64_t i = 0; i < M; ++i) {
-    i128 acc[8];
+    i128 acc[32];
     for (int64_t j = 0; j < N; ++j) {
       int smin = 1 << 20, smax = -(1 << 20);
       for (int64_t d = 0; d < K; ++d) {
@@ -502,9 +558,9 @@ int64_t oracle_gemm_elem(int ida, int idb, const uint8_t* A, const int8_t* eA, c
           int s1, n1, s2, n2;
           if (!odecode(&fa, A[i * K + d], &s1, &n1)) continue;
           if (!odecode(&fb, B[j * K + d], &s2, &n2)) continue;
-          int u = n1 * l.wa + n2 * l.wb;
-          int h = floormod(u, l.L);
-          int t = floordiv(u, l.L) + eA[i * K + d] + eB[j * K + d];
+          int h, t;
+          oaddr(&l, n1, n2, &h, &t);
+          t += eA[i * K + d] + eB[j * K + d];
           i128 term = (i128)1 << (t - lambda);
           acc[h] += (s1 ^ s2) ? -term : term;
         }
@@ -535,6 +591,7 @@ int oracle_histogram(int ida, int idb, int G, const uint8_t* a, const int8_t* sa
   ofmt fa, fb;
   if (ofmt_get(ida, &fa) || ofmt_get(idb, &fb)) return -1;
   olattice l = olattice_of(&fa, &fb);
+  if (!l.ok) return -1;
   memset(counts, 0, sizeof(int64_t) * (size_t)l.L * (size_t)nt);
   for (int64_t d = 0; d < K; ++d) {
     int delta, h, t;
