@@ -206,6 +206,27 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
     res["gemm_q32"] = {"workload": "E4C3 1024x1024x4096", "ms": round(ms, 4),
                        "gmac_per_s": round(1024 * 1024 * 4096 / (ms / 1e3) / 1e9, 1)}
     del Xq, Wq, aq, saq, bq, sbq, outq
+    # rational radix (E4C3 with r = 2^{8/9}, 2^{3/4}; the radix-frontier
+    # setting G512): quantizer bandwidth and the exact 9- / 32-phase GEMM
+    res["radix"] = []
+    Xr = torch.randn((8192, 8192), device="cuda", generator=torch.Generator(device="cuda").manual_seed(3))
+    Ar = torch.randn((1024, 4096), device="cuda", generator=torch.Generator(device="cuda").manual_seed(5))
+    Br = torch.randn((1024, 4096), device="cuda", generator=torch.Generator(device="cuda").manual_seed(6)) * 0.02
+    for fmt in ("E4C3", "E4C3_R8_9", "E4C3_R3_4"):
+        cr = torch.empty(Xr.shape, dtype=torch.uint8, device="cuda")
+        sr = torch.empty((8192, 8192 // 512), dtype=torch.int8, device="cuda")
+        ms_q = _time_ms(torch, stream, lambda: cfp.quantize(Xr, fmt, 512, 0, codes=cr, scales=sr, stream=stream),
+                        flush_l2)
+        (ar, sar), (br, sbr) = cfp.quantize(Ar, fmt, 512, 0, stream=stream), cfp.quantize(Br, fmt, 512, 0, stream=stream)
+        ms_g = _time_ms(torch, stream, lambda: cfp.gemm(ar, sar, br, sbr, fmt, fmt, 512, "exact", stream=stream),
+                        flush_l2, reps=3, warm=1)
+        res["radix"].append({"format": fmt, "phases": cfp.phase_count(fmt, fmt),
+                             "quantize_fp32_8192x8192_G512_ms": round(ms_q, 4),
+                             "quantize_gbs": round(Xr.numel() * (4 + 1 + 1 / 512) / (ms_q / 1e3) / 1e9, 1),
+                             "exact_gemm_1024x1024x4096_ms": round(ms_g, 4),
+                             "exact_gemm_gmac_per_s": round(1024 * 1024 * 4096 / (ms_g / 1e3) / 1e9, 1)})
+        del cr, sr, ar, sar, br, sbr
+    del Xr, Ar, Br
     # training triplet, E4C3 weights/activations, E5C2 gradients
     X, Wt, dY = inputs.training_triplet_cuda()
     gemm_case("fwd X.W", q(X, "E4C3", 0), "E4C3", q(Wt, "E4C3", 1), "E4C3", 64)

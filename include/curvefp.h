@@ -7,7 +7,9 @@
  * (Sec. 3.1, Eq. 1), multiplies codes exactly by adding curve indices with a
  * carry into the exponent (Sec. 3.2, Eq. 2), accumulates products per phase
  * of the radix's phase schedule (Eq. 4, Eq. 5, App. A.1) and combines the
- * phases with fixed constants 2^{h/H}.  Binary radix (r = 2) only.
+ * phases with fixed constants 2^{h/H}.  Binary radix (r = 2) throughout, and
+ * the two rational-radix E4C3 variants of the radix frontier (see
+ * curvefp_format_t).
  *
  * Conventions for every entry point
  *   - All tensor pointers are DEVICE pointers to caller-owned memory.  The
@@ -45,7 +47,24 @@ extern "C" {
 
 /* Table 1: E3C3 (CurveFP7, 7 bits, 63 positive levels, H = 8), E4C3 and E5C2
  * (CurveFP8, 8 bits, 127 positive levels, H = 8 and 4). */
-typedef enum { CURVEFP_E3C3 = 0, CURVEFP_E4C3 = 1, CURVEFP_E5C2 = 2 } curvefp_format_t;
+/* E3C3 (CurveFP7), E4C3 and E5C2 (CurveFP8): Table 1, binary radix.
+ * E4C3_R8_9, E4C3_R3_4: E4C3 codes with the rational radices r = 2^{8/9}
+ * (9 phases) and r = 2^{3/4} (32 phases) of the radix frontier (Sec. 3.1
+ * Eq. 1 with r = 2^{p/q}, Eq. 4, Table 7): level x = (-1)^s 2^{a_b}
+ * 2^{p n/(8q)}; block scale = the smallest a_b with max|x| <= 2^{a_b}
+ * 2^{63 p/(8q)}; an exact tie in the nearest-level search (only between zero
+ * and L_nmin = 2^{-7} for r = 2^{8/9}) goes to zero; dequantization is
+ * RN32(RN32(2^{j/(8q)}) 2^{a_b + floor(p n/(8q))}), j = p n mod 8q.  They are
+ * accepted by curvefp_quantize (block_axis 0), curvefp_dequantize and the
+ * EXACT GEMMs (both operands of the same format); every other entry point
+ * returns CURVEFP_ERR_UNSUPPORTED for them. */
+typedef enum {
+  CURVEFP_E3C3 = 0,
+  CURVEFP_E4C3 = 1,
+  CURVEFP_E5C2 = 2,
+  CURVEFP_E4C3_R8_9 = 3,
+  CURVEFP_E4C3_R3_4 = 4
+} curvefp_format_t;
 
 typedef enum { CURVEFP_F32 = 0, CURVEFP_BF16 = 1 } curvefp_dtype_t;
 

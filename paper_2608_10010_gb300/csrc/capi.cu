@@ -10,7 +10,9 @@
 
 namespace {
 
-bool fmt_ok(int f) { return f == CURVEFP_E3C3 || f == CURVEFP_E4C3 || f == CURVEFP_E5C2; }
+bool fmt_ok(int f) { return f == CURVEFP_E3C3 || f == CURVEFP_E4C3 || f == CURVEFP_E5C2; }  // binary radix
+bool fmt_radix(int f) { return f == CURVEFP_E4C3_R8_9 || f == CURVEFP_E4C3_R3_4; }      // rational radix
+bool fmt_any(int f) { return fmt_ok(f) || fmt_radix(f); }
 bool block_ok(int g) { return g == 32 || g == 64 || g == 128 || g == 256 || g == 512; }
 bool al16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 int fmt_k(int f) { return f == CURVEFP_E5C2 ? 4 : 8; }
@@ -31,9 +33,10 @@ extern "C" {
 curvefp_status_t curvefp_quantize(curvefp_format_t fmt, int block, const void* x, curvefp_dtype_t dtype,
                                   int64_t rows, int64_t cols, int64_t ld, int block_axis, uint8_t* codes,
                                   int8_t* scales, uint32_t* device_status, void* stream) {
-  if (!fmt_ok(fmt) || !block_ok(block) || (dtype != CURVEFP_F32 && dtype != CURVEFP_BF16)) return CURVEFP_ERR_INVALID_ARG;
+  if (!fmt_any(fmt) || !block_ok(block) || (dtype != CURVEFP_F32 && dtype != CURVEFP_BF16)) return CURVEFP_ERR_INVALID_ARG;
   if (block_axis != 0 && block_axis != 1) return CURVEFP_ERR_INVALID_ARG;
   if (rows < 0 || cols < 0 || ld < cols) return CURVEFP_ERR_INVALID_ARG;
+  if (fmt_radix(fmt) && block_axis != 0) return CURVEFP_ERR_UNSUPPORTED;
   if (rows == 0 || cols == 0) return CURVEFP_OK;
   if (!x || !codes || !scales) return CURVEFP_ERR_INVALID_ARG;
   const int64_t esz = dtype == CURVEFP_F32 ? 4 : 2;
@@ -44,6 +47,9 @@ curvefp_status_t curvefp_quantize(curvefp_format_t fmt, int block, const void* x
   if (block_axis == 1 && rows % block != 0) return CURVEFP_ERR_INVALID_ARG;
   if (block_axis == 1 && rows / block > 65535) return CURVEFP_ERR_UNSUPPORTED;
   if (rows * cols / block > (int64_t)1 << 40) return CURVEFP_ERR_UNSUPPORTED;
+  if (fmt_radix(fmt))
+    return from_cuda(cfp::launch_quantize_radix(fmt, block, x, dtype, rows, cols, ld, codes, scales, device_status,
+                                                static_cast<cudaStream_t>(stream), sm_count()));
   return from_cuda(cfp::launch_quantize(fmt, block, x, dtype, rows, cols, ld, block_axis, codes, scales,
                                         device_status, static_cast<cudaStream_t>(stream), sm_count()));
 }
@@ -57,6 +63,7 @@ curvefp_status_t curvefp_quantize_static(curvefp_format_t fmt, int block, curvef
                                          curvefp_scale_rule_t rule, const void* x, curvefp_dtype_t dtype, int64_t rows,
                                          int64_t cols, uint8_t* codes, int8_t* scales, void* workspace,
                                          size_t workspace_bytes, uint32_t* device_status, void* stream) {
+  if (fmt_radix(fmt)) return CURVEFP_ERR_UNSUPPORTED;
   if (!fmt_ok(fmt) || !block_ok(block) || (dtype != CURVEFP_F32 && dtype != CURVEFP_BF16)) return CURVEFP_ERR_INVALID_ARG;
   if (group < CURVEFP_SCALE_BLOCK || group > CURVEFP_SCALE_TENSOR) return CURVEFP_ERR_INVALID_ARG;
   if (rule != CURVEFP_SCALE_CEIL_ABSMAX && rule != CURVEFP_SCALE_MSE) return CURVEFP_ERR_INVALID_ARG;
@@ -101,17 +108,22 @@ curvefp_status_t curvefp_quantize_static_noalloc(curvefp_format_t fmt, int block
 
 curvefp_status_t curvefp_dequantize(curvefp_format_t fmt, int block, const uint8_t* codes, const int8_t* scales,
                                     int64_t rows, int64_t cols, float* out, void* stream) {
-  if (!fmt_ok(fmt) || !block_ok(block) || rows < 0 || cols < 0) return CURVEFP_ERR_INVALID_ARG;
+  if (!fmt_any(fmt) || !block_ok(block) || rows < 0 || cols < 0) return CURVEFP_ERR_INVALID_ARG;
   if (rows == 0 || cols == 0) return CURVEFP_OK;
   if (!codes || !scales || !out || cols % block != 0 || !al16(codes) || !al16(out)) return CURVEFP_ERR_INVALID_ARG;
+  if (fmt_radix(fmt))
+    return from_cuda(cfp::launch_dequantize_radix(fmt, block, codes, scales, rows * cols, out,
+                                                  static_cast<cudaStream_t>(stream), sm_count()));
   return from_cuda(cfp::launch_dequantize(fmt, block, codes, scales, rows * cols, out,
                                           static_cast<cudaStream_t>(stream), sm_count()));
 }
 
 static curvefp_status_t gemm_args(int fa, int fb, int block, const uint8_t* a, const int8_t* sa, const uint8_t* b,
                                   const int8_t* sb, int64_t M, int64_t N, int64_t K) {
-  if (!fmt_ok(fa) || !fmt_ok(fb) || !block_ok(block)) return CURVEFP_ERR_INVALID_ARG;
+  if (!fmt_any(fa) || !fmt_any(fb) || !block_ok(block)) return CURVEFP_ERR_INVALID_ARG;
   if (M <= 0 || N <= 0 || K <= 0 || K % block != 0) return CURVEFP_ERR_INVALID_ARG;
+  // a rational radix pairs only with itself (one lattice, App. A.1)
+  if ((fmt_radix(fa) || fmt_radix(fb)) && fa != fb) return CURVEFP_ERR_UNSUPPORTED;
   if (!a || !sa || !b || !sb || !al16(a) || !al16(b)) return CURVEFP_ERR_INVALID_ARG;
   if (M > INT32_MAX || N > INT32_MAX || K > INT32_MAX) return CURVEFP_ERR_UNSUPPORTED;
   return CURVEFP_OK;
@@ -127,6 +139,8 @@ curvefp_status_t curvefp_gemm(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, 
   if (algo == CURVEFP_GEMM_EXACT)
     return from_cuda(cfp::launch_gemm_exact(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, nullptr, nullptr,
                                             device_status, st));
+  if ((algo == CURVEFP_GEMM_TENSOR || algo == CURVEFP_GEMM_TENSOR_SPARSE) && fmt_radix(fmt_a))
+    return CURVEFP_ERR_UNSUPPORTED;
   if (algo == CURVEFP_GEMM_TENSOR || algo == CURVEFP_GEMM_TENSOR_SPARSE) {
     if (!cfp::gemm_tensor_supported(fmt_a, fmt_b)) return CURVEFP_ERR_UNSUPPORTED;
     if (algo == CURVEFP_GEMM_TENSOR_SPARSE)
@@ -152,6 +166,7 @@ static bool layout_ok(int l) { return l == CURVEFP_LAYOUT_ROWS || l == CURVEFP_L
 
 static curvefp_status_t oriented_args(int fa, int fb, int block, const uint8_t* a, const int8_t* sa, int la,
                                       const uint8_t* b, const int8_t* sb, int lb, int64_t M, int64_t N, int64_t K) {
+  if (fmt_radix(fa) || fmt_radix(fb)) return CURVEFP_ERR_UNSUPPORTED;
   if (!fmt_ok(fa) || !fmt_ok(fb) || !block_ok(block) || !layout_ok(la) || !layout_ok(lb))
     return CURVEFP_ERR_INVALID_ARG;
   if (M <= 0 || N <= 0 || K <= 0) return CURVEFP_ERR_INVALID_ARG;
@@ -204,7 +219,7 @@ curvefp_status_t curvefp_gemm_requant(curvefp_gemm_algo_t algo, curvefp_format_t
                                       const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c,
                                       curvefp_format_t fmt_c, int block_c, uint8_t* codes_c, int8_t* scales_c,
                                       uint32_t* device_status, void* stream) {
-  if (!fmt_ok(fmt_c) || !block_ok(block_c) || N % block_c != 0 || !c || !codes_c || !scales_c || !al16(c))
+  if (!fmt_any(fmt_c) || !block_ok(block_c) || N % block_c != 0 || !c || !codes_c || !scales_c || !al16(c))
     return CURVEFP_ERR_INVALID_ARG;
   curvefp_status_t r = curvefp_gemm(algo, fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, device_status, stream);
   if (r != CURVEFP_OK) return r;
@@ -224,6 +239,10 @@ curvefp_status_t curvefp_gemm_q32(curvefp_format_t fmt_a, curvefp_format_t fmt_b
 }
 
 int curvefp_phase_count(curvefp_format_t fmt_a, curvefp_format_t fmt_b) {
+  if (fmt_radix(fmt_a) || fmt_radix(fmt_b)) {
+    if (fmt_a != fmt_b) return -1;
+    return fmt_a == CURVEFP_E4C3_R8_9 ? 9 : 32;  // Eq. 4: H = 8q / gcd(p, 8q)
+  }
   if (!fmt_ok(fmt_a) || !fmt_ok(fmt_b)) return -1;
   const int ka = fmt_k(fmt_a), kb = fmt_k(fmt_b);
   return ka > kb ? ka : kb;

@@ -38,21 +38,36 @@ __device__ __forceinline__ double i128_to_double(__int128 v) {
 }
 }  // namespace
 
-template <int FA, int FB>
+// Lat: the phase-address policy (BinLat for binary radix, RadLat for a
+// rational radix).  The 16-bit-part counters (L PARTS x NT int32) and, for
+// more than 8 phases, the int128 phase sums (L x NT) live in dynamic shared
+// memory (exact_smem bytes).
+template <class Lat>
+__host__ __device__ constexpr int exact_parts() {
+  return (Lat::TMAX - Lat::TMIN) / 16 + 1;
+}
+template <class Lat>
+__host__ __device__ constexpr size_t exact_smem() {
+  return (size_t)Lat::L * exact_parts<Lat>() * NT * 4 + (Lat::L > 8 ? (size_t)Lat::L * NT * 16 : 0);
+}
+
+template <class Lat>
 __global__ void __launch_bounds__(NT) gemm_exact_kernel(const uint8_t* __restrict__ A, const int8_t* __restrict__ sA,
                                                         const uint8_t* __restrict__ B, const int8_t* __restrict__ sB,
                                                         int M, int N, int K, int G, float* __restrict__ C,
                                                         int64_t* __restrict__ phase_sums,
                                                         int32_t* __restrict__ phase_lsb, uint32_t* status) {
-  using P = Pair<FA, FB>;
-  constexpr int L = P::L;
-  constexpr int DT = P::TMAX - P::TMIN;   // largest bin offset sh
-  constexpr int PARTS = DT / 16 + 1;      // 16-bit parts of a bin offset
-  constexpr uint32_t MA = Fmt<FA>::MMASK, MB = Fmt<FB>::MMASK;
+  constexpr int L = Lat::L;
+  constexpr int DT = Lat::TMAX - Lat::TMIN;  // largest bin offset sh
+  constexpr int PARTS = exact_parts<Lat>();   // 16-bit parts of a bin offset
+  constexpr uint32_t MA = Lat::MA, MB = Lat::MB;
+  constexpr bool SREG = L <= 8;               // int128 sums in registers
 
   __shared__ uint32_t As[TM][KC / 4];
   __shared__ uint32_t Bs[TN][KC / 4];
-  __shared__ int32_t acc[L * PARTS][NT];
+  extern __shared__ __align__(16) uint8_t exact_dyn[];
+  int32_t(*acc)[NT] = reinterpret_cast<int32_t(*)[NT]>(exact_dyn);
+  __int128(*Ssm)[NT] = reinterpret_cast<__int128(*)[NT]>(exact_dyn + (size_t)L * PARTS * NT * 4);
 
   const int tid = threadIdx.x;
   const int ty = tid / TN, tx = tid % TN;
@@ -71,9 +86,14 @@ __global__ void __launch_bounds__(NT) gemm_exact_kernel(const uint8_t* __restric
   const bool in_range = live && i128_bitlen_ok(smax - smin, DT, K);
   if (live && !in_range && status) atomicOr(status, CURVEFP_DEV_RANGE);
 
-  __int128 S[L];
+  __int128 S[SREG ? L : 1];
 #pragma unroll
-  for (int h = 0; h < L; ++h) S[h] = 0;
+  for (int h = 0; h < L; ++h) {
+    if constexpr (SREG)
+      S[h] = 0;
+    else
+      Ssm[h][tid] = 0;
+  }
 #pragma unroll
   for (int q = 0; q < L * PARTS; ++q) acc[q][tid] = 0;
 
@@ -99,10 +119,10 @@ __global__ void __launch_bounds__(NT) gemm_exact_kernel(const uint8_t* __restric
           const uint32_t ca = (aw >> (8 * q)) & 0xFFu, cb = (bw >> (8 * q)) & 0xFFu;
           const uint32_t ma = ca & MA, mb = cb & MB;
           if (ma != 0u && mb != 0u) {
-            const uint32_t u = ma * P::WA + mb * P::WB;
-            const uint32_t sh = u >> P::LOG2L;
-            const int idx = (int)(u & (L - 1)) * PARTS + (int)(sh >> 4);
-            const int32_t v = (int32_t)(1u << (sh & 15u));
+            int h, sh;
+            Lat::addr(ma, mb, h, sh);
+            const int idx = h * PARTS + (sh >> 4);
+            const int32_t v = (int32_t)(1u << (sh & 15));
             acc[idx][tid] += ((ca ^ cb) & 0x80u) ? -v : v;
           }
         }
@@ -119,7 +139,13 @@ __global__ void __launch_bounds__(NT) gemm_exact_kernel(const uint8_t* __restric
 #pragma unroll
           for (int p = 0; p < PARTS; ++p) {
             const int32_t part = acc[h * PARTS + p][tid];
-            if (part != 0) S[h] += (__int128)((unsigned __int128)(__int128)part << (16 * p + sb));
+            if (part != 0) {
+              const __int128 v = (__int128)((unsigned __int128)(__int128)part << (16 * p + sb));
+              if constexpr (SREG)
+                S[h] += v;
+              else
+                Ssm[h][tid] += v;
+            }
           }
       }
 #pragma unroll
@@ -128,17 +154,22 @@ __global__ void __launch_bounds__(NT) gemm_exact_kernel(const uint8_t* __restric
   }
 
   if (!live) return;
-  const int lambda = smin + P::TMIN;
+  const int lambda = smin + Lat::TMIN;
   const int64_t o = (int64_t)i * N + j;
+  auto sum_of = [&](int h) -> __int128 {
+    if constexpr (SREG)
+      return S[h];
+    else
+      return Ssm[h][tid];
+  };
   if (C) {
     float out;
     if (in_range) {
       double c = 0.0;
 #pragma unroll
       for (int h = 0; h < L; ++h) {
-        const double sd = i128_to_double(S[h]);
-        const uint64_t cb = L == 8 ? CFP_PHASE_F64_L8_DEV[h] : CFP_PHASE_F64_L4_DEV[h];
-        c = fma(__longlong_as_double((long long)cb), sd, c);
+        const double sd = i128_to_double(sum_of(h));
+        c = fma(__longlong_as_double((long long)Lat::phase64(h)), sd, c);
       }
       out = (float)scalbn(c, lambda);
     } else {
@@ -149,8 +180,9 @@ __global__ void __launch_bounds__(NT) gemm_exact_kernel(const uint8_t* __restric
   if (phase_sums) {
 #pragma unroll
     for (int h = 0; h < L; ++h) {
-      phase_sums[(o * L + h) * 2 + 0] = (int64_t)(uint64_t)S[h];
-      phase_sums[(o * L + h) * 2 + 1] = (int64_t)(S[h] >> 64);
+      const __int128 v = sum_of(h);
+      phase_sums[(o * L + h) * 2 + 0] = (int64_t)(uint64_t)v;
+      phase_sums[(o * L + h) * 2 + 1] = (int64_t)(v >> 64);
     }
   }
   if (phase_lsb) phase_lsb[o] = lambda;
@@ -300,12 +332,19 @@ cudaError_t launch_gemm_exact_oriented(int fa, int fb, int G, const uint8_t* a, 
   return cudaErrorInvalidValue;
 }
 
-template <int FA, int FB>
+template <class Lat>
 static cudaError_t launch_exact_t(int G, const uint8_t* a, const int8_t* sa, const uint8_t* b, const int8_t* sb,
                                   int64_t M, int64_t N, int64_t K, float* c, int64_t* ps, int32_t* pl, uint32_t* st,
                                   cudaStream_t s) {
+  constexpr size_t smem = exact_smem<Lat>();
+  static_assert(smem + 2 * TM * KC <= 227 * 1024, "shared memory");
+  auto kern = gemm_exact_kernel<Lat>;
+  if (smem > 48 * 1024) {
+    const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
   dim3 grid((unsigned)((N + TN - 1) / TN), (unsigned)((M + TM - 1) / TM));
-  gemm_exact_kernel<FA, FB><<<grid, NT, 0, s>>>(a, sa, b, sb, (int)M, (int)N, (int)K, G, c, ps, pl, st);
+  kern<<<grid, NT, smem, s>>>(a, sa, b, sb, (int)M, (int)N, (int)K, G, c, ps, pl, st);
   return cudaGetLastError();
 }
 
@@ -313,7 +352,7 @@ cudaError_t launch_gemm_exact(int fa, int fb, int G, const uint8_t* a, const int
                               const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, int64_t* ps,
                               int32_t* pl, uint32_t* st, cudaStream_t s) {
 #define CFP_E(X, Y) \
-  if (fa == X && fb == Y) return launch_exact_t<X, Y>(G, a, sa, b, sb, M, N, K, c, ps, pl, st, s);
+  if (fa == X && fb == Y) return launch_exact_t<BinLat<X, Y>>(G, a, sa, b, sb, M, N, K, c, ps, pl, st, s);
   CFP_E(CURVEFP_E3C3, CURVEFP_E3C3)
   CFP_E(CURVEFP_E3C3, CURVEFP_E4C3)
   CFP_E(CURVEFP_E3C3, CURVEFP_E5C2)
@@ -324,6 +363,10 @@ cudaError_t launch_gemm_exact(int fa, int fb, int G, const uint8_t* a, const int
   CFP_E(CURVEFP_E5C2, CURVEFP_E4C3)
   CFP_E(CURVEFP_E5C2, CURVEFP_E5C2)
 #undef CFP_E
+  if (fa == CURVEFP_E4C3_R8_9 && fb == CURVEFP_E4C3_R8_9)
+    return launch_exact_t<RadLat<CURVEFP_E4C3_R8_9>>(G, a, sa, b, sb, M, N, K, c, ps, pl, st, s);
+  if (fa == CURVEFP_E4C3_R3_4 && fb == CURVEFP_E4C3_R3_4)
+    return launch_exact_t<RadLat<CURVEFP_E4C3_R3_4>>(G, a, sa, b, sb, M, N, K, c, ps, pl, st, s);
   return cudaErrorInvalidValue;
 }
 

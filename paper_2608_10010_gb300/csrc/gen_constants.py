@@ -15,7 +15,10 @@ Constants (binary radix, K in {4, 8}):
   * MU_Z:   1 + mant/2^23 > 2^{1/K}    iff mant >= MU_Z   (zero boundary).
   * C_K[k]: FP32 bits of RN32(2^{k/K}) (dequantization).
   * Q16_K[k]: round(2^{k/K} 2^16), the tile's integer coefficients (App. C.1).
-  * phase constants 2^{h/L} for L in {4, 8}, as FP32 and FP64 bits.
+  * phase constants 2^{h/L} for L in {4, 8, 9, 32}, as FP32 and FP64 bits.
+  * rational radix r = 2^{p/q} (E4C3 with r = 2^{8/9}, 2^{3/4}): the
+    nearest-level tables per binade class, the ceil-absmax and zero-boundary
+    thresholds and the exact GEMM's address offsets (see radix_params).
 
 Run:  python gen_constants.py > curvefp_constants.h
 """
@@ -166,6 +169,87 @@ def rank_table(E: int, C: int) -> tuple[int, list[int]]:
     return nbin, out
 
 
+# ---- rational radix r = 2^{p/q}, K = 8 (E4C3 variants) ---------------------
+# Level n has exponent lambda(n) = p n / (qK).  For a scaled value y with
+# binade b and 23-bit mantissa mu, the nearest level of the unbounded lattice
+# is n*(y) = N0[b mod PB] + floor(b / PB) NPER + #{i : mu >= THR[b mod PB][i]},
+# N0[c] = n*(2^c) and THR[c] the mantissa thresholds of the level midpoints
+# inside [2^c, 2^{c+1}); the pattern repeats every PB binades (NPER levels).
+RADIX_FORMATS = {"R8_9": (8, 9), "R3_4": (3, 4)}
+RADIX_K, RADIX_NMAX = 8, 63
+RADIX_MAXTHR = 11  # largest number of midpoints in one binade
+
+
+def fixp(num: int, den: int) -> int:
+    """floor(2^{num/den} 2^P) for any integer num (den > 0)."""
+    i, f = divmod(num, den)
+    v = fix_pow2(f, den)
+    return v << i if i >= 0 else v >> (-i)
+
+
+def gcd(a: int, b: int) -> int:
+    while b:
+        a, b = b, a % b
+    return a
+
+
+def radix_params(p: int, q: int) -> dict:
+    K, nmax = RADIX_K, RADIX_NMAX
+    N = q * K
+    g = gcd(p, N)
+    H = N // g
+    PB = p // g          # binades per period
+    NPER = PB * N // p   # levels per period
+    one = 1 << P
+
+    def mid_rel(n: int, c: int) -> int:
+        """floor-ish 2 (2^{lambda(n)-c} + 2^{lambda(n+1)-c}) 2^P / 2 (error < 2 units)."""
+        return fixp(p * n - c * N, N) + fixp(p * (n + 1) - c * N, N)  # = 2 mid / 2^c, 2^P units
+
+    n0, thr = [], []
+    for c in range(PB):
+        # nearest level at y = 2^c
+        n = (c * N) // p  # lambda(n) <= c < lambda(n + 1)
+        if p * n == c * N:
+            nstar = n
+        else:
+            s2 = mid_rel(n, c)            # 2 mid / 2^c in 2^P units
+            assert abs(s2 - 2 * one) > 4
+            nstar = n if 2 * one < s2 else n + 1
+        n0.append(nstar)
+        ts = []
+        for m in range(n - 2, n + NPER + 3):
+            s2 = mid_rel(m, c)
+            if not (2 * one <= s2 < 4 * one):
+                assert abs(s2 - 2 * one) > 4 and abs(s2 - 4 * one) > 4
+                continue
+            frac = s2 - 2 * one           # 2 (mid/2^c - 1), 2^P units
+            shift = P - 23 + 1
+            qq, r = divmod(frac, 1 << shift)
+            assert 4 < r < (1 << shift) - 4, "midpoint too close to an FP32 mantissa"
+            ts.append(qq + 1)
+        assert ts == sorted(ts) and len(ts) <= RADIX_MAXTHR
+        thr.append(ts)
+    for c in range(PB):  # the counts tile the period
+        nxt = n0[c + 1] if c + 1 < PB else n0[0] + NPER
+        assert n0[c] + len(thr[c]) == nxt
+    # ceil-absmax: lambda(nmax) = F + f; MU_SAT = smallest mu with 1 + mu 2^-23 > 2^f
+    F, fnum = divmod(p * nmax, N)
+    mu_sat = 1 if fnum == 0 else mant_threshold_fix(fix_pow2(fnum, N), False)
+    # zero boundary L_nmin / 2 = 2^{lambda(-nmax) - 1} = 2^{ZB} 2^{zf}
+    ZB, zfnum = divmod(-p * nmax - N, N)
+    zthr = 1 if zfnum == 0 else mant_threshold_fix(fix_pow2(zfnum, N), False)
+    # exact GEMM addressing on biased ranks: V = p (m_a + m_b) - R0 + N >= 0,
+    # h = (V mod N) / g, t - t_min = floor(V / N) - OFF
+    B = 64
+    Q, R0 = divmod(2 * p * B, N)
+    us = [p * (na + nb) for na in range(-nmax, nmax + 1) for nb in range(-nmax, nmax + 1)]
+    tmin, tmax = min(u // N for u in us), max(u // N for u in us)
+    off = Q + 1 + tmin
+    return dict(N=N, g=g, H=H, PB=PB, NPER=NPER, N0=n0, THR=thr, F=F, MU_SAT=mu_sat, ZB=ZB, ZTHR=zthr,
+                R0=R0, OFF=off, TMIN=tmin, TMAX=tmax)
+
+
 def main(out=sys.stdout):
     w = out.write
     w("/* Generated by gen_constants.py from exact integer arithmetic; do not edit. */\n")
@@ -189,9 +273,38 @@ def main(out=sys.stdout):
         for i in range(0, len(tab), 8):
             w("  " + ", ".join(f"0x{v:08x}u" for v in tab[i:i + 8]) + ", \\\n")
         w("}\n")
-    for L in (4, 8):
+    for L in (4, 8, 9, 32):
         w(f"#define CFP_PHASE_F32_L{L}_INIT {{" + ", ".join(f"0x{f32_bits_pow2(h, L):08x}u" for h in range(L)) + "}\n")
         w(f"#define CFP_PHASE_F64_L{L}_INIT {{" + ", ".join(f"0x{f64_bits_pow2(h, L):016x}ull" for h in range(L)) + "}\n")
+    for name, (p, q) in RADIX_FORMATS.items():
+        r = radix_params(p, q)
+        w(f"/* E4C3, r = 2^({p}/{q}): N = qK = {r['N']}, H = {r['H']} phases, period {r['PB']} binade(s) / "
+          f"{r['NPER']} levels */\n")
+        for key in ("N", "g", "H", "PB", "NPER", "F", "ZB", "R0", "OFF", "TMIN", "TMAX"):
+            w(f"#define CFP_{name}_{key} ({r[key]})\n")
+        w(f"#define CFP_{name}_MU_SAT 0x{r['MU_SAT']:06x}u\n")
+        w(f"#define CFP_{name}_ZTHR 0x{r['ZTHR']:06x}u\n")
+        w(f"#define CFP_{name}_N0_INIT {{" + ", ".join(str(v) for v in r["N0"]) + "}\n")
+        w(f"#define CFP_{name}_CNT_INIT {{" + ", ".join(str(len(t)) for t in r["THR"]) + "}\n")
+        rows = []
+        for t in r["THR"]:
+            rows += t + [1 << 23] * (RADIX_MAXTHR - len(t))  # padding is never reached
+        w(f"#define CFP_{name}_THR_INIT {{" + ", ".join(f"0x{v:06x}u" for v in rows) + "}\n")
+        # bucket LUT per class (as lut_for): top 8 mantissa bits -> thresholds
+        # passed by the whole bucket << 24 | the one threshold inside it
+        lut = []
+        for t in r["THR"]:
+            assert all(b - a > (1 << 15) for a, b in zip(t, t[1:]))
+            for idx in range(256):
+                lo, hi = idx << 15, (idx + 1) << 15
+                inside = [v for v in t if lo < v < hi]
+                assert len(inside) <= 1
+                lut.append((sum(1 for v in t if v <= lo) << 24) | (inside[0] if inside else (1 << 23)))
+        w(f"#define CFP_{name}_LUT_INIT {{ \\\n")
+        for i in range(0, len(lut), 8):
+            w("  " + ", ".join(f"0x{v:08x}u" for v in lut[i:i + 8]) + ", \\\n")
+        w("}\n")
+    w(f"#define CFP_RADIX_MAXTHR {RADIX_MAXTHR}\n")
 
 
 if __name__ == "__main__":

@@ -121,6 +121,26 @@ def test_oriented_gemm_validation(lib):
     assert call(algo=0, ps=d, pl=None) == INVALID      # exact: both phase arrays or neither
 
 
+def test_rational_radix_host_rules(lib):
+    """The rational-radix formats: phase counts (Table 7: 9 and 32), pairing
+    only with themselves, and the entry points that do not take them."""
+    P = ctypes.c_void_p
+    d = P(4096)
+    INVALID, UNSUPPORTED = 1, 2
+    assert lib.curvefp_phase_count(3, 3) == 9 and lib.curvefp_phase_count(4, 4) == 32
+    assert lib.curvefp_phase_count(3, 1) == -1 and lib.curvefp_phase_count(4, 3) == -1
+    assert lib.curvefp_phase_count(5, 5) == -1
+    # quantize: block axis 1 is not provided for them
+    assert lib.curvefp_quantize(3, 32, d, 0, 64, 64, 64, 1, d, d, None, None) == UNSUPPORTED
+    assert lib.curvefp_quantize(5, 32, d, 0, 4, 64, 64, 0, d, d, None, None) == INVALID
+    # GEMM: mixed radix, and the tensor-core algorithms
+    assert lib.curvefp_gemm(0, 3, 1, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED
+    assert lib.curvefp_gemm(1, 3, 3, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED
+    assert lib.curvefp_gemm(2, 4, 4, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED
+    assert lib.curvefp_gemm_q32(3, 3, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED
+    assert lib.curvefp_quantize_static(3, 32, 0, 0, d, 0, 4, 64, d, d, None, 0, None, None) == UNSUPPORTED
+
+
 def test_product_path_does_not_touch_the_oracle():
     """The CUDA library and its binding neither import nor link the oracle."""
     pkg = os.path.join(ROOT, "paper_2608_10010_gb300")
