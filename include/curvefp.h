@@ -55,9 +55,11 @@ extern "C" {
  * 2^{63 p/(8q)}; an exact tie in the nearest-level search (only between zero
  * and L_nmin = 2^{-7} for r = 2^{8/9}) goes to zero; dequantization is
  * RN32(RN32(2^{j/(8q)}) 2^{a_b + floor(p n/(8q))}), j = p n mod 8q.  They are
- * accepted by curvefp_quantize (block_axis 0), curvefp_dequantize and the
- * EXACT GEMMs (both operands of the same format); every other entry point
- * returns CURVEFP_ERR_UNSUPPORTED for them. */
+ * accepted by curvefp_quantize, curvefp_quantize_static (and its variants),
+ * curvefp_dequantize, curvefp_gemm_requant's destination and the EXACT GEMMs
+ * (curvefp_gemm, curvefp_gemm_phases; both operands of the same format); the
+ * tensor-core algorithms, curvefp_gemm_q32 and curvefp_gemm_oriented return
+ * CURVEFP_ERR_UNSUPPORTED for them. */
 typedef enum {
   CURVEFP_E3C3 = 0,
   CURVEFP_E4C3 = 1,

@@ -36,7 +36,6 @@ curvefp_status_t curvefp_quantize(curvefp_format_t fmt, int block, const void* x
   if (!fmt_any(fmt) || !block_ok(block) || (dtype != CURVEFP_F32 && dtype != CURVEFP_BF16)) return CURVEFP_ERR_INVALID_ARG;
   if (block_axis != 0 && block_axis != 1) return CURVEFP_ERR_INVALID_ARG;
   if (rows < 0 || cols < 0 || ld < cols) return CURVEFP_ERR_INVALID_ARG;
-  if (fmt_radix(fmt) && block_axis != 0) return CURVEFP_ERR_UNSUPPORTED;
   if (rows == 0 || cols == 0) return CURVEFP_OK;
   if (!x || !codes || !scales) return CURVEFP_ERR_INVALID_ARG;
   const int64_t esz = dtype == CURVEFP_F32 ? 4 : 2;
@@ -48,8 +47,8 @@ curvefp_status_t curvefp_quantize(curvefp_format_t fmt, int block, const void* x
   if (block_axis == 1 && rows / block > 65535) return CURVEFP_ERR_UNSUPPORTED;
   if (rows * cols / block > (int64_t)1 << 40) return CURVEFP_ERR_UNSUPPORTED;
   if (fmt_radix(fmt))
-    return from_cuda(cfp::launch_quantize_radix(fmt, block, x, dtype, rows, cols, ld, codes, scales, device_status,
-                                                static_cast<cudaStream_t>(stream), sm_count()));
+    return from_cuda(cfp::launch_quantize_radix(fmt, block, x, dtype, rows, cols, ld, block_axis, codes, scales,
+                                                device_status, static_cast<cudaStream_t>(stream), sm_count()));
   return from_cuda(cfp::launch_quantize(fmt, block, x, dtype, rows, cols, ld, block_axis, codes, scales,
                                         device_status, static_cast<cudaStream_t>(stream), sm_count()));
 }
@@ -63,8 +62,7 @@ curvefp_status_t curvefp_quantize_static(curvefp_format_t fmt, int block, curvef
                                          curvefp_scale_rule_t rule, const void* x, curvefp_dtype_t dtype, int64_t rows,
                                          int64_t cols, uint8_t* codes, int8_t* scales, void* workspace,
                                          size_t workspace_bytes, uint32_t* device_status, void* stream) {
-  if (fmt_radix(fmt)) return CURVEFP_ERR_UNSUPPORTED;
-  if (!fmt_ok(fmt) || !block_ok(block) || (dtype != CURVEFP_F32 && dtype != CURVEFP_BF16)) return CURVEFP_ERR_INVALID_ARG;
+  if (!fmt_any(fmt) || !block_ok(block) || (dtype != CURVEFP_F32 && dtype != CURVEFP_BF16)) return CURVEFP_ERR_INVALID_ARG;
   if (group < CURVEFP_SCALE_BLOCK || group > CURVEFP_SCALE_TENSOR) return CURVEFP_ERR_INVALID_ARG;
   if (rule != CURVEFP_SCALE_CEIL_ABSMAX && rule != CURVEFP_SCALE_MSE) return CURVEFP_ERR_INVALID_ARG;
   if (rows < 0 || cols < 0) return CURVEFP_ERR_INVALID_ARG;
@@ -76,6 +74,10 @@ curvefp_status_t curvefp_quantize_static(curvefp_format_t fmt, int block, curvef
   if (need && (!workspace || workspace_bytes < need || (reinterpret_cast<uintptr_t>(workspace) & 15) != 0))
     return CURVEFP_ERR_INVALID_ARG;
   if (rows * cols > (int64_t)1 << 40) return CURVEFP_ERR_UNSUPPORTED;
+  if (fmt_radix(fmt))
+    return from_cuda(cfp::launch_quantize_static_radix(fmt, block, group, rule, x, dtype, rows, cols, codes, scales,
+                                                       workspace, device_status, static_cast<cudaStream_t>(stream),
+                                                       sm_count()));
   return from_cuda(cfp::launch_quantize_static(fmt, block, group, rule, x, dtype, rows, cols, codes, scales, workspace,
                                                device_status, static_cast<cudaStream_t>(stream), sm_count()));
 }

@@ -250,6 +250,36 @@ def radix_params(p: int, q: int) -> dict:
                 R0=R0, OFF=off, TMIN=tmin, TMAX=tmax)
 
 
+def radix_rank_table(r: dict) -> tuple[int, list[int]]:
+    """rank_table for a rational radix: binades ZB - 1 .. F of the scaled
+    value (nothing above F occurs under the block's own ceil-absmax scale;
+    keys of smaller values clamp to the all-zero binade ZB - 1), same entry
+    layout; ranks from the nearest-level rule of radix_params."""
+    B, nmax = 64, RADIX_NMAX
+
+    def rank(F: int, mant: int) -> int:
+        if F < r["ZB"] or (F == r["ZB"] and mant < r["ZTHR"]):
+            return 0
+        k, c = divmod(F, r["PB"])
+        n = r["N0"][c] + k * r["NPER"] + sum(1 for t in r["THR"][c] if mant >= t)
+        return min(max(n, -nmax), nmax) + B
+
+    nbin = r["F"] - r["ZB"] + 2
+    out = []
+    for fo in range(nbin):
+        F = r["ZB"] - 1 + fo
+        thr = r["THR"][F % r["PB"]] + ([r["ZTHR"]] if F == r["ZB"] else [])
+        for m7 in range(128):
+            lo, hi = m7 << 16, (m7 << 16) | 0xFFFF
+            r_lo, r_hi = rank(F, lo), rank(F, hi)
+            cuts = [t for t in thr if lo < t <= hi and rank(F, t - 1) != rank(F, t)]
+            assert len(cuts) <= 1
+            if not cuts:
+                assert r_lo == r_hi
+            out.append(r_lo | (r_hi << 8) | (((cuts[0] & 0xFFFF) if cuts else 0) << 16))
+    return nbin, out
+
+
 def main(out=sys.stdout):
     w = out.write
     w("/* Generated by gen_constants.py from exact integer arithmetic; do not edit. */\n")
@@ -300,6 +330,12 @@ def main(out=sys.stdout):
                 inside = [v for v in t if lo < v < hi]
                 assert len(inside) <= 1
                 lut.append((sum(1 for v in t if v <= lo) << 24) | (inside[0] if inside else (1 << 23)))
+        nbin, tab = radix_rank_table(r)
+        w(f"#define CFP_RANK_E4C3_{name}_NBIN {nbin}\n")
+        w(f"#define CFP_RANK_E4C3_{name}_INIT {{ \\\n")
+        for i in range(0, len(tab), 8):
+            w("  " + ", ".join(f"0x{v:08x}u" for v in tab[i:i + 8]) + ", \\\n")
+        w("}\n")
         w(f"#define CFP_{name}_LUT_INIT {{ \\\n")
         for i in range(0, len(lut), 8):
             w("  " + ", ".join(f"0x{v:08x}u" for v in lut[i:i + 8]) + ", \\\n")

@@ -26,7 +26,11 @@ cudaError_t launch_gemm_tensor_sparse(int fa, int fb, int G, const uint8_t* a, c
 bool gemm_tensor_supported(int fa, int fb);
 bool is_radix_format(int fmt);
 cudaError_t launch_quantize_radix(int fmt, int G, const void* x, int dtype, int64_t rows, int64_t cols, int64_t ld,
-                                  uint8_t* codes, int8_t* scales, uint32_t* status, cudaStream_t st, int sms);
+                                  int axis, uint8_t* codes, int8_t* scales, uint32_t* status, cudaStream_t st,
+                                  int sms);
+cudaError_t launch_quantize_static_radix(int fmt, int G, int group, int rule, const void* x, int dtype, int64_t rows,
+                                         int64_t cols, uint8_t* codes, int8_t* scales, void* ws, uint32_t* status,
+                                         cudaStream_t st, int sms);
 cudaError_t launch_dequantize_radix(int fmt, int G, const uint8_t* codes, const int8_t* scales, int64_t n, float* out,
                                     cudaStream_t st, int sms);
 cudaError_t launch_gemm_exact_oriented(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, int la,

@@ -130,15 +130,15 @@ def test_rational_radix_host_rules(lib):
     assert lib.curvefp_phase_count(3, 3) == 9 and lib.curvefp_phase_count(4, 4) == 32
     assert lib.curvefp_phase_count(3, 1) == -1 and lib.curvefp_phase_count(4, 3) == -1
     assert lib.curvefp_phase_count(5, 5) == -1
-    # quantize: block axis 1 is not provided for them
-    assert lib.curvefp_quantize(3, 32, d, 0, 64, 64, 64, 1, d, d, None, None) == UNSUPPORTED
+    # quantize: the same shape rules as the binary formats; unknown ids rejected
+    assert lib.curvefp_quantize(3, 32, d, 0, 48, 64, 64, 1, d, d, None, None) == INVALID
     assert lib.curvefp_quantize(5, 32, d, 0, 4, 64, 64, 0, d, d, None, None) == INVALID
     # GEMM: mixed radix, and the tensor-core algorithms
     assert lib.curvefp_gemm(0, 3, 1, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED
     assert lib.curvefp_gemm(1, 3, 3, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED
     assert lib.curvefp_gemm(2, 4, 4, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED
     assert lib.curvefp_gemm_q32(3, 3, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED
-    assert lib.curvefp_quantize_static(3, 32, 0, 0, d, 0, 4, 64, d, d, None, 0, None, None) == UNSUPPORTED
+    assert lib.curvefp_quantize_static(3, 32, 1, 0, d, 0, 4, 64, d, d, None, 0, None, None) == INVALID  # no workspace
 
 
 def test_product_path_does_not_touch_the_oracle():

@@ -22,14 +22,14 @@ def torch():
     return t
 
 
-def check_q(torch, x, fmt, block, dtype="f32"):
+def check_q(torch, x, fmt, block, dtype="f32", axis=0):
     import paper_2608_10010_gb300 as cfp
 
     xd = to_dev(torch, x, dtype)
     st = new_status(torch)
-    codes, scales = cfp.quantize(xd, fmt, block, 0, status=st)
+    codes, scales = cfp.quantize(xd, fmt, block, axis, status=st)
     torch.cuda.synchronize()
-    rc, rs, nan = oracle.quantize(widen(torch, xd), fmt, block, 0)
+    rc, rs, nan = oracle.quantize(widen(torch, xd), fmt, block, axis)
     assert np.array_equal(scales.cpu().numpy(), rs), (fmt, block, dtype)
     assert np.array_equal(codes.cpu().numpy(), rc), (fmt, block, dtype)
     assert bool(status_bits(st) & 1) == nan
@@ -67,6 +67,45 @@ def test_quantize_distributions(torch, fmt, dtype, block):
     wide = (2.0 ** rng.uniform(-140, 120, (40, 1024))).astype(np.float32)
     wide *= np.where(rng.random((40, 1024)) < 0.5, -1, 1).astype(np.float32)
     check_q(torch, wide, fmt, block, dtype)
+
+
+@pytest.mark.parametrize("fmt", RADIX)
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_quantize_shapes_and_paths(torch, fmt, dtype):
+    """Every kernel path of the shared quantizer: dense G32 rows (bulk-fed),
+    strided rows (register-fed), G 64..512, and block axis 1 (transposed
+    output)."""
+    x = inputs.elementwise_outliers((37, 1024), 8)
+    for block in (32, 64, 128, 256, 512):
+        check_q(torch, x, fmt, block, dtype)
+    y = inputs.elementwise_outliers((1024, 40), 9)
+    for block in (32, 64, 512):
+        check_q(torch, y, fmt, block, dtype, axis=1)
+    # a strided view (ld > cols): the register-fed kernel
+    import paper_2608_10010_gb300 as cfp
+
+    big = to_dev(torch, inputs.outlier_channels((64, 1536), 10), dtype)
+    view = big[:, :1024]
+    st = new_status(torch)
+    codes, scales = cfp.quantize(view, fmt, 32, 0, status=st)
+    torch.cuda.synchronize()
+    rc, rs, _ = oracle.quantize(np.ascontiguousarray(widen(torch, view)), fmt, 32, 0)
+    assert np.array_equal(codes.cpu().numpy(), rc) and np.array_equal(scales.cpu().numpy(), rs)
+
+
+@pytest.mark.parametrize("fmt", RADIX)
+@pytest.mark.parametrize("group,rule", [("block", "mse"), ("row", "mse"), ("tensor", "ceil")])
+def test_quantize_static(torch, fmt, group, rule):
+    """Static-operand scales (block / row / tensor groups, MSE search) with
+    the rational levels, bit-exact against the oracle."""
+    import paper_2608_10010_gb300 as cfp
+
+    x = inputs.normal((48, 1024), 11, 0.02)
+    xd = to_dev(torch, x)
+    codes, scales = cfp.quantize_static(xd, fmt, 512, group, rule)
+    torch.cuda.synchronize()
+    rc, rs, _ = oracle.quantize_static(x, fmt, 512, group, rule)
+    assert np.array_equal(scales.cpu().numpy(), rs) and np.array_equal(codes.cpu().numpy(), rc)
 
 
 @pytest.mark.parametrize("fmt", RADIX)
