@@ -205,6 +205,13 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
                   flush_l2, reps=3, warm=1)
     res["gemm_q32"] = {"workload": "E4C3 1024x1024x4096", "ms": round(ms, 4),
                        "gmac_per_s": round(1024 * 1024 * 4096 / (ms / 1e3) / 1e9, 1)}
+    # the histogram accumulation layout (signed-popcount merged counts), a
+    # validation GEMM: 256 x 256 x 4096 of the same operands
+    ah, sah, bh, sbh = aq[:256].contiguous(), saq[:256].contiguous(), bq[:256].contiguous(), sbq[:256].contiguous()
+    ms = _time_ms(torch, stream, lambda: cfp.gemm_phases_histogram(ah, sah, bh, sbh, "E4C3", "E4C3", G, stream=stream),
+                  flush_l2, reps=3, warm=1)
+    res["gemm_histogram"] = {"workload": "E4C3 256x256x4096", "ms": round(ms, 4),
+                             "gmac_per_s": round(256 * 256 * 4096 / (ms / 1e3) / 1e9, 1)}
     del Xq, Wq, aq, saq, bq, sbq, outq
     # rational radix (E4C3 with r = 2^{8/9}, 2^{3/4}; the radix-frontier
     # setting G512): quantizer bandwidth and the exact 9- / 32-phase GEMM

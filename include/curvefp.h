@@ -45,9 +45,8 @@
 extern "C" {
 #endif
 
-/* Table 1: E3C3 (CurveFP7, 7 bits, 63 positive levels, H = 8), E4C3 and E5C2
- * (CurveFP8, 8 bits, 127 positive levels, H = 8 and 4). */
-/* E3C3 (CurveFP7), E4C3 and E5C2 (CurveFP8): Table 1, binary radix.
+/* E3C3 (CurveFP7, 7 bits, 63 positive levels, H = 8), E4C3 and E5C2
+ * (CurveFP8, 8 bits, 127 positive levels, H = 8 and 4): Table 1, binary radix.
  * E4C3_R8_9, E4C3_R3_4: E4C3 codes with the rational radices r = 2^{8/9}
  * (9 phases) and r = 2^{3/4} (32 phases) of the radix frontier (Sec. 3.1
  * Eq. 1 with r = 2^{p/q}, Eq. 4, Table 7): level x = (-1)^s 2^{a_b}
@@ -246,6 +245,18 @@ curvefp_status_t curvefp_gemm_oriented(curvefp_gemm_algo_t algo, curvefp_format_
                                        int64_t N, int64_t K, float* c, int64_t* phase_sums, int32_t* phase_lsb,
                                        void* workspace, size_t workspace_bytes, uint32_t* device_status,
                                        void* stream);
+
+/* curvefp_gemm_phases computed with the histogram layout (Eq. 5, App. A.1:
+ * "equal addresses can be merged with signed popcounts"): every product's
+ * address (phase h, bin t) is counted in a per-output histogram n_{h,t}
+ * (lanes of a warp with equal addresses merge by signed popcount), and
+ * S_h = sum_t n_{h,t} 2^t.  Same outputs, requirements and format pairs as
+ * curvefp_gemm_phases (rational radices included); the phase sums are
+ * bit-identical to it.  Validation kernel (one warp per output). */
+curvefp_status_t curvefp_gemm_phases_histogram(curvefp_format_t fmt_a, curvefp_format_t fmt_b, int block,
+                                               const uint8_t* a, const int8_t* sa, const uint8_t* b, const int8_t* sb,
+                                               int64_t M, int64_t N, int64_t K, float* c, int64_t* phase_sums,
+                                               int32_t* phase_lsb, uint32_t* device_status, void* stream);
 
 /* GEMM followed by output requantization (Sec. 3.2: closure holds on the
  * widened product coordinates; the explicit requantization to an E-bit

@@ -43,6 +43,7 @@ def load(build_if_missing: bool = False):
         lib.curvefp_dequantize.argtypes = [I, I, P, P, L, L, P, P]
         lib.curvefp_gemm.argtypes = [I, I, I, I, P, P, P, P, L, L, L, P, P, P]
         lib.curvefp_gemm_phases.argtypes = [I, I, I, P, P, P, P, L, L, L, P, P, P, P, P]
+        lib.curvefp_gemm_phases_histogram.argtypes = [I, I, I, P, P, P, P, L, L, L, P, P, P, P, P]
         lib.curvefp_phase_count.argtypes = [I, I]
         lib.curvefp_quantize_static_workspace.argtypes = [L, L, I, I]
         lib.curvefp_quantize_static_workspace.restype = ctypes.c_size_t
@@ -59,7 +60,7 @@ def load(build_if_missing: bool = False):
         lib.curvefp_version.restype = ctypes.c_char_p
         for f in ("curvefp_quantize", "curvefp_quantize_static", "curvefp_quantize_static_noalloc",
                   "curvefp_dequantize", "curvefp_gemm", "curvefp_gemm_phases", "curvefp_gemm_q32",
-                  "curvefp_gemm_requant", "curvefp_gemm_oriented"):
+                  "curvefp_gemm_requant", "curvefp_gemm_oriented", "curvefp_gemm_phases_histogram"):
             getattr(lib, f).restype = I
         _lib = lib
     return _lib
@@ -245,6 +246,22 @@ def gemm_q32(a, sa, b, sb, fmt_a, fmt_b, block: int = 32, out=None, status=None,
     _check(load().curvefp_gemm_q32(_fmt(fmt_a), _fmt(fmt_b), block, _p(a), _p(sa), _p(b), _p(sb), M, N, K, _p(out),
                                    _p(status), _stream(stream)))
     return out
+
+
+def gemm_phases_histogram(a, sa, b, sb, fmt_a, fmt_b, block: int = 32, status=None, stream=None):
+    """gemm_phases computed with the histogram layout (signed-popcount merged
+    counts n_{h,t}); returns (C, phase sums, LSBs) like gemm_phases."""
+    import torch
+
+    M, K = a.shape
+    N = b.shape[0]
+    H = phase_count(fmt_a, fmt_b)
+    c = torch.empty((M, N), dtype=torch.float32, device=a.device)
+    ps = torch.empty((M, N, H, 2), dtype=torch.int64, device=a.device)
+    pl = torch.empty((M, N), dtype=torch.int32, device=a.device)
+    _check(load().curvefp_gemm_phases_histogram(_fmt(fmt_a), _fmt(fmt_b), block, _p(a), _p(sa), _p(b), _p(sb), M, N,
+                                                K, _p(c), _p(ps), _p(pl), _p(status), _stream(stream)))
+    return c, ps, pl
 
 
 def gemm_phases(a, sa, b, sb, fmt_a, fmt_b, block: int = 32, status=None, stream=None):

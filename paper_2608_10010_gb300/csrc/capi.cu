@@ -216,6 +216,17 @@ curvefp_status_t curvefp_gemm_oriented(curvefp_gemm_algo_t algo, curvefp_format_
                                                  workspace, device_status, st));
 }
 
+curvefp_status_t curvefp_gemm_phases_histogram(curvefp_format_t fmt_a, curvefp_format_t fmt_b, int block,
+                                               const uint8_t* a, const int8_t* sa, const uint8_t* b, const int8_t* sb,
+                                               int64_t M, int64_t N, int64_t K, float* c, int64_t* phase_sums,
+                                               int32_t* phase_lsb, uint32_t* device_status, void* stream) {
+  curvefp_status_t r = gemm_args(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K);
+  if (r != CURVEFP_OK) return r;
+  if (!phase_sums || !phase_lsb) return CURVEFP_ERR_INVALID_ARG;
+  return from_cuda(cfp::launch_gemm_hist(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, phase_sums, phase_lsb,
+                                         device_status, static_cast<cudaStream_t>(stream), sm_count()));
+}
+
 curvefp_status_t curvefp_gemm_requant(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, curvefp_format_t fmt_b,
                                       int block, const uint8_t* a, const int8_t* sa, const uint8_t* b,
                                       const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c,
