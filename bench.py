@@ -166,17 +166,19 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
     def q(t, fmt, axis):
         return cfp.quantize(t, fmt, G, axis, stream=stream)
 
-    def gemm_case(name, A, fa, B, fb, planes, hbm_bound=False):
+    def gemm_case(name, A, fa, B, fb, planes, hbm_bound=False, algo="tensor"):
         a, sa = A
         b, sb = B
         Mx, Kx = a.shape
         Nx = b.shape[0]
         out = torch.empty((Mx, Nx), dtype=torch.float32, device=a.device)
-        ms = _time_ms(torch, stream, lambda: cfp.gemm(a, sa, b, sb, fa, fb, G, "tensor", out=out, stream=stream),
+        ms = _time_ms(torch, stream, lambda: cfp.gemm(a, sa, b, sb, fa, fb, G, algo, out=out, stream=stream),
                       flush_l2)
         tops = 2.0 * Mx * Nx * Kx / (ms / 1e3) / 1e12
-        r = {"case": name, "M": Mx, "N": Nx, "K": Kx, "formats": f"{fa}x{fb}", "ms": round(ms, 4),
-             "tops": round(tops, 3), "tensor_work_frac": round(tops * planes / fp8_peak, 4)}
+        r = {"case": name, "algo": algo, "M": Mx, "N": Nx, "K": Kx, "formats": f"{fa}x{fb}", "ms": round(ms, 4),
+             "tops": round(tops, 3)}
+        if algo == "tensor":
+            r["tensor_work_frac"] = round(tops * planes / fp8_peak, 4)
         if hbm_bound:
             wbytes = Nx * Kx + Nx * Kx // G
             r["weight_code_gbs"] = round(wbytes / (ms / 1e3) / 1e9, 1)
@@ -265,6 +267,9 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
             Xf, Wf = inputs.ffn_cuda(Mf, Kf)
             gemm_case(f"ffn M={Mf} K={Kf}", q(Xf, "E3C3", 0), "E3C3", q(Wf, "E3C3", 1), "E3C3", 64,
                       hbm_bound=Mf <= 128)
+            if Mf <= 8:  # decode sizes: the CUDA-core kernel as well
+                gemm_case(f"ffn M={Mf} K={Kf} skinny", q(Xf, "E3C3", 0), "E3C3", q(Wf, "E3C3", 1), "E3C3", 64,
+                          hbm_bound=True, algo="skinny")
             del Xf, Wf
     torch.cuda.empty_cache()
     return res

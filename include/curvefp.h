@@ -81,12 +81,20 @@ typedef enum {
  * kernel over power-of-two phase planes with FP32 per-phase accumulation, one
  * plane pair per dense MMA.  TENSOR_SPARSE: the same method with two plane
  * pairs per 2:4-sparse MMA (half the tensor work, more producer arithmetic;
- * code tiles streamed by TMA). */
+ * code tiles streamed by TMA).  SKINNY: decode-sized GEMMs (M <=
+ * CURVEFP_SKINNY_MAX_M) on the CUDA cores with the same FP32 per-phase
+ * accumulation, every product formed from the two codes (the tensor-core
+ * tile costs the same for any M up to 128).  AUTO: SKINNY for M <=
+ * CURVEFP_AUTO_SKINNY_M, else TENSOR. */
 typedef enum {
   CURVEFP_GEMM_EXACT = 0,
   CURVEFP_GEMM_TENSOR = 1,
-  CURVEFP_GEMM_TENSOR_SPARSE = 2
+  CURVEFP_GEMM_TENSOR_SPARSE = 2,
+  CURVEFP_GEMM_SKINNY = 3,
+  CURVEFP_GEMM_AUTO = 4
 } curvefp_gemm_algo_t;
+#define CURVEFP_SKINNY_MAX_M 8
+#define CURVEFP_AUTO_SKINNY_M 4
 
 /* Bits of the device status word. */
 #define CURVEFP_DEV_NAN 1u     /* quantize: a NaN input was encoded as 0x00        */
@@ -184,7 +192,11 @@ curvefp_status_t curvefp_dequantize(curvefp_format_t fmt, int block, const uint8
  * TENSOR, TENSOR_SPARSE: S_h accumulated in FP32 on the tensor cores, combine
  *   in FP32; plane values below 2^-14 of a row's largest block scale flush.
  *   Format pairs: E3C3 x E3C3, E4C3 x E4C3, E5C2 x E4C3, E4C3 x E5C2,
- *   E5C2 x E5C2 (others return CURVEFP_ERR_UNSUPPORTED). */
+ *   E5C2 x E5C2 (others return CURVEFP_ERR_UNSUPPORTED).
+ * SKINNY (M <= CURVEFP_SKINNY_MAX_M, else CURVEFP_ERR_UNSUPPORTED), AUTO:
+ *   S_h accumulated in FP32 per output (products relative to the output's
+ *   largest scale sum; products below the FP32 normal range relative to it
+ *   flush), combine in FP32; every binary-radix format pair. */
 curvefp_status_t curvefp_gemm(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, curvefp_format_t fmt_b, int block,
                               const uint8_t* a, const int8_t* sa, const uint8_t* b, const int8_t* sb, int64_t M,
                               int64_t N, int64_t K, float* c, uint32_t* device_status, void* stream);

@@ -141,8 +141,14 @@ curvefp_status_t curvefp_gemm(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, 
   if (algo == CURVEFP_GEMM_EXACT)
     return from_cuda(cfp::launch_gemm_exact(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, nullptr, nullptr,
                                             device_status, st));
-  if ((algo == CURVEFP_GEMM_TENSOR || algo == CURVEFP_GEMM_TENSOR_SPARSE) && fmt_radix(fmt_a))
-    return CURVEFP_ERR_UNSUPPORTED;
+  if (algo != CURVEFP_GEMM_EXACT && fmt_radix(fmt_a)) return CURVEFP_ERR_UNSUPPORTED;
+  // AUTO: the CUDA-core kernel where it is faster than a 128-row tensor-core
+  // tile (measured up to M = 4 on the FFN decode shapes)
+  if (algo == CURVEFP_GEMM_AUTO) algo = M <= CURVEFP_AUTO_SKINNY_M ? CURVEFP_GEMM_SKINNY : CURVEFP_GEMM_TENSOR;
+  if (algo == CURVEFP_GEMM_SKINNY) {
+    if (M > CURVEFP_SKINNY_MAX_M) return CURVEFP_ERR_UNSUPPORTED;
+    return from_cuda(cfp::launch_gemm_skinny(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, st, sm_count()));
+  }
   if (algo == CURVEFP_GEMM_TENSOR || algo == CURVEFP_GEMM_TENSOR_SPARSE) {
     if (!cfp::gemm_tensor_supported(fmt_a, fmt_b)) return CURVEFP_ERR_UNSUPPORTED;
     if (algo == CURVEFP_GEMM_TENSOR_SPARSE)

@@ -25,6 +25,8 @@ cudaError_t launch_gemm_tensor_sparse(int fa, int fb, int G, const uint8_t* a, c
                                       cudaStream_t st);
 bool gemm_tensor_supported(int fa, int fb);
 bool is_radix_format(int fmt);
+cudaError_t launch_gemm_skinny(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
+                               const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, cudaStream_t st, int sms);
 cudaError_t launch_gemm_hist(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
                              const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, int64_t* phase_sums,
                              int32_t* phase_lsb, uint32_t* status, cudaStream_t st, int sms);

@@ -67,6 +67,8 @@ def test_host_side_validation(lib):
     assert lib.curvefp_quantize(1, 32, None, 0, 0, 64, 64, 0, None, None, None, None) == 0
     assert lib.curvefp_dequantize(1, 32, None, None, 0, 64, None, None) == 0
     assert lib.curvefp_dequantize(1, 32, dummy, dummy, 4, 48, dummy, None) == INVALID
+    # GEMM: SKINNY takes at most CURVEFP_SKINNY_MAX_M (8) rows
+    assert lib.curvefp_gemm(3, 1, 1, 32, dummy, dummy, dummy, dummy, 9, 4, 64, dummy, None, None) == 2
     # GEMM: K not a multiple of the block, non-positive sizes, bad algo
     assert lib.curvefp_gemm(0, 1, 1, 32, dummy, dummy, dummy, dummy, 4, 4, 48, dummy, None, None) == INVALID
     assert lib.curvefp_gemm(0, 1, 1, 32, dummy, dummy, dummy, dummy, 0, 4, 64, dummy, None, None) == INVALID

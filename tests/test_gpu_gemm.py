@@ -288,3 +288,49 @@ def test_gemm_requant(torch, algo, fa, fb, fc):
     assert normalised_error(c, ref["C"], na, nb) <= TOL
     rc, rs, _ = oracle.quantize(c, fc, 32, 0)
     assert np.array_equal(codes.cpu().numpy(), rc) and np.array_equal(scales.cpu().numpy(), rs)
+
+
+# ---- decode-sized GEMMs on the CUDA cores ------------------------------------
+
+@pytest.mark.parametrize("fa,fb", [(a, b) for a in ("E3C3", "E4C3", "E5C2") for b in ("E3C3", "E4C3", "E5C2")])
+@pytest.mark.parametrize("M", [1, 3, 8])
+def test_skinny_within_tolerance(torch, fa, fb, M):
+    """SKINNY (FP32 per-phase accumulation of exact powers of two, M <= 8):
+    within 1e-5 of the oracle; N = 300 leaves a partial CTA of rows."""
+    import paper_2608_10010_gb300 as cfp
+
+    N, K, G = 300, 1024, 32
+    a, sa = quantized(inputs.lognormal_channels((M, K), 20 + M), fa, G)
+    b, sb = quantized(inputs.normal((N, K), 21, 0.02), fb, G)
+    st = new_status(torch)
+    c = cfp.gemm(to_dev(torch, a), to_dev(torch, sa), to_dev(torch, b), to_dev(torch, sb), fa, fb, G, "skinny",
+                 status=st)
+    torch.cuda.synchronize()
+    ref = oracle.gemm(a, sa, b, sb, fa, fb, G, phases=False)
+    na, nb = oracle.row_norms(a, sa, fa, G), oracle.row_norms(b, sb, fb, G)
+    assert status_bits(st) == 0
+    assert normalised_error(c.cpu().numpy(), ref["C"], na, nb) <= TOL
+
+
+@pytest.mark.parametrize("M", [1, 8])
+def test_skinny_ffn_full_size_sampled(torch, M):
+    """The decode shapes of the FFN sweep (E3C3, W[14336 x 4096]) through
+    SKINNY: 256 sampled columns against the oracle; AUTO (SKINNY up to M = 4,
+    else TENSOR) equal to the kernel it picks, bit for bit."""
+    import paper_2608_10010_gb300 as cfp
+
+    G = 32
+    Xf, Wf = inputs.ffn_cuda(M, 4096)
+    a, sa = cfp.quantize(Xf, "E3C3", G, 0)
+    b, sb = cfp.quantize(Wf, "E3C3", G, 1)
+    c = cfp.gemm(a, sa, b, sb, "E3C3", "E3C3", G, "skinny")
+    c2 = cfp.gemm(a, sa, b, sb, "E3C3", "E3C3", G, "auto")
+    c3 = cfp.gemm(a, sa, b, sb, "E3C3", "E3C3", G, "skinny" if M <= 4 else "tensor")
+    torch.cuda.synchronize()
+    assert torch.equal(c2.view(torch.int32), c3.view(torch.int32))
+    jj = np.sort(np.random.default_rng(3).choice(b.shape[0], 256, replace=False))
+    ah, sah = a.cpu().numpy(), sa.cpu().numpy()
+    bh, sbh = b.cpu().numpy()[jj], sb.cpu().numpy()[jj]
+    ref = oracle.gemm(ah, sah, bh, sbh, "E3C3", "E3C3", G, phases=False)
+    na, nb = oracle.row_norms(ah, sah, "E3C3", G), oracle.row_norms(bh, sbh, "E3C3", G)
+    assert normalised_error(c.cpu().numpy()[:, jj], ref["C"], na, nb) <= TOL
