@@ -13,8 +13,9 @@
 //
 // A warp owns one weight row j (one output column) at a time: its lanes read
 // 16 consecutive codes each (512 contiguous bytes per warp step), every lane
-// keeps M x L accumulators in shared memory ([M L][threads], conflict-free),
-// and the lane partials are summed by a fixed butterfly at the end.  The
+// keeps M x L accumulators in shared memory ([M L][threads], conflict-free;
+// only the lane itself touches its slots), and the lane partials are summed
+// by a fixed butterfly at the end.  The
 // weight codes are read once; the activation rows stay in L1.
 #include "cfp_common.cuh"
 #include "kernels.cuh"
@@ -102,11 +103,18 @@ __global__ void __launch_bounds__(SKW * 32) gemm_skinny_kernel(const uint8_t* __
             // common case: every FP32 exponent field x + k0f is in [1, 254], so
             // the fields form in byte lanes; zero products get field 0 (+-0.0)
             const uint32_t f4 = (x4 + (uint32_t)k0f * R1) & prmt_sign4(nz);
+            // float bits of product c: byte 3 = sign | field >> 1 (from t4),
+            // bit 23 = field & 1 (bit 7 of byte c of u4), nothing below
+            const uint32_t t4 = ((f4 >> 1) & 0x7F7F7F7Fu) | s4;
+            const uint32_t u4 = (f4 << 7) & 0x80808080u;
+            const uint32_t hx4 = h4 << 2;  // phase x 4 per byte (<= 28)
+            char* accb = reinterpret_cast<char*>(acc);
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
-              // byte c of f4 to bits 23..30, its sign to bit 31
-              const uint32_t bits = (byte_to_top(f4, c) >> 1) | (byte_to_top(s4, c) & 0x80000000u);
-              atomicAdd(acc + (byte_to_top(h4, c) >> 16), __uint_as_float(bits));  // h NT, NT = 256
+              const uint32_t bits = __byte_perm(t4, u4, 0x0004u | (uint32_t)c << 12 | (uint32_t)(4 + c) << 8) & 0xFFFF0000u;
+              // byte offset of slot h NT (NT = 256 floats): (4 h) << 8
+              float* slot = reinterpret_cast<float*>(accb + __byte_perm(hx4, 0u, 0x4404u | (uint32_t)c << 4));
+              *slot += __uint_as_float(bits);
             }
           } else {
 #pragma unroll
@@ -114,7 +122,7 @@ __global__ void __launch_bounds__(SKW * 32) gemm_skinny_kernel(const uint8_t* __
               const int field = (int)((x4 >> (8 * c)) & 0x7Fu) + k0f;
               if (((nz >> (8 * c)) & 0x80u) && field > 0) {
                 const uint32_t bits = ((uint32_t)(field > 254 ? 254 : field) << 23) | (((s4 >> (8 * c)) & 0x80u) << 24);
-                atomicAdd(acc + ((h4 >> (8 * c)) & 0xFFu) * NT, __uint_as_float(bits));
+                acc[((h4 >> (8 * c)) & 0xFFu) * NT] += __uint_as_float(bits);
               }
             }
           }
