@@ -221,6 +221,9 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
     Xr = torch.randn((8192, 8192), device="cuda", generator=torch.Generator(device="cuda").manual_seed(3))
     Ar = torch.randn((1024, 4096), device="cuda", generator=torch.Generator(device="cuda").manual_seed(5))
     Br = torch.randn((1024, 4096), device="cuda", generator=torch.Generator(device="cuda").manual_seed(6)) * 0.02
+    Xl = torch.randn((2048, 4096), device="cuda", generator=torch.Generator(device="cuda").manual_seed(7))
+    Wl = torch.randn((4096, 4096), device="cuda", generator=torch.Generator(device="cuda").manual_seed(8)) * 0.02
+    Cl = torch.empty((2048, 4096), dtype=torch.float32, device="cuda")
     for fmt in ("E4C3", "E4C3_R8_9", "E4C3_R3_4"):
         cr = torch.empty(Xr.shape, dtype=torch.uint8, device="cuda")
         sr = torch.empty((8192, 8192 // 512), dtype=torch.int8, device="cuda")
@@ -229,13 +232,22 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
         (ar, sar), (br, sbr) = cfp.quantize(Ar, fmt, 512, 0, stream=stream), cfp.quantize(Br, fmt, 512, 0, stream=stream)
         ms_g = _time_ms(torch, stream, lambda: cfp.gemm(ar, sar, br, sbr, fmt, fmt, 512, "exact", stream=stream),
                         flush_l2, reps=3, warm=1)
+        tc_ms = None
+        if fmt in ("E4C3", "E4C3_R8_9"):  # the tensor-core kernel on the Llama-7B-like linear, G512
+            (al, sal), (bl, sbl) = cfp.quantize(Xl, fmt, 512, 0, stream=stream), cfp.quantize(Wl, fmt, 512, 0,
+                                                                                               stream=stream)
+            tc_ms = _time_ms(torch, stream, lambda: cfp.gemm(al, sal, bl, sbl, fmt, fmt, 512, "tensor",
+                                                             out=Cl, stream=stream), flush_l2)
+            del al, sal, bl, sbl
         res["radix"].append({"format": fmt, "phases": cfp.phase_count(fmt, fmt),
+                             "tensor_gemm_2048x4096x4096_G512_ms": None if tc_ms is None else round(tc_ms, 4),
+                             "tensor_gemm_tops": None if tc_ms is None else round(2 * 2048 * 4096 * 4096 / (tc_ms / 1e3) / 1e12, 3),
                              "quantize_fp32_8192x8192_G512_ms": round(ms_q, 4),
                              "quantize_gbs": round(Xr.numel() * (4 + 1 + 1 / 512) / (ms_q / 1e3) / 1e9, 1),
                              "exact_gemm_1024x1024x4096_ms": round(ms_g, 4),
                              "exact_gemm_gmac_per_s": round(1024 * 1024 * 4096 / (ms_g / 1e3) / 1e9, 1)})
         del cr, sr, ar, sar, br, sbr
-    del Xr, Ar, Br
+    del Xr, Ar, Br, Xl, Wl, Cl
     # training triplet, E4C3 weights/activations, E5C2 gradients
     X, Wt, dY = inputs.training_triplet_cuda()
     gemm_case("fwd X.W", q(X, "E4C3", 0), "E4C3", q(Wt, "E4C3", 1), "E4C3", 64)

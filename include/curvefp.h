@@ -55,9 +55,11 @@ extern "C" {
  * and L_nmin = 2^{-7} for r = 2^{8/9}) goes to zero; dequantization is
  * RN32(RN32(2^{j/(8q)}) 2^{a_b + floor(p n/(8q))}), j = p n mod 8q.  They are
  * accepted by curvefp_quantize, curvefp_quantize_static (and its variants),
- * curvefp_dequantize, curvefp_gemm_requant's destination and the EXACT GEMMs
- * (curvefp_gemm, curvefp_gemm_phases; both operands of the same format); the
- * tensor-core algorithms, curvefp_gemm_q32 and curvefp_gemm_oriented return
+ * curvefp_dequantize, curvefp_gemm_requant's destination, the EXACT GEMMs
+ * (curvefp_gemm, curvefp_gemm_phases, curvefp_gemm_phases_histogram; both
+ * operands of the same format) and, for r = 2^{8/9}, curvefp_gemm TENSOR
+ * (nine planes per operand, 81 plane pairs, three passes of three phases);
+ * the other algorithms, curvefp_gemm_q32 and curvefp_gemm_oriented return
  * CURVEFP_ERR_UNSUPPORTED for them. */
 typedef enum {
   CURVEFP_E3C3 = 0,
@@ -192,7 +194,8 @@ curvefp_status_t curvefp_dequantize(curvefp_format_t fmt, int block, const uint8
  * TENSOR, TENSOR_SPARSE: S_h accumulated in FP32 on the tensor cores, combine
  *   in FP32; plane values below 2^-14 of a row's largest block scale flush.
  *   Format pairs: E3C3 x E3C3, E4C3 x E4C3, E5C2 x E4C3, E4C3 x E5C2,
- *   E5C2 x E5C2 (others return CURVEFP_ERR_UNSUPPORTED).
+ *   E5C2 x E5C2, and (TENSOR) E4C3_R8_9 x E4C3_R8_9 (others return
+ *   CURVEFP_ERR_UNSUPPORTED).
  * SKINNY (M <= CURVEFP_SKINNY_MAX_M, else CURVEFP_ERR_UNSUPPORTED), AUTO:
  *   S_h accumulated in FP32 per output (products relative to the output's
  *   largest scale sum; products below the FP32 normal range relative to it

@@ -141,7 +141,8 @@ curvefp_status_t curvefp_gemm(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, 
   if (algo == CURVEFP_GEMM_EXACT)
     return from_cuda(cfp::launch_gemm_exact(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, nullptr, nullptr,
                                             device_status, st));
-  if (algo != CURVEFP_GEMM_EXACT && fmt_radix(fmt_a)) return CURVEFP_ERR_UNSUPPORTED;
+  // rational radix: EXACT, and TENSOR for r = 2^{8/9}
+  if (fmt_radix(fmt_a) && algo != CURVEFP_GEMM_TENSOR) return CURVEFP_ERR_UNSUPPORTED;
   // AUTO: the CUDA-core kernel where it is faster than a 128-row tensor-core
   // tile (measured up to M = 4 on the FFN decode shapes)
   if (algo == CURVEFP_GEMM_AUTO) algo = M <= CURVEFP_AUTO_SKINNY_M ? CURVEFP_GEMM_SKINNY : CURVEFP_GEMM_TENSOR;
@@ -251,7 +252,7 @@ curvefp_status_t curvefp_gemm_q32(curvefp_format_t fmt_a, curvefp_format_t fmt_b
   curvefp_status_t r = gemm_args(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K);
   if (r != CURVEFP_OK) return r;
   if (!acc) return CURVEFP_ERR_INVALID_ARG;
-  if (!cfp::gemm_tensor_supported(fmt_a, fmt_b)) return CURVEFP_ERR_UNSUPPORTED;  // same format pairs
+  if (fmt_radix(fmt_a) || !cfp::gemm_tensor_supported(fmt_a, fmt_b)) return CURVEFP_ERR_UNSUPPORTED;  // same format pairs
   if ((M + 15) / 16 > 65535) return CURVEFP_ERR_UNSUPPORTED;
   return from_cuda(cfp::launch_gemm_q32(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, acc, device_status,
                                         static_cast<cudaStream_t>(stream)));

@@ -7,7 +7,7 @@ namespace cfp {
 bool gemm_tensor_supported(int fa, int fb) {
   return (fa == CURVEFP_E3C3 && fb == CURVEFP_E3C3) || (fa == CURVEFP_E4C3 && fb == CURVEFP_E4C3) ||
          (fa == CURVEFP_E5C2 && fb == CURVEFP_E4C3) || (fa == CURVEFP_E4C3 && fb == CURVEFP_E5C2) ||
-         (fa == CURVEFP_E5C2 && fb == CURVEFP_E5C2);
+         (fa == CURVEFP_E5C2 && fb == CURVEFP_E5C2) || (fa == CURVEFP_E4C3_R8_9 && fb == CURVEFP_E4C3_R8_9);
 }
 
 cudaError_t launch_gemm_tensor(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
@@ -22,6 +22,7 @@ cudaError_t launch_gemm_tensor(int fa, int fb, int G, const uint8_t* a, const in
   CFP_T(CURVEFP_E5C2, CURVEFP_E4C3)
   CFP_T(CURVEFP_E4C3, CURVEFP_E5C2)
   CFP_T(CURVEFP_E5C2, CURVEFP_E5C2)
+  CFP_T(CURVEFP_E4C3_R8_9, CURVEFP_E4C3_R8_9)
 #undef CFP_T
   return cudaErrorInvalidValue;
 }

@@ -53,10 +53,23 @@ namespace cfp {
 
 namespace {
 
+// Planes per operand and the product lattice: binary radix on the shared
+// lattice L = max(K_a, K_b) (Eq. 2); E4C3 with r = 2^{8/9}: nine planes, nine
+// phases, unit weights (Eq. 4).
+template <int FA, int FB>
+struct TcLattice {
+  using P = Pair<FA, FB>;
+  static constexpr int KA = Fmt<FA>::K, KB = Fmt<FB>::K, L = P::L, WA = P::WA, WB = P::WB;
+};
+template <>
+struct TcLattice<CURVEFP_E4C3_R8_9, CURVEFP_E4C3_R8_9> {
+  static constexpr int KA = 9, KB = 9, L = 9, WA = 1, WB = 1;
+};
+
 template <int FA, int FB, int PT>
 struct TcCfg {
-  using P = Pair<FA, FB>;
-  static constexpr int KA = Fmt<FA>::K, KB = Fmt<FB>::K, L = P::L, WA = P::WA, WB = P::WB, LOG2L = P::LOG2L;
+  using T = TcLattice<FA, FB>;
+  static constexpr int KA = T::KA, KB = T::KB, L = T::L, WA = T::WA, WB = T::WB;
   static constexpr int FA_ = FA, FB_ = FB;
   static constexpr int BM = 128;
   static constexpr int KS = PT == PLANE_BF16 ? 16 : 32;  // K per MMA = K per pipeline step (32 bytes per row)
@@ -64,7 +77,7 @@ struct TcCfg {
   // columns leave 128 TMEM columns for A; N = 96 still runs the MMA at full
   // rate (the per-instruction floor is ~45 cycles, a 128x96x32 FP8 MMA is 48).
   static constexpr int BN = 96;
-  static constexpr int PP = 4;                            // phases per pass
+  static constexpr int PP = L == 9 ? 3 : 4;               // phases per pass
   static constexpr int NP = (L + PP - 1) / PP;            // passes
   static constexpr int ACC_COLS = PP * BN;
   // A planes of a step occupy AU_COLS TMEM columns (8 per plane); two steps
@@ -87,8 +100,8 @@ struct TcCfg {
   // D = F32, A = B = BF16 (kind::f16) or E5M2 (kind::f8f6f4): same bit pattern
   static constexpr uint32_t IDESC = tc::idesc_bf16_f32(BM, BN);
 
-  __host__ __device__ static constexpr int phase(int k1, int k2) { return (k1 * WA + k2 * WB) & (L - 1); }
-  __host__ __device__ static constexpr int carry(int k1, int k2) { return (k1 * WA + k2 * WB) >> LOG2L; }
+  __host__ __device__ static constexpr int phase(int k1, int k2) { return (k1 * WA + k2 * WB) % L; }
+  __host__ __device__ static constexpr int carry(int k1, int k2) { return (k1 * WA + k2 * WB) / L; }
   // Does pass p need B plane (k2, c)?
   __host__ __device__ static constexpr bool needed(int p, int c, int k2) {
     for (int k1 = 0; k1 < KA; ++k1)
@@ -132,8 +145,7 @@ struct TcCfg {
 // One 16-byte core-matrix row (chunk kc of the run) of every B plane the pass needs.
 template <class Cfg, int PT, int PASS>
 __device__ __forceinline__ void write_b_planes(uint8_t* stage, int row, int kc, const uint32_t (&v)[4],
-                                               const uint32_t (&vc)[4], const uint32_t (&mk)[4][3]) {
-  constexpr int KBITS = Fmt<Cfg::FB_>::C;
+                                               const uint32_t (&vc)[4], const uint32_t (&mk)[4][4]) {
   const uint32_t core = (uint32_t)((row >> 3) * 256 + kc * 128 + (row & 7) * 16);
 #pragma unroll
   for (int c = 0; c < 2; ++c) {
@@ -141,9 +153,9 @@ __device__ __forceinline__ void write_b_planes(uint8_t* stage, int row, int kc, 
 #pragma unroll
     for (int k2 = 0; k2 < Cfg::KB; ++k2) any = any || Cfg::slot(PASS, c, k2) >= 0;
     if (!any) continue;
-    uint32_t pw[4][8];
+    uint32_t pw[4][Cfg::KB > 8 ? Cfg::KB : 8];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) planes_of<KBITS>(c ? vc[q] : v[q], mk[q], pw[q]);
+    for (int q = 0; q < 4; ++q) PlaneFmt<Cfg::FB_>::planes(c ? vc[q] : v[q], mk[q], pw[q]);
 #pragma unroll
     for (int k2 = 0; k2 < Cfg::KB; ++k2) {
       const int sl = Cfg::slot(PASS, c, k2);
@@ -303,14 +315,14 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
       const int off = raw_scale - ref - bias;
       const int p = pass_of(g), s = g - p * nsub;
       if (is_a) {
-        uint32_t v[NWA], vc[NWA], mk[NWA][3];
+        uint32_t v[NWA], vc[NWA], mk[NWA][4];
         if constexpr (PES)
           decode_words_pes<FA, NWA>(cw, dw, bias, v, vc, mk, false);
         else
-          decode_words<FA, PT, NWA>(cw, off, v, vc, mk, false);
-        uint32_t pl[NWA][8];
+          PlaneFmt<FA>::template decode<PT, NWA>(cw, off, v, vc, mk, false);
+        uint32_t pl[NWA][Cfg::KA > 8 ? Cfg::KA : 8];
 #pragma unroll
-        for (int c = 0; c < NWA; ++c) planes_of<Fmt<FA>::C>(v[c], mk[c], pl[c]);
+        for (int c = 0; c < NWA; ++c) PlaneFmt<FA>::planes(v[c], mk[c], pl[c]);
         const int buf = g & 1;
         if (g >= 2) {
           // warp-uniform outcome: the TMEM stores below are warp-collective
@@ -394,11 +406,11 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
           sh.abort_flag = 1;
           return false;
         }
-        uint32_t v[4], vc[4], mk[4][3];
+        uint32_t v[4], vc[4], mk[4][4];
         if constexpr (PES)
           decode_words_pes<FB, 4>(cw, dw, bias, v, vc, mk, true);
         else
-          decode_words<FB, PT, 4>(cw, off, v, vc, mk, true);
+          PlaneFmt<FB>::template decode<PT, 4>(cw, off, v, vc, mk, true);
         uint8_t* stg = bstage + (size_t)st * Cfg::BSTAGE;
         if (p == 0) write_b_planes<Cfg, PT, 0>(stg, rloc, part, v, vc, mk);
         if (NP > 1 && p == 1) write_b_planes<Cfg, PT, (NP > 1 ? 1 : 0)>(stg, rloc, part, v, vc, mk);

@@ -173,7 +173,7 @@ __device__ __forceinline__ void write_b_op(uint8_t* stage, uint32_t core, int ha
 
 template <class Cfg, int PASS>
 __device__ __forceinline__ void write_b_ops(uint8_t* stage, int row, int half, const uint32_t (&v)[4],
-                                            const uint32_t (&vc)[4], const uint32_t (&mk)[4][3]) {
+                                            const uint32_t (&vc)[4], const uint32_t (&mk)[4][4]) {
   constexpr int KBITS = Fmt<Cfg::FB_>::C;
   uint32_t pw[2][4][8];
 #pragma unroll
@@ -348,7 +348,7 @@ __global__ void __launch_bounds__(TcsCfg<FA, FB>::THREADS, 1)
       const int p = pass_of(g), s = g - p * nsub;
       if (is_a) {
         constexpr int KBITS = Fmt<FA>::C;
-        uint32_t v[4], vc[4], mk[4][3];
+        uint32_t v[4], vc[4], mk[4][4];
         decode_words<FA, PLANE_E5M2, 4>(cw, off, v, vc, mk, false);
         const uint32_t wc[4] = {cw.x, cw.y, cw.z, cw.w};
         const uint32_t meta = sparse_meta<Cfg::MBIT>(wc);
@@ -448,7 +448,7 @@ __global__ void __launch_bounds__(TcsCfg<FA, FB>::THREADS, 1)
           sh.abort_flag = 1;
           return false;
         }
-        uint32_t v[4], vc[4], mk[4][3];
+        uint32_t v[4], vc[4], mk[4][4];
         decode_words<FB, PLANE_E5M2, 4>(cw, off, v, vc, mk, true);
         uint8_t* stg = bstage + (size_t)st * Cfg::BSTAGE;
         if (p == 0) write_b_ops<Cfg, 0>(stg, rloc, half, v, vc, mk);

@@ -117,7 +117,8 @@ __device__ __forceinline__ uint32_t bf16_word(uint32_t w2, int off) {
 // Masks of the curve-index bits (0xFF / 0xFFFF per lane where bit b of k is 1):
 // shift bit b of every lane's low byte to bit 7, then replicate it.
 template <int PT, int KBITS>
-__device__ __forceinline__ void k_masks(uint32_t w, uint32_t (&mk)[3]) {
+__device__ __forceinline__ void k_masks(uint32_t w, uint32_t (&mk)[4]) {
+  mk[3] = 0u;
 #pragma unroll
   for (int b = 0; b < 3; ++b) {
     if (b >= KBITS)
@@ -129,8 +130,9 @@ __device__ __forceinline__ void k_masks(uint32_t w, uint32_t (&mk)[3]) {
 
 // All 2^KBITS planes of a value word: the four products of v with the two
 // low-bit masks are shared, the third bit splits each of them in two.
-template <int KBITS>
-__device__ __forceinline__ void planes_of(uint32_t v, const uint32_t (&mk)[3], uint32_t (&out)[8]) {
+template <int KBITS, int NOUT>
+__device__ __forceinline__ void planes_of(uint32_t v, const uint32_t (&mk)[4], uint32_t (&out)[NOUT]) {
+  static_assert(NOUT >= 8, "eight plane slots");
   const uint32_t p0 = v & ~mk[0] & ~mk[1], p1 = v & mk[0] & ~mk[1];
   const uint32_t p2 = v & ~mk[0] & mk[1], p3 = v & mk[0] & mk[1];
   if (KBITS > 2) {
@@ -148,7 +150,7 @@ __device__ __forceinline__ void planes_of(uint32_t v, const uint32_t (&mk)[3], u
 // the curve-index masks of every word.
 template <int FMT, int PT, int NW>
 __device__ __forceinline__ void decode_words(const uint4& cw, int off, uint32_t (&v)[NW], uint32_t (&vc)[NW],
-                                             uint32_t (&mk)[NW][3], bool want_carry) {
+                                             uint32_t (&mk)[NW][4], bool want_carry) {
   constexpr int KBITS = Fmt<FMT>::C;
   const uint32_t w[4] = {cw.x, cw.y, cw.z, cw.w};
   if (PT == PLANE_E5M2) {
@@ -195,7 +197,7 @@ __device__ __forceinline__ uint32_t e5m2_word_pes(uint32_t w, uint32_t dp, uint3
 // of the sixteen codes of cw).
 template <int FMT, int NW>
 __device__ __forceinline__ void decode_words_pes(const uint4& cw, const uint4& dw, int bias, uint32_t (&v)[NW],
-                                                 uint32_t (&vc)[NW], uint32_t (&mk)[NW][3], bool want_carry) {
+                                                 uint32_t (&vc)[NW], uint32_t (&mk)[NW][4], bool want_carry) {
   constexpr int KBITS = Fmt<FMT>::C;
   const uint32_t w[4] = {cw.x, cw.y, cw.z, cw.w};
   const uint32_t d[4] = {dw.x, dw.y, dw.z, dw.w};
@@ -209,8 +211,77 @@ __device__ __forceinline__ void decode_words_pes(const uint4& cw, const uint4& d
   }
 }
 
+// ---------------------------------------------------------------------------
+// E4C3 codes with the rational radix r = 2^{8/9} (Sec. 3.1 Eq. 1, Eq. 4):
+// level 2^{n/9}, n = m - 64.  With v = m - 1 = 9 q + j (q in [0, 14],
+// j in [0, 8]) the element is 2^{q - 7} 2^{j/9}: it sits in plane j with the
+// power-of-two value 2^{a_b - ref + q - 7}, and plane j1 times plane j2 lands
+// on phase (j1 + j2) mod 9 with carry (j1 + j2) >= 9.  Nine planes per word:
+// q and j per byte from a 16-bit-lane multiply (floor(v/9) = (57 v) >> 9 for
+// v <= 127), the E5M2 exponent e5 = q + 8 + off kept where e5 >= 1 (as for
+// the binary planes: 2^14 below the row reference flushes), and the bits of
+// j as masks (mk[0..2] its low bits, mk[3] bit 3, which only j = 8 has).
+template <int NW>
+__device__ __forceinline__ void decode_words_r89(const uint4& cw, int off, uint32_t (&v)[NW], uint32_t (&vc)[NW],
+                                                 uint32_t (&mk)[NW][4], bool want_carry) {
+  const uint32_t w[4] = {cw.x, cw.y, cw.z, cw.w};
+  int cu = 8 + off - 1 + 128;  // u = q + cu = e5 + 127 per lane; off <= 0, so cu <= 135 and u <= 149
+  cu = cu < 0 ? 0 : cu;
+  const uint32_t cu4 = (uint32_t)cu * 0x01010101u;
+#pragma unroll
+  for (int i = 0; i < NW; ++i) {
+    const uint32_t m4 = w[i] & 0x7F7F7F7Fu;
+    const uint32_t nz = (m4 + 0x7F7F7F7Fu) & 0x80808080u;                    // m != 0
+    const uint32_t v4 = ((m4 | 0x80808080u) - 0x01010101u) & 0x7F7F7F7Fu;    // m - 1 (no borrow)
+    const uint32_t ql = (((v4 & 0x00FF00FFu) * 57u) >> 9) & 0x001F001Fu;
+    const uint32_t qh = ((((v4 >> 8) & 0x00FF00FFu) * 57u) >> 9) & 0x001F001Fu;
+    const uint32_t q4 = ql | (qh << 8);
+    const uint32_t j4 = v4 - q4 * 9u;                                        // per lane in [0, 8]
+    const uint32_t u = q4 + cu4;
+    const uint32_t keep = prmt_sign(u & nz, 0xBA98u);
+    const uint32_t e5 = ((u & 0x7F7F7F7Fu) + 0x01010101u) & keep;           // q + 8 + off where kept
+    v[i] = (w[i] & 0x80808080u & keep) | (e5 << 2);
+    vc[i] = want_carry ? v[i] + (keep & 0x04040404u) : 0u;                  // exponent + 1
+#pragma unroll
+    for (int b = 0; b < 4; ++b) mk[i][b] = prmt_sign(j4 << (7 - b), 0xBA98u);
+  }
+}
+
+// Plane split of a format: PlaneFmt<FMT>::KP planes of a value word.
+template <int FMT>
+struct PlaneFmt {
+  static constexpr int KP = Fmt<FMT>::K;
+  template <int PT, int NW>
+  __device__ __forceinline__ static void decode(const uint4& cw, int off, uint32_t (&v)[NW], uint32_t (&vc)[NW],
+                                                uint32_t (&mk)[NW][4], bool want_carry) {
+    decode_words<FMT, PT, NW>(cw, off, v, vc, mk, want_carry);
+  }
+  template <int NOUT>
+  __device__ __forceinline__ static void planes(uint32_t v, const uint32_t (&mk)[4], uint32_t (&out)[NOUT]) {
+    planes_of<Fmt<FMT>::C>(v, mk, out);
+  }
+};
+template <>
+struct PlaneFmt<CURVEFP_E4C3_R8_9> {
+  static constexpr int KP = 9;
+  template <int PT, int NW>
+  __device__ __forceinline__ static void decode(const uint4& cw, int off, uint32_t (&v)[NW], uint32_t (&vc)[NW],
+                                                uint32_t (&mk)[NW][4], bool want_carry) {
+    static_assert(PT == PLANE_E5M2, "E5M2 planes");
+    decode_words_r89<NW>(cw, off, v, vc, mk, want_carry);
+  }
+  template <int NOUT>
+  __device__ __forceinline__ static void planes(uint32_t v, const uint32_t (&mk)[4], uint32_t (&out)[NOUT]) {
+    static_assert(NOUT >= 9, "nine plane slots");
+    planes_of<3>(v & ~mk[3], mk, out);
+    out[8] = v & mk[3];
+  }
+};
+
+static __constant__ uint32_t CFP_PHASE_F32_L9_TC[9] = CFP_PHASE_F32_L9_INIT;
+
 __device__ __forceinline__ float phase_const(int L, int h) {
-  return __uint_as_float(L == 8 ? CFP_PHASE_F32_L8_DEV[h] : CFP_PHASE_F32_L4_DEV[h]);
+  return __uint_as_float(L == 8 ? CFP_PHASE_F32_L8_DEV[h] : (L == 9 ? CFP_PHASE_F32_L9_TC[h] : CFP_PHASE_F32_L4_DEV[h]));
 }
 
 

@@ -137,7 +137,8 @@ def test_rational_radix_host_rules(lib):
     assert lib.curvefp_quantize(5, 32, d, 0, 4, 64, 64, 0, d, d, None, None) == INVALID
     # GEMM: mixed radix, and the tensor-core algorithms
     assert lib.curvefp_gemm(0, 3, 1, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED
-    assert lib.curvefp_gemm(1, 3, 3, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED
+    assert lib.curvefp_gemm(1, 4, 4, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED  # r = 2^{3/4}
+    assert lib.curvefp_gemm(3, 3, 3, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED  # skinny
     assert lib.curvefp_gemm(2, 4, 4, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED
     assert lib.curvefp_gemm_q32(3, 3, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED
     assert lib.curvefp_quantize_static(3, 32, 1, 0, d, 0, 4, 64, d, d, None, 0, None, None) == INVALID  # no workspace

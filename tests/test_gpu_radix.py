@@ -195,3 +195,51 @@ def test_llama_linear_g512_sampled(torch, fmt):
     ref = oracle.gemm(rx, rsx, rw, rsw, fmt, fmt, G)
     assert status_bits(st) == 0
     assert np.array_equal(ps.cpu().numpy(), ref["S_raw"]) and np.array_equal(pl.cpu().numpy(), ref["lsb"])
+
+
+@pytest.mark.parametrize("block", [32, 512])
+def test_tensor_gemm_r89_within_tolerance(torch, block):
+    """Tensor-core GEMM for r = 2^{8/9} (nine planes per operand, 81 plane
+    pairs, nine phases in three passes): within 1e-5 of the oracle's fp64
+    combine, normalised by the row norms; M, N ragged against the tiles."""
+    import paper_2608_10010_gb300 as cfp
+    from tests.gpu_util import normalised_error
+
+    fmt = "E4C3_R8_9"
+    M, N, K = 200, 320, 1024
+    a, sa, _ = oracle.quantize(inputs.outlier_channels((M, K), 17), fmt, block, 0)
+    b, sb, _ = oracle.quantize(inputs.normal((N, K), 18, 0.02), fmt, block, 0)
+    st = new_status(torch)
+    c = cfp.gemm(to_dev(torch, a), to_dev(torch, sa), to_dev(torch, b), to_dev(torch, sb), fmt, fmt, block, "tensor",
+                 status=st)
+    torch.cuda.synchronize()
+    ref = oracle.gemm(a, sa, b, sb, fmt, fmt, block, phases=False)
+    assert status_bits(st) == 0
+    err = normalised_error(c.cpu().numpy(), ref["C"], oracle.row_norms(a, sa, fmt, block),
+                           oracle.row_norms(b, sb, fmt, block))
+    assert err <= 1e-5, err
+
+
+def test_tensor_gemm_r89_llama_g512_sampled(torch):
+    """The radix-frontier setting at full size (Llama-7B-like linear, G512)
+    on the tensor cores: 64 x 64 sampled outputs against the oracle."""
+    import paper_2608_10010_gb300 as cfp
+    from tests.gpu_util import normalised_error
+
+    fmt, G = "E4C3_R8_9", 512
+    X, W = inputs.llama7b_linear(2048, 4096, 4096)
+    qx, sx = cfp.quantize(to_dev(torch, X), fmt, G, 0)
+    qw, sw = cfp.quantize(to_dev(torch, W), fmt, G, 0)
+    st = new_status(torch)
+    c = cfp.gemm(qx, sx, qw, sw, fmt, fmt, G, "tensor", status=st)
+    torch.cuda.synchronize()
+    assert status_bits(st) == 0
+    rng = np.random.default_rng(19)
+    ii = np.sort(rng.choice(2048, 64, replace=False))
+    jj = np.sort(rng.choice(4096, 64, replace=False))
+    ah, sah = qx.cpu().numpy()[ii], sx.cpu().numpy()[ii]
+    bh, sbh = qw.cpu().numpy()[jj], sw.cpu().numpy()[jj]
+    ref = oracle.gemm(ah, sah, bh, sbh, fmt, fmt, G, phases=False)
+    err = normalised_error(c.cpu().numpy()[np.ix_(ii, jj)], ref["C"], oracle.row_norms(ah, sah, fmt, G),
+                           oracle.row_norms(bh, sbh, fmt, G))
+    assert err <= 1e-5, err
