@@ -621,7 +621,8 @@ def run_reference(args):
 def run_only(args):
     """One kernel of the path, a few launches, no timing: the target of the
     ncu captures (--only gemm: the tensor-core GEMM of the workload above;
-    --only quantize: 2^28 BF16 elements, E4C3, block 32)."""
+    --only quantize: 2^28 BF16 elements, E4C3, block 32; skinny, reuse, r89:
+    the decode GEMM, the reused-operand dgrad and the r = 2^{8/9} GEMM)."""
     import torch
 
     import paper_2608_10010_gb300 as cfp
@@ -637,12 +638,37 @@ def run_only(args):
             c = cfp.gemm(a, sa, b, sb, FMT, FMT, G, "tensor")
         torch.cuda.synchronize()
         print(json.dumps({"only": "gemm", "launches": args.steps, "c00": float(c[0, 0])}))
-    else:
+    elif args.only == "quantize":
         x = inputs.bandwidth_tensor_cuda(1 << 28, 4096, 3)
         for _ in range(args.steps):
             codes, _ = cfp.quantize(x, "E4C3", G, 0)
         torch.cuda.synchronize()
         print(json.dumps({"only": "quantize", "launches": args.steps, "code00": int(codes[0, 0])}))
+    elif args.only == "skinny":  # decode GEMM: FFN M = 1, E3C3, W[14336 x 4096]
+        Xf, Wf = inputs.ffn_cuda(1, 4096)
+        a, sa = cfp.quantize(Xf, "E3C3", G, 0)
+        b, sb = cfp.quantize(Wf, "E3C3", G, 1)
+        for _ in range(args.steps):
+            c = cfp.gemm(a, sa, b, sb, "E3C3", "E3C3", G, "skinny")
+        torch.cuda.synchronize()
+        print(json.dumps({"only": "skinny", "launches": args.steps, "c00": float(c[0, 0])}))
+    elif args.only == "reuse":  # dgrad on the reused weight, triplet shape (T 4096, 4096 -> 11008)
+        X, Wt, dY = inputs.training_triplet_cuda()
+        qw, sw = cfp.quantize(Wt, "E4C3", G, 1)
+        qg, sg = cfp.quantize(dY, "E5C2", G, 0)
+        del X, Wt, dY
+        for _ in range(args.steps):
+            c = cfp.gemm_oriented(qg, sg, "rows", qw, sw, "cols", "E5C2", "E4C3", G, "tensor")
+        torch.cuda.synchronize()
+        print(json.dumps({"only": "reuse", "launches": args.steps, "c00": float(c[0, 0])}))
+    else:  # r89: the tensor-core GEMM for r = 2^{8/9}, Llama-7B-like linear, G512
+        X, W = inputs.llama7b_linear(M, K, N)
+        a, sa = cfp.quantize(torch.from_numpy(X).to(dev), "E4C3_R8_9", 512, 0)
+        b, sb = cfp.quantize(torch.from_numpy(W).to(dev), "E4C3_R8_9", 512, 0)
+        for _ in range(args.steps):
+            c = cfp.gemm(a, sa, b, sb, "E4C3_R8_9", "E4C3_R8_9", 512, "tensor")
+        torch.cuda.synchronize()
+        print(json.dumps({"only": "r89", "launches": args.steps, "c00": float(c[0, 0])}))
 
 
 def main():
@@ -652,7 +678,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--only", choices=["gemm", "quantize"], default=None)
+    ap.add_argument("--only", choices=["gemm", "quantize", "skinny", "reuse", "r89"], default=None)
     ap.add_argument("--no-sweep", action="store_true", help="skip the other workloads (quantize sweep, GEMM shapes)")
     args = ap.parse_args()
     if args.only:
