@@ -421,18 +421,40 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
       }
       return true;
     };
-    // Two register sets of codes, each loaded two steps before it is used and
-    // never copied, so that no register move waits on an in-flight load.
-    uint4 q0, q1, d0, d1;
-    int r0, r1;
-    load(0, q0, r0, d0);
-    load(1, q1, r1, d1);
-    for (int g = 0; g < total; g += 2) {
-      if (!step(g, q0, r0, d0)) break;
-      load(g + 2, q0, r0, d0);
-      if (g + 1 >= total) break;
-      if (!step(g + 1, q1, r1, d1)) break;
-      load(g + 3, q1, r1, d1);
+    // PF register sets of codes, each loaded PF steps before it is used and
+    // never copied, so that no register move waits on an in-flight load.  Two
+    // sets where the operands stay in L2 (the codes of one step arrive in
+    // less than two steps); four for the per-element-scale operands, whose
+    // large-K training shapes miss L2 and wait on DRAM.
+    if constexpr (PES) {
+      constexpr int PF = 4;
+      uint4 q[PF], dq[PF];
+      int rq[PF];
+#pragma unroll
+      for (int u = 0; u < PF; ++u) load(u, q[u], rq[u], dq[u]);
+      bool run = true;
+      for (int g = 0; g < total && run; g += PF) {
+#pragma unroll
+        for (int u = 0; u < PF; ++u) {
+          if (g + u >= total || !step(g + u, q[u], rq[u], dq[u])) {
+            run = false;
+            break;
+          }
+          load(g + u + PF, q[u], rq[u], dq[u]);
+        }
+      }
+    } else {
+      uint4 q0, q1, d0, d1;
+      int r0, r1;
+      load(0, q0, r0, d0);
+      load(1, q1, r1, d1);
+      for (int g = 0; g < total; g += 2) {
+        if (!step(g, q0, r0, d0)) break;
+        load(g + 2, q0, r0, d0);
+        if (g + 1 >= total) break;
+        if (!step(g + 1, q1, r1, d1)) break;
+        load(g + 3, q1, r1, d1);
+      }
     }
   } else {
     // ------------------------------ MMA issuer -------------------------------
