@@ -424,9 +424,10 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
     // PF register sets of codes, each loaded PF steps before it is used and
     // never copied, so that no register move waits on an in-flight load.  Two
     // sets where the operands stay in L2 (the codes of one step arrive in
-    // less than two steps); four for the per-element-scale operands, whose
-    // large-K training shapes miss L2 and wait on DRAM.
-    if constexpr (PES) {
+    // less than two steps); four for the per-element-scale operands and for
+    // A with four planes (the mixed pairs of the training GEMMs), whose
+    // large-K shapes miss L2 and whose short steps leave the loads exposed.
+    if constexpr (PES || Cfg::KA == 4) {
       constexpr int PF = 4;
       uint4 q[PF], dq[PF];
       int rq[PF];
