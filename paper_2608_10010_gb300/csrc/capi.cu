@@ -74,6 +74,11 @@ curvefp_status_t curvefp_quantize_static(curvefp_format_t fmt, int block, curvef
   if (need && (!workspace || workspace_bytes < need || (reinterpret_cast<uintptr_t>(workspace) & 15) != 0))
     return CURVEFP_ERR_INVALID_ARG;
   if (rows * cols > (int64_t)1 << 40) return CURVEFP_ERR_UNSUPPORTED;
+  // block groups with the ceil-absmax rule are the quantizer itself (R11):
+  // the streaming kernels where their alignment rules hold
+  if (group == CURVEFP_SCALE_BLOCK && rule == CURVEFP_SCALE_CEIL_ABSMAX && al16(x) && al16(codes) &&
+      (cols * esz) % 16 == 0)
+    return curvefp_quantize(fmt, block, x, dtype, rows, cols, cols, 0, codes, scales, device_status, stream);
   if (fmt_radix(fmt))
     return from_cuda(cfp::launch_quantize_static_radix(fmt, block, group, rule, x, dtype, rows, cols, codes, scales,
                                                        workspace, device_status, static_cast<cudaStream_t>(stream),

@@ -110,3 +110,15 @@ def test_mse_special_groups(fmt):
     codes, scales, nan = oracle.quantize_static(x, fmt, 32, "block", "mse")
     assert nan and scales[0, 0] == 0 and not codes[0].any()
     assert scales[1, 0] == 127 and codes[2, 5] == 0
+
+
+@pytest.mark.parametrize("fmt", ["E3C3", "E4C3", "E5C2", "E4C3_R8_9"])
+def test_block_ceil_is_the_quantizer(oracle, fmt):
+    """R11: a block scale group with the ceil-absmax rule is Q(X) itself (the
+    C ABI routes it to the streaming quantizer)."""
+    from paper_2608_10010_gb300 import inputs
+
+    x = inputs.elementwise_outliers((24, 256), 31)
+    c0, s0, n0 = oracle.quantize(x, fmt, 32, 0)
+    c1, s1, n1 = oracle.quantize_static(x, fmt, 32, "block", "ceil")
+    assert np.array_equal(c0, c1) and np.array_equal(s0, s1) and n0 == n1
