@@ -225,7 +225,7 @@ curvefp_status_t curvefp_gemm_oriented(curvefp_gemm_algo_t algo, curvefp_format_
   if (!workspace || workspace_bytes < need || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
     return CURVEFP_ERR_INVALID_ARG;
   return from_cuda(cfp::launch_gemm_tensor_reuse(fmt_a, fmt_b, block, a, sa, layout_a, b, sb, layout_b, M, N, K, c,
-                                                 workspace, device_status, st));
+                                                 workspace, device_status, st, sm_count()));
 }
 
 curvefp_status_t curvefp_gemm_phases_histogram(curvefp_format_t fmt_a, curvefp_format_t fmt_b, int block,

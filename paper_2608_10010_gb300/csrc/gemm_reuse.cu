@@ -176,7 +176,7 @@ size_t gemm_reuse_workspace(int la, int lb, int64_t M, int64_t N, int64_t K) {
 
 cudaError_t launch_gemm_tensor_reuse(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, int la,
                                      const uint8_t* b, const int8_t* sb, int lb, int64_t M, int64_t N, int64_t K,
-                                     float* c, void* ws, uint32_t* status, cudaStream_t s) {
+                                     float* c, void* ws, uint32_t* status, cudaStream_t s, int sms) {
   uint8_t* w = static_cast<uint8_t*>(ws);
   Prepared pa, pb;
   cudaError_t e = prepare(la, a, sa, M, K, G, w, s, pa);
@@ -186,7 +186,7 @@ cudaError_t launch_gemm_tensor_reuse(int fa, int fb, int G, const uint8_t* a, co
   const PesOperands pes{pa.dp, pb.dp, pa.ref, pb.ref, pa.rsh, pb.rsh};
   constexpr int PT = PLANE_E5M2;
 #define CFP_R(X, Y) \
-  if (fa == X && fb == Y) return launch_tc_t<X, Y, PT, true>(G, pa.codes, nullptr, pb.codes, nullptr, M, N, K, c, status, s, pes);
+  if (fa == X && fb == Y) return launch_tc_t<X, Y, PT, true>(G, pa.codes, nullptr, pb.codes, nullptr, M, N, K, c, status, s, pes, sms);
   CFP_R(CURVEFP_E3C3, CURVEFP_E3C3)
   CFP_R(CURVEFP_E4C3, CURVEFP_E4C3)
   CFP_R(CURVEFP_E5C2, CURVEFP_E4C3)

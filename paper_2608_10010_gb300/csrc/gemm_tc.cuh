@@ -139,7 +139,10 @@ struct TcCfg {
   }
   static constexpr int MAXS = maxslots();
   static constexpr int BSTAGE = MAXS * PLANE_BYTES;
-  static constexpr size_t SMEM = (size_t)NSB * BSTAGE + 2048;
+  // B stages, the barrier block, and the FP32 stash of a K-piece's earlier
+  // passes (tail tiles split in K, see TailPlan)
+  static constexpr size_t STASH = (size_t)BM * BN * 4;
+  static constexpr size_t SMEM = (size_t)NSB * BSTAGE + 2048 + STASH;
 };
 
 // One 16-byte core-matrix row (chunk kc of the run) of every B plane the pass needs.
@@ -197,6 +200,20 @@ __device__ __forceinline__ void issue_step(uint32_t leader, int p, uint32_t tmem
 
 }  // namespace
 
+// The last partial wave (tiles % SMs CTAs on an otherwise idle GPU) is
+// spread out: its tiles are split in K into a larger and a smaller piece
+// (steps [0, split_step) and [split_step, nsub) of every pass), launched
+// after the whole tiles, so the pieces of two waves' worth of work share the
+// SMs.  A piece keeps its earlier passes in shared memory and adds its total
+// to C with one atomic add per output; C of those tiles is zeroed first, so
+// every output receives exactly two additions onto 0 and the sum does not
+// depend on their order (IEEE addition is commutative).
+struct TailPlan {
+  int ntiles_full;  // CTAs that own a whole tile (tiles 0 .. ntiles_full - 1)
+  int nsplit;       // tiles split in K (tiles ntiles_full .. + nsplit - 1)
+  int split_step;   // first step of the second piece
+};
+
 // Per-element scales of both operands (PES = true; reused operands of the
 // training GEMMs): dp[r][k] = max(a(r,k) - ref, -64) + 64 beside the codes,
 // and the row reference ref = max_k a(r,k) read as refs[r >> rsh].
@@ -218,7 +235,7 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
                                                          const uint8_t* __restrict__ B, const int8_t* __restrict__ sB,
                                                          int M, int N, int K, int G, int gshift,
                                                          float* __restrict__ C, uint32_t* status,
-                                                         const PesOperands pes) {
+                                                         const PesOperands pes, const TailPlan plan) {
   using Cfg = TcCfg<FA, FB, PT>;
   constexpr int L = Cfg::L, PP = Cfg::PP, NP = Cfg::NP, BN = Cfg::BN, NSB = Cfg::NSB;
   constexpr int NAW = Cfg::NAW, NWA = Cfg::NWA, ATPR = Cfg::ATPR;
@@ -230,8 +247,23 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
   TcShared& sh = *reinterpret_cast<TcShared*>(smem + (size_t)NSB * Cfg::BSTAGE);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int m0 = blockIdx.y * Cfg::BM, n0 = blockIdx.x * BN;
-  const int nb = K / G, nsub = K / Cfg::KS, total = NP * nsub;
+  // this CTA's job: a whole tile, or one K piece of a tail tile
+  const int ntn = (N + BN - 1) / BN;
+  int tile = blockIdx.x, s0 = 0, s1 = K / Cfg::KS;
+  const bool split = tile >= plan.ntiles_full;
+  if (split) {
+    const int q = tile - plan.ntiles_full;
+    if (q < plan.nsplit) {
+      tile = plan.ntiles_full + q;
+      s1 = plan.split_step;
+    } else {
+      tile = plan.ntiles_full + q - plan.nsplit;
+      s0 = plan.split_step;
+    }
+  }
+  const int m0 = (tile / ntn) * Cfg::BM, n0 = (tile % ntn) * BN;
+  const int nb = K / G, nsub = s1 - s0, total = NP * nsub;  // nsub: this job's steps per pass
+  float* stash = reinterpret_cast<float*>(smem + (size_t)NSB * Cfg::BSTAGE + 2048);
 
   if (tid == 0) {
     for (int s = 0; s < NSB; ++s) {
@@ -291,7 +323,7 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
       dw = make_uint4(0, 0, 0, 0);
       off = 0;
       if (rowok && g < total) {
-        const int s = g - pass_of(g) * nsub;
+        const int s = s0 + g - pass_of(g) * nsub;  // step of the whole K
         const uint8_t* p = src + (int64_t)s * Cfg::KS;
         const int nbytes = (is_a ? NWA : 4) * CB;  // 16, 8 or 4
         if (nbytes == 16) {
@@ -378,7 +410,19 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
               }
               float* dst = C + (int64_t)r * N + n0 + c0;
               const bool full8 = n0 + c0 + 8 <= N && ((reinterpret_cast<uintptr_t>(dst) & 15) == 0);
-              if (full8) {
+              if (split) {
+                // K piece: earlier passes wait in the stash, the last one adds
+                // the piece's total to C (zeroed, two pieces per output)
+                float* st8 = stash + rloc * BN + c0;
+                if (p < NP - 1) {
+#pragma unroll
+                  for (int c = 0; c < 8; ++c) st8[c] = p == 0 ? y[c] : st8[c] + y[c];
+                } else {
+#pragma unroll
+                  for (int c = 0; c < 8; ++c)
+                    if (n0 + c0 + c < N) atomicAdd(dst + c, p == 0 ? y[c] : st8[c] + y[c]);
+                }
+              } else if (full8) {
                 float4* d4 = reinterpret_cast<float4*>(dst);
                 float4 a0 = make_float4(y[0], y[1], y[2], y[3]), a1 = make_float4(y[4], y[5], y[6], y[7]);
                 if (p > 0) {
@@ -495,10 +539,28 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
   }
 }
 
+// Which tiles to split: with T tiles on P SMs, the T mod P tiles of the last
+// partial wave.  Up to P/2 of them split in halves (all pieces run at once:
+// the tail costs half a tile instead of a whole one); up to 2P/3 in a 2/3
+// and a 1/3 piece (the big pieces and P - T_s small ones start together, the
+// other small ones follow on the SMs the first small ones free: 2/3 of a
+// tile).  Otherwise the wave is full enough to be left alone.
+inline TailPlan tail_plan(int64_t tiles, int sms, int nsub) {
+  TailPlan t{(int)tiles, 0, 0};
+  const int64_t rem = sms > 0 ? tiles % sms : 0;
+  if (tiles < sms || rem == 0) return t;
+  if (2 * rem <= sms && nsub >= 2) {
+    t = TailPlan{(int)(tiles - rem), (int)rem, nsub / 2};
+  } else if (3 * rem <= 2 * (int64_t)sms && nsub >= 3) {
+    t = TailPlan{(int)(tiles - rem), (int)rem, (2 * nsub) / 3};
+  }
+  return t;
+}
+
 template <int FA, int FB, int PT, bool PES>
 static cudaError_t launch_tc_t(int G, const uint8_t* a, const int8_t* sa, const uint8_t* b, const int8_t* sb,
                                int64_t M, int64_t N, int64_t K, float* c, uint32_t* st, cudaStream_t s,
-                               const PesOperands& pes) {
+                               const PesOperands& pes, int sms) {
   using Cfg = TcCfg<FA, FB, PT>;
   static_assert(sizeof(TcShared) <= 2048, "shared tail");
   static_assert(Cfg::SMEM <= 227 * 1024, "shared memory");
@@ -506,10 +568,18 @@ static cudaError_t launch_tc_t(int G, const uint8_t* a, const int8_t* sa, const 
   auto kern = gemm_tc_kernel<FA, FB, PT, PES>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg::SMEM);
   if (e != cudaSuccess) return e;
-  dim3 grid((unsigned)((N + Cfg::BN - 1) / Cfg::BN), (unsigned)((M + Cfg::BM - 1) / Cfg::BM));
+  const int64_t ntn = (N + Cfg::BN - 1) / Cfg::BN, ntm = (M + Cfg::BM - 1) / Cfg::BM;
+  const TailPlan plan = tail_plan(ntn * ntm, sms, (int)(K / Cfg::KS));
+  if (plan.nsplit > 0) {
+    // C of the split tiles starts at zero: whole tile rows from the first one
+    const int64_t row0 = (plan.ntiles_full / ntn) * Cfg::BM;
+    e = cudaMemsetAsync(c + row0 * N, 0, (size_t)((M - row0) * N) * sizeof(float), s);
+    if (e != cudaSuccess) return e;
+  }
+  const unsigned grid = (unsigned)(plan.ntiles_full + 2 * plan.nsplit);
   int gshift = 0;  // scale block of step s is s >> gshift (G / KS is a power of two)
   while ((Cfg::KS << gshift) < G) ++gshift;
-  kern<<<grid, Cfg::THREADS, Cfg::SMEM, s>>>(a, sa, b, sb, (int)M, (int)N, (int)K, G, gshift, c, st, pes);
+  kern<<<grid, Cfg::THREADS, Cfg::SMEM, s>>>(a, sa, b, sb, (int)M, (int)N, (int)K, G, gshift, c, st, pes, plan);
   return cudaGetLastError();
 }
 

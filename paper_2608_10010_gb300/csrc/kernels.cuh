@@ -45,7 +45,7 @@ cudaError_t launch_gemm_exact_oriented(int fa, int fb, int G, const uint8_t* a, 
 size_t gemm_reuse_workspace(int la, int lb, int64_t M, int64_t N, int64_t K);
 cudaError_t launch_gemm_tensor_reuse(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, int la,
                                      const uint8_t* b, const int8_t* sb, int lb, int64_t M, int64_t N, int64_t K,
-                                     float* c, void* ws, uint32_t* status, cudaStream_t st);
+                                     float* c, void* ws, uint32_t* status, cudaStream_t st, int sms);
 cudaError_t launch_gemm_q32(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
                             const int8_t* sb, int64_t M, int64_t N, int64_t K, int64_t* out, uint32_t* status,
                             cudaStream_t s);

@@ -200,6 +200,32 @@ def test_tensor_matches_exact_kernel(torch):
     assert normalised_error(ct, ce.astype(np.float64), na, nb) <= TOL
 
 
+@pytest.mark.parametrize("M,N,K", [(1024, 4096, 256), (2048, 4096, 96), (2048, 4096, 32)])
+def test_tensor_tail_pieces_every_output(torch, M, N, K):
+    """Tile counts whose last wave is split in K (1024 x 4096: 344 tiles, 40
+    split in halves; 2048 x 4096: 688 tiles, 80 split 2/3 + 1/3; K = 32 is
+    one step, too short to split): every output of the tensor path against
+    the exact kernel, and two runs bit-identical (the pieces' atomic
+    additions onto zero do not depend on their order)."""
+    import paper_2608_10010_gb300 as cfp
+
+    x = inputs.outlier_channels((M, K), 23)
+    w = inputs.normal((N, K), 24, 0.02)
+    a, sa = quantized(x, "E3C3")
+    b, sb = quantized(w, "E3C3")
+    args = [to_dev(torch, v) for v in (a, sa, b, sb)]
+    st = new_status(torch)
+    ce = cfp.gemm(*args, "E3C3", "E3C3", 32, "exact", status=st)
+    ct = cfp.gemm(*args, "E3C3", "E3C3", 32, "tensor", status=st)
+    ct2 = cfp.gemm(*args, "E3C3", "E3C3", 32, "tensor", status=st)
+    torch.cuda.synchronize()
+    assert status_bits(st) == 0
+    assert torch.equal(ct.view(torch.int32), ct2.view(torch.int32))
+    na = oracle.row_norms(a, sa, "E3C3")
+    nb = oracle.row_norms(b, sb, "E3C3")
+    assert normalised_error(ct.cpu().numpy(), ce.cpu().numpy().astype(np.float64), na, nb) <= TOL
+
+
 # ---- full-size workloads, sampled rows ---------------------------------------------
 
 SAMPLE_ROWS = 16
