@@ -36,6 +36,12 @@
 // sits on the path between two MMAs, so the stages are whole steps.  Every
 // wait is bounded.
 #pragma once
+#include <functional>
+#include <mutex>
+#include <queue>
+#include <unordered_map>
+#include <vector>
+
 #include "cfp_common.cuh"
 #include "kernels.cuh"
 #include "tc_planes.cuh"
@@ -539,21 +545,68 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
   }
 }
 
-// Which tiles to split: with T tiles on P SMs, the T mod P tiles of the last
-// partial wave.  Up to P/2 of them split in halves (all pieces run at once:
-// the tail costs half a tile instead of a whole one); up to 2P/3 in a 2/3
-// and a 1/3 piece (the big pieces and P - T_s small ones start together, the
-// other small ones follow on the SMs the first small ones free: 2/3 of a
-// tile).  Otherwise the wave is full enough to be left alone.
-inline TailPlan tail_plan(int64_t tiles, int sms, int nsub) {
-  TailPlan t{(int)tiles, 0, 0};
-  const int64_t rem = sms > 0 ? tiles % sms : 0;
-  if (tiles < sms || rem == 0) return t;
-  if (2 * rem <= sms && nsub >= 2) {
-    t = TailPlan{(int)(tiles - rem), (int)rem, nsub / 2};
-  } else if (3 * rem <= 2 * (int64_t)sms && nsub >= 3) {
-    t = TailPlan{(int)(tiles - rem), (int)rem, (2 * nsub) / 3};
+// Which tiles to split, and where.  The launch order (whole tiles, then the
+// first pieces, then the second pieces) is dispatched greedily to the SMs as
+// they free; the plan is the one whose simulated makespan is smallest over
+// the last s = T mod P (+ P, + 2P) tiles split at 1/2, 2/3 or 3/4 of K (a
+// piece costs its share of a tile's steps plus a small fixed overhead, so a
+// split must gain more than that).  At the headline shape (688 tiles, 152
+// SMs) this is the 80 tail tiles at 2/3: 4.67 instead of 5 waves.
+inline double tail_makespan(int64_t tiles, int sms, int64_t s, double x) {
+  const double ovh = 0.02;  // per-piece overhead, in tiles
+  // after the whole tiles, (tiles - s) mod P SMs carry one tile more
+  const int64_t w = tiles - s, base = w / sms, extra = w % sms;
+  std::priority_queue<double, std::vector<double>, std::greater<double>> q;
+  for (int i = 0; i < sms; ++i) q.push((double)(base + (i < extra ? 1 : 0)));
+  auto run = [&](int64_t n, double d) {
+    for (int64_t i = 0; i < n; ++i) {
+      const double t = q.top();
+      q.pop();
+      q.push(t + d);
+    }
+  };
+  run(s, x + ovh);
+  run(s, 1.0 - x + ovh);
+  double m = 0.0;
+  while (!q.empty()) {
+    m = q.top() > m ? q.top() : m;
+    q.pop();
   }
+  return m;
+}
+
+inline TailPlan tail_plan_search(int64_t tiles, int sms, int nsub) {
+  TailPlan best{(int)tiles, 0, 0};
+  if (sms <= 0 || tiles < sms || nsub < 2 || tiles % sms == 0) return best;
+  double best_m = tail_makespan(tiles, sms, 0, 0.5);
+  const double xs[3] = {0.5, 2.0 / 3.0, 0.75};
+  for (int64_t s = tiles % sms; s <= tiles && s <= tiles % sms + 2 * (int64_t)sms; s += sms)
+    for (double x : xs) {
+      const int split = (int)(x * nsub + 0.5);
+      if (split < 1 || split >= nsub) continue;
+      const double m = tail_makespan(tiles, sms, s, (double)split / nsub);
+      if (m < best_m - 1e-9) {
+        best_m = m;
+        best = TailPlan{(int)(tiles - s), (int)s, split};
+      }
+    }
+  return best;
+}
+
+// The plan of a shape is searched once per process (a few hundred
+// microseconds of host time) and remembered.
+inline TailPlan tail_plan(int64_t tiles, int sms, int nsub) {
+  static std::mutex mu;
+  static std::unordered_map<uint64_t, TailPlan> memo;
+  const uint64_t key = ((uint64_t)tiles << 32) ^ ((uint64_t)sms << 16) ^ (uint64_t)nsub;
+  {
+    std::lock_guard<std::mutex> lk(mu);
+    auto it = memo.find(key);
+    if (it != memo.end()) return it->second;
+  }
+  const TailPlan t = tail_plan_search(tiles, sms, nsub);
+  std::lock_guard<std::mutex> lk(mu);
+  memo[key] = t;
   return t;
 }
 

@@ -200,13 +200,14 @@ def test_tensor_matches_exact_kernel(torch):
     assert normalised_error(ct, ce.astype(np.float64), na, nb) <= TOL
 
 
-@pytest.mark.parametrize("M,N,K", [(1024, 4096, 256), (2048, 4096, 96), (2048, 4096, 32)])
+@pytest.mark.parametrize("M,N,K", [(1024, 4096, 256), (2048, 4096, 96), (2048, 4096, 32), (1280, 9120, 128)])
 def test_tensor_tail_pieces_every_output(torch, M, N, K):
-    """Tile counts whose last wave is split in K (1024 x 4096: 344 tiles, 40
-    split in halves; 2048 x 4096: 688 tiles, 80 split 2/3 + 1/3; K = 32 is
-    one step, too short to split): every output of the tensor path against
-    the exact kernel, and two runs bit-identical (the pieces' atomic
-    additions onto zero do not depend on their order)."""
+    """Tile counts whose tail is split in K (1024 x 4096: 344 tiles, 192 of
+    them split; 2048 x 4096: 688 tiles, 80 split 2/3 + 1/3; 1280 x 9120:
+    950 tiles, split 3/4 + 1/4; K = 32 is one step, too short to split):
+    every output of the tensor path against the exact kernel, and two runs
+    bit-identical (the pieces' atomic additions onto zero do not depend on
+    their order)."""
     import paper_2608_10010_gb300 as cfp
 
     x = inputs.outlier_channels((M, K), 23)
