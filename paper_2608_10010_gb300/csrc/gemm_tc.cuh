@@ -145,9 +145,10 @@ struct TcCfg {
   }
   static constexpr int MAXS = maxslots();
   static constexpr int BSTAGE = MAXS * PLANE_BYTES;
-  // B stages, the barrier block, and the FP32 stash of a K-piece's earlier
-  // passes (tail tiles split in K, see TailPlan)
-  static constexpr size_t STASH = (size_t)BM * BN * 4;
+  // B stages, the barrier block, and the FP32 stash of the passes' partial
+  // outputs (row stride SST floats)
+  static constexpr int SST = BN + 4;
+  static constexpr size_t STASH = (size_t)BM * SST * 4;
   static constexpr size_t SMEM = (size_t)NSB * BSTAGE + 2048 + STASH;
 };
 
@@ -348,6 +349,72 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
       }
     };
     const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+    // The epilogue of pass pe (A producers, after the pass's last MMA): each
+    // 8-column chunk of this thread's share is read from TMEM, combined over
+    // the pass's phases and added to the running total in the FP32 stash (row
+    // stride BN + 4 floats: the 16-byte accesses of a warp's 32 rows hit
+    // distinct banks).  The last pass writes the total to C once: stored for
+    // a whole tile, added atomically to zeroed C for a K piece (two pieces
+    // per output).  The total is ((y_0 + y_1) + y_2) in FP32 in every case.
+    auto epilogue = [&](const int pe) -> bool {
+      const bool ok = __all_sync(0xffffffffu, tc::mbar_wait(&sh.acc_full, pe & 1));
+      if (!ok) {
+        raise_flag(status, CURVEFP_DEV_TIMEOUT);
+        sh.abort_flag = 1;
+      }
+      tc::fence_after_sync();
+      float* strow = stash + rloc * Cfg::SST;
+#pragma unroll 1
+      for (int c0 = part * (BN / ATPR); c0 < (part + 1) * (BN / ATPR); c0 += 8) {
+        uint32_t acc[PP][8];
+#pragma unroll
+        for (int q = 0; q < PP; ++q)
+          if (pe * PP + q < L) tc::tmem_ld8(lane_base + q * BN + c0, acc[q]);
+        tc::tmem_wait_ld();
+        if (rowok && ok) {
+          float y[8];
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            float t = 0.f;
+#pragma unroll
+            for (int q = 0; q < PP; ++q)
+              if (pe * PP + q < L) t = fmaf(phase_const(L, pe * PP + q), __uint_as_float(acc[q][c]), t);
+            y[c] = scalbnf(t, ref + Cfg::PBA + sh.refB[c0 + c] + Cfg::PBB);
+          }
+          float4* s4 = reinterpret_cast<float4*>(strow + c0);
+          if (pe > 0) {
+            const float4 b0 = s4[0], b1 = s4[1];
+            y[0] = b0.x + y[0]; y[1] = b0.y + y[1]; y[2] = b0.z + y[2]; y[3] = b0.w + y[3];
+            y[4] = b1.x + y[4]; y[5] = b1.y + y[5]; y[6] = b1.z + y[6]; y[7] = b1.w + y[7];
+          }
+          s4[0] = make_float4(y[0], y[1], y[2], y[3]);
+          s4[1] = make_float4(y[4], y[5], y[6], y[7]);
+        }
+      }
+      if (pe == NP - 1 && rowok && ok) {
+#pragma unroll 1
+        for (int c0 = part * (BN / ATPR); c0 < (part + 1) * (BN / ATPR); c0 += 8) {
+          const float4* s4 = reinterpret_cast<const float4*>(strow + c0);
+          const float4 a0 = s4[0], a1 = s4[1];
+          float* dst = C + (int64_t)r * N + n0 + c0;
+          if (split) {
+            const float y[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+#pragma unroll
+            for (int c = 0; c < 8; ++c)
+              if (n0 + c0 + c < N) atomicAdd(dst + c, y[c]);
+          } else if (n0 + c0 + 8 <= N && ((reinterpret_cast<uintptr_t>(dst) & 15) == 0)) {
+            reinterpret_cast<float4*>(dst)[0] = a0;
+            reinterpret_cast<float4*>(dst)[1] = a1;
+          } else {
+            const float y[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+#pragma unroll
+            for (int c = 0; c < 8; ++c)
+              if (n0 + c0 + c < N) dst[c] = y[c];
+          }
+        }
+      }
+      return ok;
+    };
     // One pipeline step of this producer thread; false ends the loop (abort).
     auto step = [&](const int g, const uint4 cw, const int raw_scale, const uint4 dw) -> bool {
       const int off = raw_scale - ref - bias;
@@ -389,64 +456,12 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(&sh.full[g % NSB]);
 
-        if (s == nsub - 1) {
-          // ---------------- epilogue of pass p -----------------------------
-          const bool ok = __all_sync(0xffffffffu, tc::mbar_wait(&sh.acc_full, p & 1));
-          if (!ok) {
-            raise_flag(status, CURVEFP_DEV_TIMEOUT);
-            sh.abort_flag = 1;
-          }
-          tc::fence_after_sync();
+        // the pass's epilogue after its last step (a one-trip loop: this form
+        // measured faster than a plain call in the unrolled step pairs)
+        const int pe_last = s == nsub - 1 ? p : -1;
 #pragma unroll 1
-          for (int c0 = part * (BN / ATPR); c0 < (part + 1) * (BN / ATPR); c0 += 8) {
-            uint32_t acc[PP][8];
-#pragma unroll
-            for (int q = 0; q < PP; ++q)
-              if (p * PP + q < L) tc::tmem_ld8(lane_base + q * BN + c0, acc[q]);
-            tc::tmem_wait_ld();
-            if (rowok && ok) {
-              float y[8];
-#pragma unroll
-              for (int c = 0; c < 8; ++c) {
-                float t = 0.f;
-#pragma unroll
-                for (int q = 0; q < PP; ++q)
-                  if (p * PP + q < L) t = fmaf(phase_const(L, p * PP + q), __uint_as_float(acc[q][c]), t);
-                y[c] = scalbnf(t, ref + Cfg::PBA + sh.refB[c0 + c] + Cfg::PBB);
-              }
-              float* dst = C + (int64_t)r * N + n0 + c0;
-              const bool full8 = n0 + c0 + 8 <= N && ((reinterpret_cast<uintptr_t>(dst) & 15) == 0);
-              if (split) {
-                // K piece: earlier passes wait in the stash, the last one adds
-                // the piece's total to C (zeroed, two pieces per output)
-                float* st8 = stash + rloc * BN + c0;
-                if (p < NP - 1) {
-#pragma unroll
-                  for (int c = 0; c < 8; ++c) st8[c] = p == 0 ? y[c] : st8[c] + y[c];
-                } else {
-#pragma unroll
-                  for (int c = 0; c < 8; ++c)
-                    if (n0 + c0 + c < N) atomicAdd(dst + c, p == 0 ? y[c] : st8[c] + y[c]);
-                }
-              } else if (full8) {
-                float4* d4 = reinterpret_cast<float4*>(dst);
-                float4 a0 = make_float4(y[0], y[1], y[2], y[3]), a1 = make_float4(y[4], y[5], y[6], y[7]);
-                if (p > 0) {
-                  const float4 b0 = d4[0], b1 = d4[1];
-                  a0.x += b0.x; a0.y += b0.y; a0.z += b0.z; a0.w += b0.w;
-                  a1.x += b1.x; a1.y += b1.y; a1.z += b1.z; a1.w += b1.w;
-                }
-                d4[0] = a0;
-                d4[1] = a1;
-              } else {
-#pragma unroll
-                for (int c = 0; c < 8; ++c)
-                  if (n0 + c0 + c < N) dst[c] = p == 0 ? y[c] : dst[c] + y[c];
-              }
-            }
-          }
-          if (!ok) return false;
-        }
+        for (int pe = p; pe <= pe_last; ++pe)
+          if (!epilogue(pe)) return false;
       } else {
         const int st = g % NSB;
         bool fail = false;
