@@ -28,6 +28,7 @@ import os
 import statistics
 import subprocess
 import sys
+import tempfile
 import threading
 import time
 
@@ -703,6 +704,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--only", choices=["gemm", "quantize", "skinny", "reuse", "r89"], default=None)
     ap.add_argument("--no-sweep", action="store_true", help="skip the other workloads (quantize sweep, GEMM shapes)")
+    ap.add_argument("--out", default=None, help="also write the JSON line to this file (atomically: temp + rename)")
     args = ap.parse_args()
     if args.only:
         run_only(args)
@@ -711,7 +713,28 @@ def main():
         args.warmup = 3
     out = run_reference(args) if args.impl == "reference" else run_ours(args)
     if out is not None:
-        print(json.dumps(out), flush=True)
+        line = json.dumps(out)
+        print(line, flush=True)
+        if args.out:
+            write_atomic(args.out, line + "\n")
+
+
+def write_atomic(path: str, text: str) -> None:
+    """Write a result file so that a reader sees the old file or the whole
+    new one, never a partial write: a temporary file in the same directory,
+    flushed to disk, then renamed over the target."""
+    d = os.path.dirname(os.path.abspath(path))
+    fd, tmp = tempfile.mkstemp(prefix=".bench-", suffix=".tmp", dir=d)
+    try:
+        with os.fdopen(fd, "w") as f:
+            f.write(text)
+            f.flush()
+            os.fsync(f.fileno())
+        os.replace(tmp, path)
+    except BaseException:
+        if os.path.exists(tmp):
+            os.unlink(tmp)
+        raise
 
 
 if __name__ == "__main__":

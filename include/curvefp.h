@@ -306,6 +306,21 @@ curvefp_status_t curvefp_gemm_q32(curvefp_format_t fmt_a, curvefp_format_t fmt_b
  * lattice L = max(K_a, K_b)); -1 for an unknown format. */
 int curvefp_phase_count(curvefp_format_t fmt_a, curvefp_format_t fmt_b);
 
+/* Failure-detection self-test (an interface of this library, not from the
+ * paper; no CurveFP arithmetic).  One warp waits on a fresh mbarrier of count
+ * 1 with the bounded wait that every pipeline hand-off of the TENSOR GEMM
+ * uses, limited here to limit_cycles SM clock cycles (1 .. 2^31; the GEMM's
+ * own limit is 2^31, about a second).  arrive != 0: lane 0 completes the
+ * barrier's phase first, the wait succeeds and *device_status is unchanged.
+ * arrive == 0: nothing completes it; the wait gives up after the limit, ORs
+ * CURVEFP_DEV_TIMEOUT into *device_status and the kernel returns normally
+ * (no trap), so the context stays usable.
+ *   device_status : device uint32_t, required.
+ * Errors: CURVEFP_ERR_INVALID_ARG for a NULL status or a limit out of range
+ * (nothing enqueued). */
+curvefp_status_t curvefp_selftest_bounded_wait(int arrive, int64_t limit_cycles, uint32_t* device_status,
+                                               void* stream);
+
 /* Static description of a status code. */
 const char* curvefp_status_string(curvefp_status_t status);
 

@@ -55,12 +55,14 @@ def load(build_if_missing: bool = False):
         lib.curvefp_gemm_oriented_workspace_bytes.restype = ctypes.c_size_t
         lib.curvefp_gemm_oriented.argtypes = [I, I, I, I, P, P, I, P, P, I, L, L, L, P, P, P, P, ctypes.c_size_t,
                                               P, P]
+        lib.curvefp_selftest_bounded_wait.argtypes = [I, L, P, P]
         lib.curvefp_status_string.argtypes = [I]
         lib.curvefp_status_string.restype = ctypes.c_char_p
         lib.curvefp_version.restype = ctypes.c_char_p
         for f in ("curvefp_quantize", "curvefp_quantize_static", "curvefp_quantize_static_noalloc",
                   "curvefp_dequantize", "curvefp_gemm", "curvefp_gemm_phases", "curvefp_gemm_q32",
-                  "curvefp_gemm_requant", "curvefp_gemm_oriented", "curvefp_gemm_phases_histogram"):
+                  "curvefp_gemm_requant", "curvefp_gemm_oriented", "curvefp_gemm_phases_histogram",
+                  "curvefp_selftest_bounded_wait"):
             getattr(lib, f).restype = I
         _lib = lib
     return _lib
@@ -278,3 +280,11 @@ def gemm_phases(a, sa, b, sb, fmt_a, fmt_b, block: int = 32, status=None, stream
     _check(load().curvefp_gemm_phases(_fmt(fmt_a), _fmt(fmt_b), block, _p(a), _p(sa), _p(b), _p(sb), M, N, K,
                                       _p(c), _p(ps), _p(pl), _p(status), _stream(stream)))
     return c, ps, pl
+
+
+def selftest_bounded_wait(arrive: bool, limit_cycles: int, status, stream=None):
+    """Failure-detection self-test of the tensor-core pipeline's bounded wait
+    (curvefp_selftest_bounded_wait): with arrive=False the wait gives up after
+    limit_cycles SM cycles and ORs the TIMEOUT bit into `status` (a CUDA
+    int32/uint32 tensor of one element)."""
+    _check(load().curvefp_selftest_bounded_wait(1 if arrive else 0, int(limit_cycles), _p(status), _stream(stream)))

@@ -273,6 +273,13 @@ int curvefp_phase_count(curvefp_format_t fmt_a, curvefp_format_t fmt_b) {
   return ka > kb ? ka : kb;
 }
 
+curvefp_status_t curvefp_selftest_bounded_wait(int arrive, int64_t limit_cycles, uint32_t* device_status,
+                                               void* stream) {
+  if (!device_status || limit_cycles < 1 || limit_cycles > (int64_t(1) << 31)) return CURVEFP_ERR_INVALID_ARG;
+  return from_cuda(cfp::launch_selftest_wait(arrive != 0, (long long)limit_cycles, device_status,
+                                             static_cast<cudaStream_t>(stream)));
+}
+
 const char* curvefp_status_string(curvefp_status_t s) {
   switch (s) {
     case CURVEFP_OK: return "ok";

@@ -26,4 +26,27 @@ cudaError_t launch_gemm_tensor(int fa, int fb, int G, const uint8_t* a, const in
   return cudaErrorInvalidValue;
 }
 
+namespace {
+
+// Failure-detection self-test of the pipeline's bounded wait (no CurveFP
+// arithmetic): one warp waits on a fresh barrier of count 1, which lane 0
+// completes first only when `arrive` is set.  A wait that gives up raises
+// TIMEOUT and the kernel returns as the GEMM's roles do.
+__global__ void __launch_bounds__(32) selftest_wait_kernel(int arrive, long long limit, uint32_t* status) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x == 0) tc::mbar_init(&bar, 1);
+  __syncthreads();
+  if (arrive && threadIdx.x == 0) tc::mbar_arrive(&bar);
+  __syncwarp();
+  const bool ok = __all_sync(0xffffffffu, tc::mbar_wait(&bar, 0, limit));
+  if (!ok && threadIdx.x == 0) raise_flag(status, CURVEFP_DEV_TIMEOUT);
+}
+
+}  // namespace
+
+cudaError_t launch_selftest_wait(int arrive, long long limit, uint32_t* status, cudaStream_t s) {
+  selftest_wait_kernel<<<1, 32, 0, s>>>(arrive, limit, status);
+  return cudaGetLastError();
+}
+
 }  // namespace cfp

@@ -17,6 +17,7 @@ cudaError_t launch_dequantize(int fmt, int G, const uint8_t* codes, const int8_t
 cudaError_t launch_gemm_exact(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
                               const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, int64_t* phase_sums,
                               int32_t* phase_lsb, uint32_t* status, cudaStream_t st);
+cudaError_t launch_selftest_wait(int arrive, long long limit, uint32_t* status, cudaStream_t s);
 cudaError_t launch_gemm_tensor(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
                                const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, uint32_t* status,
                                cudaStream_t st, int sms);

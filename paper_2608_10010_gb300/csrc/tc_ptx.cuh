@@ -50,13 +50,14 @@ __device__ __forceinline__ bool mbar_try_wait_hint(uint64_t* bar, uint32_t parit
   return ok != 0;
 }
 // Bounded wait: the thread parks in hardware (try_wait with a 0.1 ms suspend
-// hint, woken when the phase completes) and gives up after 2^31 SM cycles
-// (about a second), returning false, so that no pipeline fault can hang the GPU.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+// hint, woken when the phase completes) and gives up after `limit` SM cycles
+// (2^31 by default, about a second), returning false, so that no pipeline
+// fault can hang the GPU.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, long long limit = 1ll << 31) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   while (!mbar_try_wait_hint(bar, parity, 100000u))
-    if (clock64() - t0 > (1ll << 31)) return false;
+    if (clock64() - t0 > limit) return false;
   return true;
 }
 

@@ -85,6 +85,11 @@ def test_host_side_validation(lib):
     assert qs(1, 32, 1, 1, dummy, 0, 4, 64, dummy, dummy, None, 0, None, None) == INVALID
     assert qs(1, 32, 1, 1, dummy, 0, 4, 64, dummy, dummy, dummy, 8, None, None) == INVALID
     assert qs(1, 32, 2, 1, None, 0, 0, 64, None, None, None, 0, None, None) == 0
+    # bounded-wait self-test: the status word is required, the limit in 1 .. 2^31
+    sw = lib.curvefp_selftest_bounded_wait
+    assert sw(0, 1000, None, None) == INVALID
+    assert sw(0, 0, dummy, None) == INVALID
+    assert sw(0, (1 << 31) + 1, dummy, None) == INVALID
 
 
 def test_oriented_gemm_validation(lib):
