@@ -135,7 +135,9 @@ def rank_table(E: int, C: int) -> tuple[int, list[int]]:
     Entry = rank below the bucket's threshold | rank at/above it << 8 |
     threshold's low 16 mantissa bits << 16 (0 and equal ranks if none).
     Ranks follow the nearest-level rule: 0 below L_nmin/2, saturating at
-    2^{E+C} - 1; at most one decision threshold falls in a bucket."""
+    2^{E+C} - 1; at most one decision threshold falls in a bucket, and where
+    one does the rank steps by exactly 1 at a threshold whose low 16 bits are
+    nonzero (the FP32 kernels rely on both: rank = r_lo + [bits >= t16])."""
     K = 1 << C
     B = 1 << (E + C - 1)
     nmax = B - 1
@@ -165,6 +167,8 @@ def rank_table(E: int, C: int) -> tuple[int, list[int]]:
             t16 = (cuts[0] & 0xFFFF) if cuts else 0
             if not cuts:
                 assert r_lo == r_hi
+            else:
+                assert r_hi == r_lo + 1 and t16 >= 1
             out.append(r_lo | (r_hi << 8) | (t16 << 16))
     return nbin, out
 
@@ -276,6 +280,8 @@ def radix_rank_table(r: dict) -> tuple[int, list[int]]:
             assert len(cuts) <= 1
             if not cuts:
                 assert r_lo == r_hi
+            else:
+                assert r_hi == r_lo + 1 and (cuts[0] & 0xFFFF) >= 1
             out.append(r_lo | (r_hi << 8) | (((cuts[0] & 0xFFFF) if cuts else 0) << 16))
     return nbin, out
 

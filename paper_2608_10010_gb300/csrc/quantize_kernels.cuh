@@ -192,6 +192,17 @@ struct RankTab<CURVEFP_E4C3_R3_4> {
   __device__ static const uint32_t* src() { return CFP_RANK_E4C3_R3_4_DEV; }
 };
 
+// FP32 compare form of a rank-table entry r_lo | r_hi << 8 | t16 << 16 (a
+// bucket with a decision threshold has r_hi = r_lo + 1 and t16 >= 1, checked
+// by the table's generator): (t16 - 1) << 16 | r_lo with a threshold,
+// 0xFFFF0000 | r_lo without.  For a value with FP32 bits w, (w << 16) > entry
+// holds iff its low 16 mantissa bits are >= t16 (never without a threshold),
+// so its rank is r_lo + that comparison.
+__device__ __forceinline__ uint32_t rank_cmp_entry(uint32_t e) {
+  const uint32_t lo = e & 0xFFu;
+  return ((e >> 8) & 0xFFu) != lo ? (((e >> 16) - 1u) << 16) | lo : 0xFFFF0000u | lo;
+}
+
 // Table key of a magnitude bit pattern (FP32 bits >> 16, or BF16 bits) for
 // block scale a: (binade - F_z) * 128 + top 7 mantissa bits, clamped at 0
 // (everything below binade F_z encodes as zero).  kb = (127 + a + F_z) << 7.
@@ -211,6 +222,21 @@ __device__ __forceinline__ uint32_t max_u16x2(uint32_t a, uint32_t b) {
   uint32_t d;
   asm("max.u16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
   return d;
+}
+
+// Ranks of four FP32 values (bits w[0..3]) from the compare-form table: the
+// table keys of two values at a time in 16-bit lanes (kb2 = the block's key
+// base in both lanes), then r = r_lo + [(w << 16) > entry].
+__device__ __forceinline__ uint32_t ranks4_f32(const uint32_t* tab, const uint32_t (&w)[4], uint32_t kb2) {
+  uint32_t r[4];
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const uint32_t k2 = max_u16x2(__byte_perm(w[2 * h], w[2 * h + 1], 0x7632) & 0x7FFF7FFFu, kb2) - kb2;
+    const uint32_t e0 = tab[k2 & 0xFFFFu], e1 = tab[k2 >> 16];
+    r[2 * h] = (e0 & 0xFFu) + ((w[2 * h] << 16) > e0 ? 1u : 0u);
+    r[2 * h + 1] = (e1 & 0xFFu) + ((w[2 * h + 1] << 16) > e1 ? 1u : 0u);
+  }
+  return __byte_perm(__byte_perm(r[0], r[1], 0x0040), __byte_perm(r[2], r[3], 0x0040), 0x5410);
 }
 
 // ---------------------------------------------------------------------------
@@ -248,7 +274,7 @@ __global__ void __launch_bounds__(256) quantize_rows_kernel(const T* __restrict_
     if (BF16)
       tab8[i] = (uint8_t)(e & 0xFFu);
     else
-      tab[i] = e;
+      tab[i] = rank_cmp_entry(e);
   }
   __syncthreads();
 
@@ -335,14 +361,7 @@ __global__ void __launch_bounds__(256) quantize_rows_kernel(const T* __restrict_
             }
             *reinterpret_cast<uint2*>(d) = make_uint2(out[0], out[1]);
           } else {
-            uint32_t r[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              const uint32_t ab = w[i] & 0x7FFFFFFFu;
-              const uint32_t e = tab[max(ab >> 16, (uint32_t)kb) - (uint32_t)kb];
-              r[i] = ((ab & 0xFFFFu) >= (e >> 16)) ? ((e >> 8) & 0xFFu) : (e & 0xFFu);
-            }
-            const uint32_t r4 = r[0] | (r[1] << 8) | (r[2] << 16) | (r[3] << 24);
+            const uint32_t r4 = ranks4_f32(tab, w, (uint32_t)kb * 0x00010001u);
             const uint32_t s4 = __byte_perm(__byte_perm(w[0], w[1], 0x0073), __byte_perm(w[2], w[3], 0x7300), 0x7610);
             *reinterpret_cast<uint32_t*>(d) = merge_signs(r4, s4);
           }
@@ -414,14 +433,6 @@ __global__ void __launch_bounds__((QB_NCW + 1) * 32, CFP_QB_CTAS) quantize_rows_
   uint64_t* empty = full + NST;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int i = threadIdx.x; i < 256; i += blockDim.x) lut[i] = __ldg(lut_src<F::K>() + i);
-  for (int i = threadIdx.x; i < NTAB; i += blockDim.x) {
-    const uint32_t e = __ldg(RankTab<FMT>::src() + i);
-    if (BF16)
-      tab8[i] = (uint8_t)(e & 0xFFu);
-    else
-      tab[i] = e;
-  }
   if (threadIdx.x == 0) {
     for (int i = 0; i < NST; ++i) {
       tc::mbar_init(&full[i], 1);
@@ -430,6 +441,20 @@ __global__ void __launch_bounds__((QB_NCW + 1) * 32, CFP_QB_CTAS) quantize_rows_
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();
+  // the first copies are issued while the consumers load the tables; the
+  // consumers then meet on named barrier 1 (the producer warp does not take
+  // part), so the table loads' latency hides behind the first chunks'
+  if (warp < QB_NCW) {
+    for (int i = threadIdx.x; i < 256; i += QB_NCW * 32) lut[i] = __ldg(lut_src<F::K>() + i);
+    for (int i = threadIdx.x; i < NTAB; i += QB_NCW * 32) {
+      const uint32_t e = __ldg(RankTab<FMT>::src() + i);
+      if (BF16)
+        tab8[i] = (uint8_t)(e & 0xFFu);
+      else
+        tab[i] = rank_cmp_entry(e);
+    }
+    asm volatile("bar.sync 1, %0;" ::"n"(QB_NCW * 32) : "memory");
+  }
 
   const int64_t nchunks = (nblk + CH_BLK - 1) / CH_BLK;
   if (warp == QB_NCW) {
@@ -532,14 +557,7 @@ __global__ void __launch_bounds__((QB_NCW + 1) * 32, CFP_QB_CTAS) quantize_rows_
           }
           *reinterpret_cast<uint2*>(d) = make_uint2(out[0], out[1]);
         } else {
-          uint32_t r[4];
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const uint32_t ab = w[i] & 0x7FFFFFFFu;
-            const uint32_t e = tab[max(ab >> 16, (uint32_t)kb) - (uint32_t)kb];
-            r[i] = ((ab & 0xFFFFu) >= (e >> 16)) ? ((e >> 8) & 0xFFu) : (e & 0xFFu);
-          }
-          const uint32_t r4 = r[0] | (r[1] << 8) | (r[2] << 16) | (r[3] << 24);
+          const uint32_t r4 = ranks4_f32(tab, w, (uint32_t)kb * 0x00010001u);
           const uint32_t s4 = __byte_perm(__byte_perm(w[0], w[1], 0x0073), __byte_perm(w[2], w[3], 0x7300), 0x7610);
           *reinterpret_cast<uint32_t*>(d) = merge_signs(r4, s4);
         }
