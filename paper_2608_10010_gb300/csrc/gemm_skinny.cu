@@ -56,6 +56,7 @@ __global__ void __launch_bounds__(SKW * 32) gemm_skinny_kernel(const uint8_t* __
   extern __shared__ float sk_acc[];                                 // [M L][NT]
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nb = K / G;
+  const int gs = __ffs(G) - 1;  // G is a power of two
 
   for (int j = blockIdx.x * SKW + warp; j < N; j += gridDim.x * SKW) {
     // ref_i = max_b (a_i,b + b_j,b)
@@ -74,7 +75,7 @@ __global__ void __launch_bounds__(SKW * 32) gemm_skinny_kernel(const uint8_t* __
     for (int k0 = lane * 16; k0 < K; k0 += 512) {
       const uint4 wv = wnext;  // the next step's codes are in flight while these are used
       if (k0 + 512 < K) wnext = __ldg(reinterpret_cast<const uint4*>(brow + k0 + 512));
-      const int blk = k0 / G;  // G >= 32: the 16 codes share a block
+      const int blk = k0 >> gs;  // G >= 32: the 16 codes share a block
       const int sb = (int)sB[(int64_t)j * nb + blk];
       const uint32_t w[4] = {wv.x, wv.y, wv.z, wv.w};
       uint32_t kb4[4], eb4[4], nzb[4];

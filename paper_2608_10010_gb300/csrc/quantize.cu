@@ -41,7 +41,7 @@ cudaError_t launch_quantize_static(int fmt, int G, int group, int rule, const vo
 
 cudaError_t launch_dequantize(int fmt, int G, const uint8_t* codes, const int8_t* scales, int64_t n, float* out,
                               cudaStream_t st, int sms) {
-  int64_t grid = (n / 16 + 255) / 256;
+  int64_t grid = (n / 4 + 1023) / 1024;  // 256 threads x 4 words of 4 codes
   const int64_t cap = (int64_t)sms * 8;
   if (grid > cap) grid = cap;
   if (grid < 1) grid = 1;

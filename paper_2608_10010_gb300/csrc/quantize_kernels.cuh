@@ -659,39 +659,55 @@ __global__ void __launch_bounds__(256) dequantize_kernel(const uint8_t* __restri
     tab[m] = v;
   }
   __syncthreads();
-  const int64_t nchunks = n / 16;
-  for (int64_t ch = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; ch < nchunks;
-       ch += (int64_t)gridDim.x * blockDim.x) {
-    uint4 cv = __ldcs(reinterpret_cast<const uint4*>(codes) + ch);
-    const int a = scales[(ch * 16) / G];
-    const bool fast = (a + EMIN >= -126) && (a + F::EMAX <= 126);
-    uint32_t cw[4] = {cv.x, cv.y, cv.z, cv.w};
-    uint32_t o[16];
+  // A thread takes words of 4 codes, U at a time (all loads issued first); the
+  // warp's loads cover 128 contiguous bytes and its stores 512 contiguous
+  // bytes per instruction.  n is a multiple of the block size (>= 32).
+  constexpr int U = 4;
+  const int64_t nw = n >> 2;
+  const int64_t tile = (int64_t)blockDim.x * U;
+  const int gs = __ffs(G) - 1;  // G is a power of two: block of code i = i >> gs
+  const uint32_t* codes32 = reinterpret_cast<const uint32_t*>(codes);
+  uint4* out4 = reinterpret_cast<uint4*>(out);
+  for (int64_t t0 = (int64_t)blockIdx.x * tile; t0 < nw; t0 += (int64_t)gridDim.x * tile) {
+    uint32_t cw[U];
+    int sc[U];
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      uint32_t code = (cw[i >> 2] >> (8 * (i & 3))) & 0xFFu;
-      uint32_t m = code & F::MMASK;
-      uint32_t r;
-      if (fast) {
-        r = m ? tab[m] + (uint32_t)(a * (1 << 23)) : 0u;
-      } else if (m == 0u) {
-        r = 0u;
-      } else {
-        int nn = (int)m - F::B;
-        int e = nn >> F::C, k = nn & (F::K - 1);
-        float ck = __uint_as_float(F::K == 8 ? CFP_CK_F32_K8_DEV[k] : CFP_CK_F32_K4_DEV[k]);
-        int E = a + e;
-        int E1 = E < -126 ? -126 : (E > 127 ? 127 : E);
-        int E2 = E - E1;  // in [-18, 15]
-        float y = __fmul_rn(ck, __uint_as_float((uint32_t)(E1 + 127) << 23));
-        y = __fmul_rn(y, __uint_as_float((uint32_t)(E2 + 127) << 23));
-        r = __float_as_uint(y);
-      }
-      o[i] = m ? (r | ((code & 0x80u) << 24)) : 0u;
+    for (int u = 0; u < U; ++u) {
+      const int64_t w = t0 + u * (int64_t)blockDim.x + threadIdx.x;
+      cw[u] = w < nw ? __ldcs(codes32 + w) : 0u;
+      sc[u] = w < nw ? (int)scales[(w << 2) >> gs] : 0;
     }
-    uint4* d = reinterpret_cast<uint4*>(out) + ch * 4;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) __stcs(d + q, make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]));
+    for (int u = 0; u < U; ++u) {
+      const int64_t w = t0 + u * (int64_t)blockDim.x + threadIdx.x;
+      if (w >= nw) continue;
+      const int a = sc[u];
+      const bool fast = (a + EMIN >= -126) && (a + F::EMAX <= 126);
+      uint32_t o[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const uint32_t code = (cw[u] >> (8 * i)) & 0xFFu;
+        const uint32_t m = code & F::MMASK;
+        uint32_t r;
+        if (fast) {
+          r = m ? tab[m] + (uint32_t)(a * (1 << 23)) : 0u;
+        } else if (m == 0u) {
+          r = 0u;
+        } else {
+          const int nn = (int)m - F::B;
+          const int e = nn >> F::C, k = nn & (F::K - 1);
+          const float ck = __uint_as_float(F::K == 8 ? CFP_CK_F32_K8_DEV[k] : CFP_CK_F32_K4_DEV[k]);
+          const int E = a + e;
+          const int E1 = E < -126 ? -126 : (E > 127 ? 127 : E);
+          const int E2 = E - E1;  // in [-18, 15]
+          float y = __fmul_rn(ck, __uint_as_float((uint32_t)(E1 + 127) << 23));
+          y = __fmul_rn(y, __uint_as_float((uint32_t)(E2 + 127) << 23));
+          r = __float_as_uint(y);
+        }
+        o[i] = m ? (r | ((code & 0x80u) << 24)) : 0u;
+      }
+      __stcs(out4 + w, make_uint4(o[0], o[1], o[2], o[3]));
+    }
   }
 }
 
@@ -854,6 +870,7 @@ __global__ void __launch_bounds__(256) qs_encode_kernel(const T* __restrict__ x,
   __shared__ uint32_t lut[256];
   for (int i = threadIdx.x; i < 256; i += blockDim.x) lut[i] = __ldg(lut_src<Fmt<FMT>::K>() + i);
   __syncthreads();
+  const int gs = __ffs(G) - 1;
   bool nan = false;
   int64_t run_g = -1;
   int a = 0;
@@ -864,7 +881,7 @@ __global__ void __launch_bounds__(256) qs_encode_kernel(const T* __restrict__ x,
       a = choose_scale<FMT>(amax[g], D ? D + g * 10 : nullptr, D ? rule : 0);
     }
     codes[i] = (uint8_t)encode_slow<FMT>(lut, load_bits(x, i), a, nan);
-    if (i % G == 0) scales[i / G] = (int8_t)a;
+    if ((i & (G - 1)) == 0) scales[i >> gs] = (int8_t)a;  // G is a power of two
   }
   if (nan && status) atomicOr(status, CURVEFP_DEV_NAN);
 }

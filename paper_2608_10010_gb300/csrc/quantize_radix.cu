@@ -12,8 +12,9 @@ template <int FMT>
 __global__ void __launch_bounds__(256) dequantize_radix_kernel(const uint8_t* __restrict__ codes,
                                                                const int8_t* __restrict__ scales, int64_t n, int G,
                                                                float* __restrict__ out) {
+  const int gs = __ffs(G) - 1;  // G is a power of two
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
-    out[i] = radix_recon_f32<FMT>(__ldg(codes + i), (int)__ldg(scales + i / G));
+    out[i] = radix_recon_f32<FMT>(__ldg(codes + i), (int)__ldg(scales + (i >> gs)));
 }
 
 }  // namespace

@@ -160,6 +160,22 @@ def test_dequantize_all_codes_all_scales(torch, fmt):
 
 
 @pytest.mark.parametrize("fmt", FORMATS)
+def test_dequantize_large_grid(torch, fmt):
+    """8.4M random codes (more words than one pass of the grid covers, so the
+    grid-stride loop runs several times) under random scales, bit-exact."""
+    import paper_2608_10010_gb300 as cfp
+
+    rng = np.random.default_rng(404)
+    codes = rng.integers(0, 256, size=(4096, 2048), dtype=np.uint8)
+    if fmt == "E3C3":
+        codes &= 0xBF
+    scales = rng.integers(-40, 40, size=(4096, 2048 // 32), dtype=np.int8)
+    out = cfp.dequantize(to_dev(torch, codes), to_dev(torch, scales), fmt, 32)
+    ref = oracle.dequantize(codes, scales, fmt, 32)
+    assert np.array_equal(out.cpu().numpy().view(np.uint32), ref.view(np.uint32))
+
+
+@pytest.mark.parametrize("fmt", FORMATS)
 def test_roundtrip_on_gpu(torch, fmt):
     """deq(Q(x)) on the GPU equals the oracle's, and re-quantizing it with the
     GPU gives the oracle's codes (the round-trip invariants are pinned on the
