@@ -153,18 +153,26 @@ curvefp_status_t curvefp_quantize_static(curvefp_format_t fmt, int block, curvef
                                          int64_t cols, uint8_t* codes, int8_t* scales, void* workspace,
                                          size_t workspace_bytes, uint32_t* device_status, void* stream);
 
-/* curvefp_quantize_static without a workspace argument: the scratch lives
- * in a fixed device array inside the library (CURVEFP_NOALLOC_SCRATCH_BYTES,
- * enough for row groups of up to ~100,000 rows; tensor and block groups need
- * almost none), so the call allocates nothing and takes nothing from the
- * caller.  Not from the paper: an interface variant of the static quantizer.
- *   Returns CURVEFP_ERR_UNSUPPORTED when the groups need more scratch than the
- *   array holds.  The array is shared by every call on a device: calls must
- *   not overlap (one stream at a time, or ordered by events).  The first call
- *   on a device looks the array up (cudaGetSymbolAddress) and so must not be
- *   the first call made inside a CUDA-graph capture; later calls are
- *   capturable (one memset and three kernels).  Other arguments, results and
- *   errors as curvefp_quantize_static. */
+/* curvefp_quantize_static without a workspace argument, for callers that
+ * cannot allocate device memory: code running where cudaMalloc is not
+ * allowed or would stall other work (it can synchronize the device), code
+ * whose device memory is owned by a host framework's own pool, and hosts
+ * with a fixed memory budget that reserve everything up front.  The paper
+ * has no counterpart; this is an interface variant of the static quantizer.
+ *   The scratch lives in a fixed file-scope device array of the library,
+ *   CURVEFP_NOALLOC_SCRATCH_BYTES (8 MiB) on every GPU that loads the library,
+ *   held until the process exits.  That is enough for row groups of up to
+ *   ~100,000 rows; tensor and block groups need almost none.  The call makes
+ *   no cudaMalloc, cudaFree or other allocating call.
+ *   Returns CURVEFP_ERR_UNSUPPORTED, before any device work, when the groups
+ *   need more scratch than the array holds.
+ *   The array is shared by every call on a device and keeps the last call's
+ *   contents; each call clears the part it uses before its kernels.  Calls
+ *   that overlap on the GPU (different streams without ordering) race on it.
+ *   The first call on a device looks the array's device address up
+ *   (cudaGetSymbolAddress, with that device current); make that first call
+ *   before any stream capture.  Other arguments, results and errors as
+ *   curvefp_quantize_static. */
 #define CURVEFP_NOALLOC_SCRATCH_BYTES (8u << 20)
 curvefp_status_t curvefp_quantize_static_noalloc(curvefp_format_t fmt, int block, curvefp_scale_group_t group,
                                                  curvefp_scale_rule_t rule, const void* x, curvefp_dtype_t dtype,

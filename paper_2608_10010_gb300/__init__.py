@@ -138,8 +138,10 @@ def quantize_static(x, fmt, block: int = 32, group: str = "block", rule: str = "
 
 def quantize_static_noalloc(x, fmt, block: int = 32, group: str = "block", rule: str = "mse", codes=None,
                             scales=None, status=None, stream=None):
-    """quantize_static through the entry point that takes no workspace (its
-    scratch is a fixed device array inside the library)."""
+    """quantize_static through the entry point that allocates nothing, for
+    callers that cannot allocate device memory: its scratch is a fixed device
+    array inside the library (row groups up to ~100,000 rows), shared by every
+    call on the device, so calls that overlap on the GPU race."""
     import torch
 
     assert x.dim() == 2 and x.is_cuda and x.is_contiguous()

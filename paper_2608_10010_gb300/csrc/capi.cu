@@ -87,8 +87,11 @@ curvefp_status_t curvefp_quantize_static(curvefp_format_t fmt, int block, curvef
                                                device_status, static_cast<cudaStream_t>(stream), sm_count()));
 }
 
-/* Scratch for curvefp_quantize_static_noalloc: a file-scope device array
- * (reserved when the library's module loads, never allocated by a call). */
+/* Scratch for curvefp_quantize_static_noalloc, the entry point for callers
+ * that cannot allocate device memory: a file-scope device array (reserved on
+ * each GPU when the library's module loads, held until exit, never allocated
+ * by a call).  In host code its name is only a host-side stand-in; kernels
+ * get the device address from cudaGetSymbolAddress. */
 static __device__ __align__(256) unsigned char g_static_scratch[CURVEFP_NOALLOC_SCRATCH_BYTES];
 
 curvefp_status_t curvefp_quantize_static_noalloc(curvefp_format_t fmt, int block, curvefp_scale_group_t group,

@@ -1,7 +1,14 @@
-"""The static quantizer's no-workspace entry point (scratch in a fixed
-device array inside the library): same results as the workspace entry point
-on two calls in a row, and oversize requests rejected before any device work.
-Collected last so that it also runs after every other GPU test."""
+"""The static quantizer's entry point that allocates nothing.
+
+Some callers cannot allocate device memory: code where cudaMalloc is not
+allowed or would stall other work (it can synchronize the device), code whose
+device memory belongs to a host framework's own pool, and hosts that reserve a
+fixed memory budget up front.  For them the library keeps the static
+quantizer's scratch in a fixed device array of its own.  This file checks that
+entry point against the workspace entry point on two calls in a row (the
+array keeps the previous call's contents, so each call must clear what it
+needs) and that oversize requests are rejected before any device work.  It is
+collected last so that it also runs after every other GPU test."""
 import ctypes
 
 import numpy as np
