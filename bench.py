@@ -178,7 +178,7 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
         tops = 2.0 * Mx * Nx * Kx / (ms / 1e3) / 1e12
         r = {"case": name, "algo": algo, "M": Mx, "N": Nx, "K": Kx, "formats": f"{fa}x{fb}", "ms": round(ms, 4),
              "tops": round(tops, 3)}
-        if algo == "tensor":
+        if algo in ("tensor", "tensor_narrow"):
             r["tensor_work_frac"] = round(tops * planes / fp8_peak, 4)
         if hbm_bound:
             wbytes = Nx * Kx + Nx * Kx // G
@@ -280,6 +280,9 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
             Xf, Wf = inputs.ffn_cuda(Mf, Kf)
             gemm_case(f"ffn M={Mf} K={Kf}", q(Xf, "E3C3", 0), "E3C3", q(Wf, "E3C3", 1), "E3C3", 64,
                       hbm_bound=Mf <= 128)
+            if Mf <= 128:  # few activation rows: phases along the MMA's N dimension
+                gemm_case(f"ffn M={Mf} K={Kf} narrow", q(Xf, "E3C3", 0), "E3C3", q(Wf, "E3C3", 1), "E3C3", 64,
+                          hbm_bound=True, algo="tensor_narrow")
             if Mf <= 8:  # decode sizes: the CUDA-core kernel as well
                 gemm_case(f"ffn M={Mf} K={Kf} skinny", q(Xf, "E3C3", 0), "E3C3", q(Wf, "E3C3", 1), "E3C3", 64,
                           hbm_bound=True, algo="skinny")
@@ -659,8 +662,9 @@ def run_reference(args):
 def run_only(args):
     """One kernel of the path, a few launches, no timing: the target of the
     ncu captures (--only gemm: the tensor-core GEMM of the workload above;
-    --only quantize: 2^28 BF16 elements, E4C3, block 32; skinny, reuse, r89:
-    the decode GEMM, the reused-operand dgrad and the r = 2^{8/9} GEMM)."""
+    --only quantize: 2^28 BF16 elements, E4C3, block 32; skinny, narrow,
+    reuse, r89: the decode GEMM, the few-row tensor-core GEMM, the
+    reused-operand dgrad and the r = 2^{8/9} GEMM)."""
     import torch
 
     import paper_2608_10010_gb300 as cfp
@@ -690,6 +694,14 @@ def run_only(args):
             c = cfp.gemm(a, sa, b, sb, "E3C3", "E3C3", G, "skinny")
         torch.cuda.synchronize()
         print(json.dumps({"only": "skinny", "launches": args.steps, "c00": float(c[0, 0])}))
+    elif args.only == "narrow":  # few-row GEMM: FFN M = --narrow-m, E3C3, W[14336 x 4096]
+        Xf, Wf = inputs.ffn_cuda(args.narrow_m, 4096)
+        a, sa = cfp.quantize(Xf, "E3C3", G, 0)
+        b, sb = cfp.quantize(Wf, "E3C3", G, 1)
+        for _ in range(args.steps):
+            c = cfp.gemm(a, sa, b, sb, "E3C3", "E3C3", G, "tensor_narrow")
+        torch.cuda.synchronize()
+        print(json.dumps({"only": "narrow", "M": args.narrow_m, "launches": args.steps, "c00": float(c[0, 0])}))
     elif args.only == "reuse":  # dgrad on the reused weight, triplet shape (T 4096, 4096 -> 11008)
         X, Wt, dY = inputs.training_triplet_cuda()
         qw, sw = cfp.quantize(Wt, "E4C3", G, 1)
@@ -716,7 +728,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--only", choices=["gemm", "quantize", "skinny", "reuse", "r89"], default=None)
+    ap.add_argument("--only", choices=["gemm", "quantize", "skinny", "narrow", "reuse", "r89"], default=None)
+    ap.add_argument("--narrow-m", type=int, default=16, help="activation rows of --only narrow")
     ap.add_argument("--no-sweep", action="store_true", help="skip the other workloads (quantize sweep, GEMM shapes)")
     ap.add_argument("--out", default=None, help="also write the JSON line to this file (atomically: temp + rename)")
     args = ap.parse_args()

@@ -86,14 +86,19 @@ typedef enum {
  * code tiles streamed by TMA).  SKINNY: decode-sized GEMMs (M <=
  * CURVEFP_SKINNY_MAX_M) on the CUDA cores with the same FP32 per-phase
  * accumulation, every product formed from the two codes (the tensor-core
- * tile costs the same for any M up to 128).  AUTO: SKINNY for M <=
- * CURVEFP_AUTO_SKINNY_M, else TENSOR. */
+ * tile costs the same for any M up to 128).  TENSOR_NARROW: the tensor-core
+ * method for few activation rows (Sec. 3.2, Eq. 2, Eq. 5): the weight rows
+ * are the 128-row operand and the L phases of every token run along the
+ * MMA's N dimension, so a step of 32 codes takes K_b MMAs of 128 x (L Mt)
+ * (Mt <= 256/L tokens per CTA) instead of K_a K_b MMAs of a 128-row tile.
+ * AUTO: SKINNY for M <= CURVEFP_AUTO_SKINNY_M, else TENSOR. */
 typedef enum {
   CURVEFP_GEMM_EXACT = 0,
   CURVEFP_GEMM_TENSOR = 1,
   CURVEFP_GEMM_TENSOR_SPARSE = 2,
   CURVEFP_GEMM_SKINNY = 3,
-  CURVEFP_GEMM_AUTO = 4
+  CURVEFP_GEMM_AUTO = 4,
+  CURVEFP_GEMM_TENSOR_NARROW = 5
 } curvefp_gemm_algo_t;
 #define CURVEFP_SKINNY_MAX_M 8
 #define CURVEFP_AUTO_SKINNY_M 4
@@ -199,11 +204,13 @@ curvefp_status_t curvefp_dequantize(curvefp_format_t fmt, int block, const uint8
  * Requirements: K % block == 0; a, b 16-byte aligned.
  * EXACT: S_h exact, combine in FP64, one FP32 rounding; outputs whose scale
  *   spread leaves the int128 window raise CURVEFP_DEV_RANGE (values undefined).
- * TENSOR, TENSOR_SPARSE: S_h accumulated in FP32 on the tensor cores, combine
- *   in FP32; plane values below 2^-14 of a row's largest block scale flush.
- *   Format pairs: E3C3 x E3C3, E4C3 x E4C3, E5C2 x E4C3, E4C3 x E5C2,
- *   E5C2 x E5C2, and (TENSOR) E4C3_R8_9 x E4C3_R8_9 (others return
- *   CURVEFP_ERR_UNSUPPORTED).
+ * TENSOR, TENSOR_SPARSE, TENSOR_NARROW: S_h accumulated in FP32 on the
+ *   tensor cores, combine in FP32; plane values below 2^-14 of a row's largest
+ *   block scale flush.  Format pairs: E3C3 x E3C3, E4C3 x E4C3, E5C2 x E4C3,
+ *   E4C3 x E5C2, E5C2 x E5C2, and (TENSOR) E4C3_R8_9 x E4C3_R8_9 (others
+ *   return CURVEFP_ERR_UNSUPPORTED).  TENSOR and TENSOR_NARROW zero parts of C
+ *   with cudaMemsetAsync before adding split-K pieces to them (two additions
+ *   per output, so results do not depend on their order).
  * SKINNY (M <= CURVEFP_SKINNY_MAX_M, else CURVEFP_ERR_UNSUPPORTED), AUTO:
  *   S_h accumulated in FP32 per output (products relative to the output's
  *   largest scale sum; products below the FP32 normal range relative to it

@@ -158,6 +158,11 @@ curvefp_status_t curvefp_gemm(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, 
     if (M > CURVEFP_SKINNY_MAX_M) return CURVEFP_ERR_UNSUPPORTED;
     return from_cuda(cfp::launch_gemm_skinny(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, st, sm_count()));
   }
+  if (algo == CURVEFP_GEMM_TENSOR_NARROW) {
+    if (!cfp::gemm_narrow_supported(fmt_a, fmt_b)) return CURVEFP_ERR_UNSUPPORTED;
+    return from_cuda(cfp::launch_gemm_tensor_narrow(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, device_status, st,
+                                                    sm_count()));
+  }
   if (algo == CURVEFP_GEMM_TENSOR || algo == CURVEFP_GEMM_TENSOR_SPARSE) {
     if (!cfp::gemm_tensor_supported(fmt_a, fmt_b)) return CURVEFP_ERR_UNSUPPORTED;
     if (algo == CURVEFP_GEMM_TENSOR_SPARSE)
