@@ -91,7 +91,10 @@ typedef enum {
  * are the 128-row operand and the L phases of every token run along the
  * MMA's N dimension, so a step of 32 codes takes K_b MMAs of 128 x (L Mt)
  * (Mt <= 256/L tokens per CTA) instead of K_a K_b MMAs of a 128-row tile.
- * AUTO: SKINNY for M <= CURVEFP_AUTO_SKINNY_M, else TENSOR. */
+ * AUTO (measured crossovers on the FFN decode shapes, N = 14336, K = 4096):
+ * SKINNY for M <= CURVEFP_AUTO_SKINNY_M; TENSOR_NARROW for M <=
+ * CURVEFP_AUTO_NARROW_M where the format pair has it; TENSOR above; SKINNY up
+ * to CURVEFP_SKINNY_MAX_M for pairs without a tensor-core kernel. */
 typedef enum {
   CURVEFP_GEMM_EXACT = 0,
   CURVEFP_GEMM_TENSOR = 1,
@@ -101,7 +104,8 @@ typedef enum {
   CURVEFP_GEMM_TENSOR_NARROW = 5
 } curvefp_gemm_algo_t;
 #define CURVEFP_SKINNY_MAX_M 8
-#define CURVEFP_AUTO_SKINNY_M 4
+#define CURVEFP_AUTO_SKINNY_M 1
+#define CURVEFP_AUTO_NARROW_M 96
 
 /* Bits of the device status word. */
 #define CURVEFP_DEV_NAN 1u     /* quantize: a NaN input was encoded as 0x00        */

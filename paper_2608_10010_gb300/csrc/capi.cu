@@ -151,9 +151,18 @@ curvefp_status_t curvefp_gemm(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, 
                                             device_status, st));
   // rational radix: EXACT, and TENSOR for r = 2^{8/9}
   if (fmt_radix(fmt_a) && algo != CURVEFP_GEMM_TENSOR) return CURVEFP_ERR_UNSUPPORTED;
-  // AUTO: the CUDA-core kernel where it is faster than a 128-row tensor-core
-  // tile (measured up to M = 4 on the FFN decode shapes)
-  if (algo == CURVEFP_GEMM_AUTO) algo = M <= CURVEFP_AUTO_SKINNY_M ? CURVEFP_GEMM_SKINNY : CURVEFP_GEMM_TENSOR;
+  // AUTO: the fastest kernel by M (crossovers measured on the FFN decode
+  // shapes): CUDA cores for one row, phases along N up to 96 rows, tiles above
+  if (algo == CURVEFP_GEMM_AUTO) {
+    if (M <= CURVEFP_AUTO_SKINNY_M)
+      algo = CURVEFP_GEMM_SKINNY;
+    else if (M <= CURVEFP_AUTO_NARROW_M && cfp::gemm_narrow_supported(fmt_a, fmt_b))
+      algo = CURVEFP_GEMM_TENSOR_NARROW;
+    else if (M <= CURVEFP_SKINNY_MAX_M && !cfp::gemm_tensor_supported(fmt_a, fmt_b))
+      algo = CURVEFP_GEMM_SKINNY;
+    else
+      algo = CURVEFP_GEMM_TENSOR;
+  }
   if (algo == CURVEFP_GEMM_SKINNY) {
     if (M > CURVEFP_SKINNY_MAX_M) return CURVEFP_ERR_UNSUPPORTED;
     return from_cuda(cfp::launch_gemm_skinny(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, st, sm_count()));

@@ -48,23 +48,30 @@ template <int FX, int FW>
 struct TcnCfg {
   using P = Pair<FX, FW>;
   static constexpr int KW = Fmt<FW>::K, L = P::L, WX = P::WA, WW = P::WB;
-  static constexpr int BM = 128;         // weight rows per CTA (TMEM lanes)
-  static constexpr int KS = 32;          // codes per pipeline step (K of one FP8 MMA)
-  static constexpr int MTMAX = 256 / L;  // tokens per CTA: L Mt <= 256 (MMA N)
-  static constexpr int NBLK = 2 * L;     // column blocks of the doubled sequence
-  static constexpr int NSB = 4;          // pipeline depth (X stages = W TMEM units)
-  static constexpr int AU_COLS = KW * 8; // TMEM columns of one step's W planes
-  static constexpr int ACOL0 = 256;      // W units after the accumulator
+  static constexpr int BM = 128;          // weight rows per CTA (TMEM lanes)
+  static constexpr int KS = 32;           // codes per pipeline step (K of one FP8 MMA)
+  static constexpr int MTMAX = 256 / L;   // tokens per CTA: L Mt <= 256 (MMA N)
+  static constexpr int NBLK = 2 * L;      // column blocks of the doubled sequence
+  static constexpr int NSB = 4;           // pipeline depth (X stages = W TMEM units)
+  static constexpr int AU_COLS = KW * 8;  // TMEM columns of one step's W planes
+  static constexpr int ACOL0 = 256;       // W units after the accumulator
   static_assert(ACOL0 + NSB * AU_COLS <= 512, "TMEM budget");
-  static constexpr int NAW = 8;              // W producer warps
-  static constexpr int NXT = 2 * MTMAX;      // X producer threads
-  static constexpr int THREADS = NAW * 32 + NXT + 32;
-  static constexpr int MMA_WARP = (NAW * 32 + NXT) / 32;
-  static_assert(NXT % 32 == 0, "X producer warps");
+  static_assert(L % 4 == 0 && KW % 2 == 0, "epilogue phase groups, plane pairs");
+  // Producer groups take turns: W group g % NGW and X group g % NGX produce
+  // step g, so each producer thread has NGW (NGX) steps of time per step.
+  static constexpr int NGW = 2;                 // W groups of 4 warps (one thread per weight row)
+  static constexpr int XPG = MTMAX / 16;        // X warps per group (two threads per token)
+  static constexpr int NGX = L == 8 ? 3 : 2;    // X groups
+  static constexpr int NWT = NGW * 128;         // W threads
+  static constexpr int NXT = NGX * XPG * 32;    // X threads
+  static constexpr int THREADS = NWT + NXT + 32;
+  static constexpr int MMA_WARP = (NWT + NXT) / 32;
   static constexpr int BSTAGE = NBLK * MTMAX * 32;  // bytes of one step's X planes
   static constexpr int PBX = FX == CURVEFP_E5C2 ? 1 : 0;  // plane exponent bias
   static constexpr int PBW = FW == CURVEFP_E5C2 ? 1 : 0;
-  static constexpr int PF = 8;  // steps of codes in flight per producer thread
+  static constexpr int PFW = 4;  // own steps of weight codes in flight per W thread
+  static constexpr int PFX = 2;  // own steps of activation codes in flight per X thread
+  static constexpr int XI = MTMAX * 8 / (XPG * 32);  // X work items (4-code words) per thread and step
   // more than half of the SM's shared memory: one CTA per SM (the split plan
   // assumes it, and the CTA allocates all of TMEM)
   static constexpr size_t SMEM_USED = (size_t)NSB * BSTAGE + 2048;
@@ -77,6 +84,38 @@ __device__ __forceinline__ uint32_t core_off(int row, int kc) {
   return (uint32_t)((row >> 3) * 256 + kc * 128 + (row & 7) * 16);
 }
 
+// Largest block scale of a row (the row reference of the plane values).
+__device__ __forceinline__ int row_ref(const int8_t* s, int nb) {
+  int ref = -128;
+  if ((nb & 15) == 0 && (reinterpret_cast<uintptr_t>(s) & 15) == 0) {
+    uint32_t m4 = 0x80808080u;
+#pragma unroll 8
+    for (int b = 0; b < nb; b += 16) {
+      const uint4 q = __ldg(reinterpret_cast<const uint4*>(s + b));
+      m4 = __vmaxs4(m4, __vmaxs4(__vmaxs4(q.x, q.y), __vmaxs4(q.z, q.w)));
+    }
+    ref = max(max((int)(int8_t)(m4 & 0xFF), (int)(int8_t)((m4 >> 8) & 0xFF)),
+              max((int)(int8_t)((m4 >> 16) & 0xFF), (int)(int8_t)(m4 >> 24)));
+  } else {
+#pragma unroll 8
+    for (int b = 0; b < nb; ++b) ref = max(ref, (int)__ldg(s + b));
+  }
+  return ref;
+}
+
+__device__ __forceinline__ bool wait_all(uint64_t* bar, uint32_t parity) {
+  return __all_sync(0xffffffffu, tc::mbar_wait(bar, parity));
+}
+
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15, %16};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
+      "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
+}
+
 }  // namespace
 
 template <int FX, int FW>
@@ -85,7 +124,7 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
                     const int8_t* __restrict__ sW, int M, int N, int K, int G, int gshift, int Mt,
                     float* __restrict__ C, uint32_t* status, const TailPlan plan) {
   using Cfg = TcnCfg<FX, FW>;
-  constexpr int L = Cfg::L, NSB = Cfg::NSB, NAW = Cfg::NAW, PF = Cfg::PF;
+  constexpr int L = Cfg::L, NSB = Cfg::NSB;
   static_assert(NSB == TC_MAX_RING, "barrier rings");
   extern __shared__ __align__(1024) uint8_t smem[];
   uint8_t* xstage = smem;
@@ -108,10 +147,15 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
   }
   const int x0 = (tile / ntw) * Mt, w0 = (tile % ntw) * Cfg::BM;
   const int nb = K / G, total = s1 - s0;
+  // Accumulator copies: consecutive MMAs of a step into one accumulator wait
+  // for each other's accumulation, so where the accumulator is at most 128
+  // columns the weight planes rotate over 2 or 4 copies (NP columns each)
+  // that the epilogue adds up.
+  const int NP = L * Mt, nacc = NP <= 64 ? 4 : (NP <= 128 ? 2 : 1);
 
   if (tid == 0) {
     for (int s = 0; s < NSB; ++s) {
-      tc::mbar_init(&sh.full[s], NAW + Cfg::NXT / 32);  // one arrival per producer warp
+      tc::mbar_init(&sh.full[s], 4 + Cfg::XPG);  // the step's W group and X group, one arrival per warp
       tc::mbar_init(&sh.empty[s], 1);
     }
     tc::mbar_init(&sh.acc_full, 1);
@@ -122,98 +166,84 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
     tc::tmem_alloc(&sh.tmem_base, 512);
     tc::tmem_relinquish();
   }
-  // producer geometry and the row's reference exponent (largest block scale)
-  const bool is_w = warp < NAW;
-  const bool is_prod = warp < Cfg::MMA_WARP;
-  const int t_x = tid - NAW * 32;
-  const int rloc = is_w ? ((warp & 3) * 32 + lane) : (t_x >> 1);  // weight row / token of the CTA
-  const int part = is_w ? (warp >> 2) : (t_x & 1);                // 16-byte half of the step's 32 codes
-  const int r = (is_w ? w0 : x0) + rloc;
-  const bool rowok = is_prod && (is_w ? r < N : (rloc < Mt && r < M));
+  const bool is_w = tid < Cfg::NWT, is_x = !is_w && warp < Cfg::MMA_WARP;
+  // W threads: weight row (TMEM lane) and group; X threads: group.  The
+  // row references: a weight row per W thread, a token per thread of the
+  // first X group.  The X stages start at zero (padding tokens and empty
+  // lattice positions are never written).
+  const int wrow = w0 + (warp & 3) * 32 + lane, gw = warp >> 2;
+  const int t_x = tid - Cfg::NWT, gx = t_x / (Cfg::XPG * 32);
   int ref = -128;
-  if (rowok) {
-    const int8_t* s = (is_w ? sW : sX) + (int64_t)r * nb;
-    if ((nb & 15) == 0 && (reinterpret_cast<uintptr_t>(s) & 15) == 0) {
-      uint32_t m4 = 0x80808080u;
-#pragma unroll 8
-      for (int b = 0; b < nb; b += 16) {
-        const uint4 q = __ldg(reinterpret_cast<const uint4*>(s + b));
-        m4 = __vmaxs4(m4, __vmaxs4(__vmaxs4(q.x, q.y), __vmaxs4(q.z, q.w)));
-      }
-      ref = max(max((int)(int8_t)(m4 & 0xFF), (int)(int8_t)((m4 >> 8) & 0xFF)),
-                max((int)(int8_t)((m4 >> 16) & 0xFF), (int)(int8_t)(m4 >> 24)));
-    } else {
-#pragma unroll 8
-      for (int b = 0; b < nb; ++b) ref = max(ref, (int)__ldg(s + b));
-    }
+  if (is_w && wrow < N) ref = row_ref(sW + (int64_t)wrow * nb, nb);
+  if (is_x && t_x < Cfg::MTMAX) {
+    int rx = -128;
+    if (t_x < Mt && x0 + t_x < M) rx = row_ref(sX + (int64_t)(x0 + t_x) * nb, nb);
+    sh.refB[t_x] = rx;
   }
-  if (!is_w && is_prod && part == 0 && rloc < Cfg::MTMAX) sh.refB[rloc] = ref;
+  for (int o = tid * 16; o < NSB * Cfg::BSTAGE; o += Cfg::THREADS * 16)
+    *reinterpret_cast<uint4*>(xstage + o) = make_uint4(0, 0, 0, 0);
+  tc::fence_proxy_async_smem();
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = sh.tmem_base;
 
-  if (is_prod) {
-    // ------------------------------ producers ------------------------------
-    const uint8_t* src = (is_w ? W : X) + (int64_t)r * K + part * 16;
-    const int8_t* srow = (is_w ? sW : sX) + (int64_t)r * nb;
-    const int bias = is_w ? Cfg::PBW : Cfg::PBX;
-    auto load = [&](int g, uint4& cw, int& raw) {
-      cw = make_uint4(0, 0, 0, 0);
+  if (is_w) {
+    // ---------------------------- W producers -----------------------------
+    constexpr int PF = Cfg::PFW, NGW = Cfg::NGW;
+    const bool rowok = wrow < N;
+    const uint8_t* src = W + (int64_t)wrow * K;
+    const int8_t* srow = sW + (int64_t)wrow * nb;
+    // own step i of this group is pipeline step g = gw + i NGW
+    auto load = [&](int i, uint4& lo, uint4& hi, int& raw) {
+      lo = hi = make_uint4(0, 0, 0, 0);
       raw = 0;
+      const int g = gw + i * NGW;
       if (rowok && g < total) {
         const int s = s0 + g;
-        cw = __ldg(reinterpret_cast<const uint4*>(src + (int64_t)s * Cfg::KS));
+        const uint4* p = reinterpret_cast<const uint4*>(src + (int64_t)s * Cfg::KS);
+        lo = __ldg(p);
+        hi = __ldg(p + 1);
         raw = (int)__ldg(srow + (s >> gshift));
       }
     };
     const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-    // Epilogue (W producers, after the last MMA): chunks of 8 tokens, this
-    // thread's half taking every other chunk; per token the phase sums
-    // D[w][h Mt + m] are combined as sum_h 2^{h/L} S_h (FP32, phase order)
-    // and scaled by 2^{ref_w + ref_m}.  A whole tile stores C, a K piece adds
-    // to zeroed C.
-    auto epilogue = [&]() -> bool {
-      const bool ok = __all_sync(0xffffffffu, tc::mbar_wait(&sh.acc_full, 0));
-      if (!ok) {
-        if (lane == 0) raise_flag(status, CURVEFP_DEV_TIMEOUT);
-        sh.abort_flag = 1;
-      }
-      tc::fence_after_sync();
-      const int nch = Mt >> 3;
-#pragma unroll 1
-      for (int ch = part; ch < nch; ch += 2) {
-        uint32_t acc[L][8];
+    // The hand-over of an own step (wait for its TMEM stores, arrive) is
+    // deferred until the next own step is decoded, so the store latency
+    // overlaps the decode; the step before is still at least two steps
+    // ahead of the empty wait that could depend on it.
+    int pend = -1;  // stage of the own step not yet handed over
+    auto hand_over = [&]() {
+      if (pend < 0) return;
+      tc::tmem_wait_st();
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&sh.full[pend]);
+      pend = -1;
+    };
+    auto step = [&](const int g, const uint4 lo, const uint4 hi, const int raw) -> bool {
+      const int st = g % NSB, off = raw - ref - Cfg::PBW;
+      // the 32 codes of the row's step: value words and curve-index masks;
+      // plane j of word w = p[w][j & 3] & (bit 2 of k set ? mk2 : ~mk2)
+      uint32_t p[8][4], m2[8];
 #pragma unroll
-        for (int h = 0; h < L; ++h) tc::tmem_ld8(lane_base + h * Mt + ch * 8, acc[h]);
-        tc::tmem_wait_ld();
-        if (rowok && ok) {
+      for (int h = 0; h < 2; ++h) {
+        uint32_t v[4], vc[4], mk[4][4];
+        PlaneFmt<FW>::template decode<PLANE_E5M2, 4>(h ? hi : lo, off, v, vc, mk, false);
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const int tok = ch * 8 + j, m = x0 + tok;
-            if (m < M) {
-              float t = 0.f;
-#pragma unroll
-              for (int h = 0; h < L; ++h) t = fmaf(phase_const(L, h), __uint_as_float(acc[h][j]), t);
-              const float y = scalbnf(t, ref + Cfg::PBW + sh.refB[tok] + Cfg::PBX);
-              float* dst = C + (int64_t)m * N + r;
-              if (split)
-                atomicAdd(dst, y);
-              else
-                *dst = y;
-            }
-          }
+        for (int c = 0; c < 4; ++c) {
+          const int w = h * 4 + c;
+          p[w][0] = v[c] & ~mk[c][0] & ~mk[c][1];
+          p[w][1] = v[c] & mk[c][0] & ~mk[c][1];
+          p[w][2] = v[c] & ~mk[c][0] & mk[c][1];
+          p[w][3] = v[c] & mk[c][0] & mk[c][1];
+          m2[w] = mk[c][2];
         }
       }
-      return ok;
-    };
-    // One pipeline step of this producer thread; false ends the loop.
-    auto step = [&](const int g, const uint4 cw, const int raw) -> bool {
-      const int off = raw - ref - bias;
-      const int st = g % NSB;
+      hand_over();
       if (g >= NSB) {
-        // stage / TMEM unit st is free once the MMAs of step g - NSB retired
-        const bool ok = __all_sync(0xffffffffu, tc::mbar_wait(&sh.empty[st], ((g / NSB) - 1) & 1));
+        // TMEM unit st is free once the MMAs of step g - NSB retired
+        const bool ok = wait_all(&sh.empty[st], ((g / NSB) - 1) & 1);
         tc::fence_after_sync();
         if (!ok) {
           if (lane == 0) raise_flag(status, CURVEFP_DEV_TIMEOUT);
@@ -221,78 +251,190 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
           return false;
         }
       }
-      if (is_w) {
-        uint32_t v[4], vc[4], mk[4][4];
-        PlaneFmt<FW>::template decode<PLANE_E5M2, 4>(cw, off, v, vc, mk, false);
-        uint32_t pl[4][8];
+      // planes 2jp and 2jp + 1: 16 consecutive columns of the unit
 #pragma unroll
-        for (int c = 0; c < 4; ++c) PlaneFmt<FW>::planes(v[c], mk[c], pl[c]);
-        // plane k_w: 8 columns of the unit, this thread's half = 4 of them
+      for (int jp = 0; jp < Cfg::KW / 2; ++jp) {
+        uint32_t r[16];
 #pragma unroll
-        for (int j = 0; j < Cfg::KW; ++j) {
-          const uint32_t reg[4] = {pl[0][j], pl[1][j], pl[2][j], pl[3][j]};
-          tc::tmem_st4(lane_base + Cfg::ACOL0 + st * Cfg::AU_COLS + j * 8 + part * 4, reg);
+        for (int e = 0; e < 2; ++e) {
+          const int j = 2 * jp + e;
+#pragma unroll
+          for (int w = 0; w < 8; ++w) r[e * 8 + w] = p[w][j & 3] & ((j & 4) ? m2[w] : ~m2[w]);
         }
-        tc::tmem_wait_st();
-        tc::fence_before_sync();
-        __syncwarp();
-        if (lane == 0) tc::mbar_arrive(&sh.full[st]);
-        if (g == total - 1) return epilogue();
-      } else {
-        uint32_t v[4], vc[4], mk[4][4];
-        PlaneFmt<FX>::template decode<PLANE_E5M2, 4>(cw, off, v, vc, mk, true);
-        uint32_t pv[4][8], pc[4][8];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          PlaneFmt<FX>::planes(v[c], mk[c], pv[c]);
-          PlaneFmt<FX>::planes(vc[c], mk[c], pc[c]);
-        }
-        if (rloc < Mt) {
-          uint8_t* stg = xstage + (size_t)st * Cfg::BSTAGE;
-          // lattice position u holds plane u / WX where WX divides u
-#pragma unroll
-          for (int u = 0; u < L; ++u) {
-            const bool on = (u % Cfg::WX) == 0;
-            const int k = u / Cfg::WX;
-            const uint4 cq = on ? make_uint4(pc[0][k], pc[1][k], pc[2][k], pc[3][k]) : make_uint4(0, 0, 0, 0);
-            const uint4 pq = on ? make_uint4(pv[0][k], pv[1][k], pv[2][k], pv[3][k]) : make_uint4(0, 0, 0, 0);
-            *reinterpret_cast<uint4*>(stg + core_off(u * Mt + rloc, part)) = cq;
-            *reinterpret_cast<uint4*>(stg + core_off((L + u) * Mt + rloc, part)) = pq;
-          }
-        }
-        tc::fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) tc::mbar_arrive(&sh.full[st]);
+        tmem_st16(lane_base + Cfg::ACOL0 + st * Cfg::AU_COLS + jp * 16, r);
       }
+      pend = st;
       return true;
     };
-    // PF register sets of codes, each loaded PF steps before its use (the
-    // weights stream from HBM and a narrow step is short)
-    uint4 q[PF];
+    // PF register sets of codes, each loaded PF own steps before its use and
+    // never copied (no register move waits on an in-flight load)
+    const int nown = (total - gw + NGW - 1) / NGW;
+    uint4 ql[PF], qh[PF];
     int rq[PF];
 #pragma unroll
-    for (int u = 0; u < PF; ++u) load(u, q[u], rq[u]);
-    bool run = true;
-    for (int g = 0; g < total && run; g += PF) {
+    for (int u = 0; u < PF; ++u) load(u, ql[u], qh[u], rq[u]);
+    bool run = true, failed = false;
+    for (int i = 0; i < nown && run; i += PF) {
 #pragma unroll
       for (int u = 0; u < PF; ++u) {
-        if (g + u >= total || !step(g + u, q[u], rq[u])) {
+        if (i + u >= nown) {
           run = false;
           break;
         }
-        load(g + u + PF, q[u], rq[u]);
+        if (!step(gw + (i + u) * NGW, ql[u], qh[u], rq[u])) {
+          run = false;
+          failed = true;
+          break;
+        }
+        load(i + u + PF, ql[u], qh[u], rq[u]);
+      }
+    }
+    if (!failed) hand_over();
+    // Epilogue (after the last MMA): chunks of 8 tokens, chunk ch taken by
+    // group ch % NGW; per token the phase sums D[w][h Mt + m] are combined as
+    // sum_h 2^{h/L} S_h (FP32, phase order) and scaled by 2^{ref_w + ref_m}.
+    // A whole tile stores C, a K piece adds to zeroed C.
+    const bool aborted = __any_sync(0xffffffffu, read_abort(&sh.abort_flag) != 0);
+    const bool ok = !aborted && wait_all(&sh.acc_full, 0);
+    if (!ok && lane == 0) raise_flag(status, CURVEFP_DEV_TIMEOUT);
+    tc::fence_after_sync();
+#pragma unroll 1
+    for (int ch = gw; ch < (Mt >> 3); ch += NGW) {
+      float t[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) t[j] = 0.f;
+#pragma unroll
+      for (int h0 = 0; h0 < L; h0 += 4) {
+        // S_h = the sum of the accumulator copies (copy order fixed)
+        float sh4[4][8];
+#pragma unroll 1
+        for (int a = 0; a < nacc; ++a) {
+          uint32_t acc[4][8];
+#pragma unroll
+          for (int h = 0; h < 4; ++h) tc::tmem_ld8(lane_base + a * NP + (h0 + h) * Mt + ch * 8, acc[h]);
+          tc::tmem_wait_ld();
+#pragma unroll
+          for (int h = 0; h < 4; ++h)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) sh4[h][j] = a ? sh4[h][j] + __uint_as_float(acc[h][j]) : __uint_as_float(acc[h][j]);
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+#pragma unroll
+          for (int h = 0; h < 4; ++h) t[j] = fmaf(phase_const(L, h0 + h), sh4[h][j], t[j]);
+      }
+      if (rowok && ok) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int tok = ch * 8 + j, m = x0 + tok;
+          if (m < M) {
+            const float y = scalbnf(t[j], ref + Cfg::PBW + sh.refB[tok] + Cfg::PBX);
+            float* dst = C + (int64_t)m * N + wrow;
+            if (split)
+              atomicAdd(dst, y);
+            else
+              *dst = y;
+          }
+        }
+      }
+    }
+  } else if (is_x) {
+    // ---------------------------- X producers -----------------------------
+    // Work item wi of a group covers one 4-code word: lane bits of wi give 8
+    // tokens x 4 words of a 16-code chunk kc, so a warp's 4-byte stores fill
+    // 128 consecutive bytes of a column block.  Items of padding tokens (and
+    // lattice positions that hold no plane) write nothing: the stages were
+    // zeroed at the start.
+    constexpr int PF = Cfg::PFX, XI = Cfg::XI, NGX = Cfg::NGX;
+    const int tg = t_x % (Cfg::XPG * 32);  // thread of the group
+    bool act[XI];
+    const uint8_t* xsrc[XI];
+    const int8_t* xsc[XI];
+    int xref[XI];
+    uint32_t xbase[XI];
+#pragma unroll
+    for (int i = 0; i < XI; ++i) {
+      const int wi = tg + i * Cfg::XPG * 32, xl = wi & 31, kc = (wi >> 5) & 1;
+      const int tok = (wi >> 6) * 8 + (xl & 7), sub = xl >> 3;
+      act[i] = wi < Mt * 8 && x0 + tok < M;
+      const int64_t row = act[i] ? x0 + tok : 0;
+      xsrc[i] = X + row * K + (kc * 4 + sub) * 4;
+      xsc[i] = sX + row * nb;
+      xref[i] = act[i] ? sh.refB[tok] : 0;
+      xbase[i] = core_off(act[i] ? tok : 0, kc) + sub * 4;  // block b adds b Mt 32 bytes
+    }
+    auto load = [&](int i, uint32_t (&cw)[XI], int (&raw)[XI]) {
+      const int g = gx + i * NGX;
+#pragma unroll
+      for (int e = 0; e < XI; ++e) {
+        cw[e] = 0u;
+        raw[e] = 0;
+        if (act[e] && g < total) {
+          const int s = s0 + g;
+          cw[e] = __ldg(reinterpret_cast<const uint32_t*>(xsrc[e] + (int64_t)s * Cfg::KS));
+          raw[e] = (int)__ldg(xsc[e] + (s >> gshift));
+        }
+      }
+    };
+    const uint32_t bstride = (uint32_t)Mt * 32;  // bytes per column block
+    auto step = [&](const int g, const uint32_t (&cw)[XI], const int (&raw)[XI]) -> bool {
+      const int st = g % NSB;
+      if (g >= NSB) {
+        const bool ok = wait_all(&sh.empty[st], ((g / NSB) - 1) & 1);
+        if (!ok) {
+          if (lane == 0) raise_flag(status, CURVEFP_DEV_TIMEOUT);
+          sh.abort_flag = 1;
+          return false;
+        }
+      }
+      uint8_t* stg = xstage + (size_t)st * Cfg::BSTAGE;
+#pragma unroll
+      for (int e = 0; e < XI; ++e) {
+        if (!act[e]) continue;
+        uint32_t v[1], vc[1], mk[1][4];
+        PlaneFmt<FX>::template decode<PLANE_E5M2, 1>(make_uint4(cw[e], 0u, 0u, 0u), raw[e] - xref[e] - Cfg::PBX, v,
+                                                     vc, mk, true);
+        uint32_t pv[8], pc[8];
+        PlaneFmt<FX>::planes(v[0], mk[0], pv);
+        PlaneFmt<FX>::planes(vc[0], mk[0], pc);
+        // lattice position u holds plane u / WX where WX divides u
+#pragma unroll
+        for (int u = 0; u < L; u += Cfg::WX) {
+          *reinterpret_cast<uint32_t*>(stg + xbase[e] + u * bstride) = pc[u / Cfg::WX];
+          *reinterpret_cast<uint32_t*>(stg + xbase[e] + (L + u) * bstride) = pv[u / Cfg::WX];
+        }
+      }
+      tc::fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&sh.full[st]);
+      return true;
+    };
+    const int nown = (total - gx + NGX - 1) / NGX;
+    uint32_t q[PF][XI];
+    int rq[PF][XI];
+#pragma unroll
+    for (int u = 0; u < PF; ++u) load(u, q[u], rq[u]);
+    bool run = true;
+    for (int i = 0; i < nown && run; i += PF) {
+#pragma unroll
+      for (int u = 0; u < PF; ++u) {
+        if (i + u >= nown || !step(gx + (i + u) * NGX, q[u], rq[u])) {
+          run = false;
+          break;
+        }
+        load(i + u + PF, q[u], rq[u]);
       }
     }
   } else {
     // ------------------------------ MMA issuer -------------------------------
     const uint32_t leader = tc::elect_one();
     const uint64_t bdesc0 = tc::smem_desc(tc::smem_u32(xstage), 128, 256);
-    const uint32_t idesc = tc::idesc_bf16_f32(Cfg::BM, L * Mt);  // E5M2 x E5M2 -> F32, N = L Mt
-    const int gbytes = (Mt >> 3) * 256;                          // bytes of one column block
+    const uint32_t idesc = tc::idesc_bf16_f32(Cfg::BM, NP);  // E5M2 x E5M2 -> F32, N = L Mt
+    const int gbytes = Mt * 32;                                   // bytes of one column block
     bool ok = true;
     for (int g = 0; g < total && ok; ++g) {
       const int st = g % NSB;
-      ok = __all_sync(0xffffffffu, tc::mbar_wait(&sh.full[st], (g / NSB) & 1));
+      ok = wait_all(&sh.full[st], (g / NSB) & 1);
       if ((g & 7) == 0) ok = ok && !read_abort(&sh.abort_flag);
       if (!ok) break;
       tc::fence_after_sync();
@@ -301,7 +443,8 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
         // weight plane k_w against the window of column blocks from L - k_w WW
         const uint32_t a_t = tmem + Cfg::ACOL0 + st * Cfg::AU_COLS + kw * 8;
         const uint32_t boff = (uint32_t)(st * Cfg::BSTAGE + (L - kw * Cfg::WW) * gbytes);
-        tc::mma_f8_ts_if(leader, tmem, a_t, bdesc0 + (uint64_t)(boff >> 4), idesc, (g == 0 && kw == 0) ? 0u : 1u);
+        const uint32_t d_t = tmem + (uint32_t)((kw & (nacc - 1)) * NP);
+        tc::mma_f8_ts_if(leader, d_t, a_t, bdesc0 + (uint64_t)(boff >> 4), idesc, (g == 0 && kw < nacc) ? 0u : 1u);
       }
       tc::mma_commit_if(leader, &sh.empty[st]);
       if (g == total - 1) tc::mma_commit_if(leader, &sh.acc_full);

@@ -342,8 +342,8 @@ def test_skinny_within_tolerance(torch, fa, fb, M):
 @pytest.mark.parametrize("M", [1, 8])
 def test_skinny_ffn_full_size_sampled(torch, M):
     """The decode shapes of the FFN sweep (E3C3, W[14336 x 4096]) through
-    SKINNY: 256 sampled columns against the oracle; AUTO (SKINNY up to M = 4,
-    else TENSOR) equal to the kernel it picks, bit for bit."""
+    SKINNY: 256 sampled columns against the oracle; AUTO (SKINNY for M = 1,
+    TENSOR_NARROW up to M = 96) equal to the kernel it picks, bit for bit."""
     import paper_2608_10010_gb300 as cfp
 
     G = 32
@@ -352,7 +352,7 @@ def test_skinny_ffn_full_size_sampled(torch, M):
     b, sb = cfp.quantize(Wf, "E3C3", G, 1)
     c = cfp.gemm(a, sa, b, sb, "E3C3", "E3C3", G, "skinny")
     c2 = cfp.gemm(a, sa, b, sb, "E3C3", "E3C3", G, "auto")
-    c3 = cfp.gemm(a, sa, b, sb, "E3C3", "E3C3", G, "skinny" if M <= 4 else "tensor")
+    c3 = cfp.gemm(a, sa, b, sb, "E3C3", "E3C3", G, "skinny" if M <= 1 else "tensor_narrow")
     torch.cuda.synchronize()
     assert torch.equal(c2.view(torch.int32), c3.view(torch.int32))
     jj = np.sort(np.random.default_rng(3).choice(b.shape[0], 256, replace=False))
