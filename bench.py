@@ -38,11 +38,15 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 M, N, K, G = 2048, 4096, 4096, 32
-# DRAM bytes (read + written) of one launch of the tensor-core GEMM at this
-# size, from an ncu capture (dram__bytes_read.sum + dram__bytes_write.sum) of
-# the kernel as it stands; set to None whenever the kernel changes until it is
-# captured again.
-GEMM_DRAM_TRAFFIC = 29_904_640 + 214_016
+# The step's GEMM: the tensor-core kernel with the phases along the MMA's N
+# dimension and 2:4-sparse pair planes (TENSOR_NARROW; 0.86 ms against the
+# 128 x 96 tile kernel's 1.08 ms at this size).
+GEMM_ALGO = "tensor_narrow"
+# DRAM bytes (read + written) of one launch of that GEMM at this size, from an
+# ncu capture (dram__bytes_read.sum + dram__bytes_write.sum) of the kernel as
+# it stands; set to None whenever the kernel changes until it is captured
+# again.
+GEMM_DRAM_TRAFFIC = 27_204_352 + 1_212_160
 FMT = "E3C3"
 WORKLOAD = "E3C3 Llama-7B-like linear: X[2048x4096] (1% outlier channels x20) . W[4096x4096]^T, block 32"
 METRIC = "CurveFP GEMM TOPS & quantize GB/s at 1 GB300, as % of roofline"
@@ -179,7 +183,9 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
         r = {"case": name, "algo": algo, "M": Mx, "N": Nx, "K": Kx, "formats": f"{fa}x{fb}", "ms": round(ms, 4),
              "tops": round(tops, 3)}
         if algo in ("tensor", "tensor_narrow"):
-            r["tensor_work_frac"] = round(tops * planes / fp8_peak, 4)
+            # the narrow kernel's same-format pairs use 2:4-sparse pair planes: half the MMA work
+            issued = planes // 2 if algo == "tensor_narrow" and fa == fb else planes
+            r["tensor_work_frac"] = round(tops * issued / fp8_peak, 4)
         if hbm_bound:
             wbytes = Nx * Kx + Nx * Kx // G
             r["weight_code_gbs"] = round(wbytes / (ms / 1e3) / 1e9, 1)
@@ -252,6 +258,7 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
     # training triplet, E4C3 weights/activations, E5C2 gradients
     X, Wt, dY = inputs.training_triplet_cuda()
     gemm_case("fwd X.W", q(X, "E4C3", 0), "E4C3", q(Wt, "E4C3", 1), "E4C3", 64)
+    gemm_case("fwd X.W narrow", q(X, "E4C3", 0), "E4C3", q(Wt, "E4C3", 1), "E4C3", 64, algo="tensor_narrow")
     gemm_case("dgrad dY.W^T", q(dY, "E5C2", 0), "E5C2", q(Wt, "E4C3", 0), "E4C3", 32)
     gemm_case("wgrad dY^T.X", q(dY, "E5C2", 1), "E5C2", q(X, "E4C3", 1), "E4C3", 32)
     # the same triplet on operands quantized once and reused (the backward
@@ -280,9 +287,9 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
             Xf, Wf = inputs.ffn_cuda(Mf, Kf)
             gemm_case(f"ffn M={Mf} K={Kf}", q(Xf, "E3C3", 0), "E3C3", q(Wf, "E3C3", 1), "E3C3", 64,
                       hbm_bound=Mf <= 128)
-            if Mf <= 128:  # few activation rows: phases along the MMA's N dimension
-                gemm_case(f"ffn M={Mf} K={Kf} narrow", q(Xf, "E3C3", 0), "E3C3", q(Wf, "E3C3", 1), "E3C3", 64,
-                          hbm_bound=True, algo="tensor_narrow")
+            # phases along the MMA's N dimension, 2:4-sparse pair planes
+            gemm_case(f"ffn M={Mf} K={Kf} narrow", q(Xf, "E3C3", 0), "E3C3", q(Wf, "E3C3", 1), "E3C3", 64,
+                      hbm_bound=Mf <= 128, algo="tensor_narrow")
             if Mf <= 8:  # decode sizes: the CUDA-core kernel as well
                 gemm_case(f"ffn M={Mf} K={Kf} skinny", q(Xf, "E3C3", 0), "E3C3", q(Wf, "E3C3", 1), "E3C3", 64,
                           hbm_bound=True, algo="skinny")
@@ -353,7 +360,7 @@ def run_ours(args):
         stream.wait_event(sync["wq"])
         if record:
             ev["g0"].record(stream)
-        cfp.gemm(a, sa, b, sb, FMT, FMT, G, "tensor", out=Cout, status=status, stream=stream)
+        cfp.gemm(a, sa, b, sb, FMT, FMT, G, GEMM_ALGO, out=Cout, status=status, stream=stream)
         if record:
             ev["g1"].record(stream)
         aux.wait_event(sync["xq"])
@@ -425,7 +432,9 @@ def run_ours(args):
         "quant_x": _time_ms(torch, stream, lambda: cfp.quantize(Xd, FMT, G, 0, codes=a, scales=sa, stream=stream),
                             flush_l2),
         "dequant": _time_ms(torch, stream, lambda: cfp.dequantize(a, sa, FMT, G, out=Xh, stream=stream), flush_l2)}
-    planes = 8 * 8  # curve-plane pairs per scale block (E3C3 x E3C3)
+    # dense-equivalent FP8 MACs the kernel issues per useful MAC: 4 pair-plane
+    # MMAs (logical K 64, the cost of a dense K 32) x 8 phase columns per token
+    planes = 4 * 8
     fp8_peak = 2.0 * bf16  # E5M2 planes: measured BF16 burst x the nominal FP8/BF16 ratio (2)
 
     # quantizer at the largest size of the bandwidth sweep: 2^30 BF16 elements,
@@ -559,7 +568,7 @@ def run_ours(args):
         "dtype": "fp8",
         "data": "synthetic (seeded; stands in for real LLM weights/activations)",
         "config": {"workload": WORKLOAD, "M": M, "N": N, "K": K, "block": G, "format": FMT,
-                   "input": "fp32", "gemm_kernel": "tensor (tcgen05 phase planes)",
+                   "input": "fp32", "gemm_kernel": "tensor_narrow (tcgen05 2:4-sparse pair planes, phases along N)",
                    "l2": "flushed between steps (256 MiB write + 256 MiB read, outside the per-step events)",
                    "schedule": "two streams: quantize W || quantize X, then GEMM || dequantize X",
                    "parallelism": f"replicas x{ws}"},
@@ -567,11 +576,12 @@ def run_ours(args):
                      "unit": "TFLOP/s", "frac": round(gemm_tops / fp8_peak, 6), "traffic": GEMM_DRAM_TRAFFIC,
                      "bytes_algorithmic": M * K + N * K + (M + N) * K // G + 4 * M * N,
                      "peak_source": f"FP8 dense = 2 x bf16 burst ({bf16} TFLOP/s, {peak_src})",
-                     "kernel": "gemm_tc_kernel (tcgen05 kind::f8f6f4, E5M2 curve planes)",
+                     "kernel": "gemm_tcn_kernel (tcgen05.mma.sp kind::f8f6f4, E5M2 pair planes, phases along N)",
                      "tensor_work_frac": round(gemm_tops * planes / fp8_peak, 4),
                      "note": f"achieved counts algorithmic closed-product ops (2 per MAC); the kernel issues "
-                             f"{planes} FP8 MACs per useful MAC (one per curve-plane pair), so the tensor-pipe "
-                             f"work is tensor_work_frac of peak"},
+                             f"{planes} dense-equivalent FP8 MACs per useful MAC (4 sparse pair-plane MMAs of "
+                             f"logical K 64 per 32 codes, 8 phase columns per token), so the tensor-pipe work "
+                             f"is tensor_work_frac of peak"},
         "kernels_ms": {k: round(v, 4) for k, v in mean.items()},
         "quantize": {"gbs_w": round(q_gbs_w, 1), "gbs_x": round(q_gbs_x, 1), "frac_w": round(q_gbs_w / hbm, 4),
                      "frac_x": round(q_gbs_x / hbm, 4), "peak_gbs": hbm, "bytes_per_elem": 4 + 1 + 1 / G,
@@ -661,7 +671,7 @@ def run_reference(args):
 
 def run_only(args):
     """One kernel of the path, a few launches, no timing: the target of the
-    ncu captures (--only gemm: the tensor-core GEMM of the workload above;
+    ncu captures (--only gemm: the step's GEMM (GEMM_ALGO) of the workload above;
     --only quantize: 2^28 BF16 elements, E4C3, block 32; skinny, narrow,
     reuse, r89: the decode GEMM, the few-row tensor-core GEMM, the
     reused-operand dgrad and the r = 2^{8/9} GEMM)."""
@@ -677,7 +687,7 @@ def run_only(args):
         a, sa = cfp.quantize(torch.from_numpy(X).to(dev), FMT, G, 0)
         b, sb = cfp.quantize(torch.from_numpy(W).to(dev), FMT, G, 0)
         for _ in range(args.steps):
-            c = cfp.gemm(a, sa, b, sb, FMT, FMT, G, "tensor")
+            c = cfp.gemm(a, sa, b, sb, FMT, FMT, G, GEMM_ALGO)
         torch.cuda.synchronize()
         print(json.dumps({"only": "gemm", "launches": args.steps, "c00": float(c[0, 0])}))
     elif args.only == "quantize":

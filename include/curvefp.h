@@ -87,14 +87,18 @@ typedef enum {
  * CURVEFP_SKINNY_MAX_M) on the CUDA cores with the same FP32 per-phase
  * accumulation, every product formed from the two codes (the tensor-core
  * tile costs the same for any M up to 128).  TENSOR_NARROW: the tensor-core
- * method for few activation rows (Sec. 3.2, Eq. 2, Eq. 5): the weight rows
- * are the 128-row operand and the L phases of every token run along the
- * MMA's N dimension, so a step of 32 codes takes K_b MMAs of 128 x (L Mt)
- * (Mt <= 256/L tokens per CTA) instead of K_a K_b MMAs of a 128-row tile.
- * AUTO (measured crossovers on the FFN decode shapes, N = 14336, K = 4096):
- * SKINNY for M <= CURVEFP_AUTO_SKINNY_M; TENSOR_NARROW for M <=
- * CURVEFP_AUTO_NARROW_M where the format pair has it; TENSOR above; SKINNY up
- * to CURVEFP_SKINNY_MAX_M for pairs without a tensor-core kernel. */
+ * method with the weight rows (B) as the 128-row operand and the L phases of
+ * every token (row of A) along the MMA's N dimension (Sec. 3.2, Eq. 2,
+ * Eq. 5): a step of 32 codes takes K_b MMAs of 128 x (L Mt) (Mt <= 256/L
+ * tokens per CTA), and for same-format pairs K_b/2 2:4-sparse MMAs (weight
+ * planes j and j + K_b/2 share one compressed operand), against K_a K_b MMAs
+ * of a 128-row tile; the fastest tensor-core kernel at every M for
+ * same-format pairs.
+ * AUTO (measured on the FFN shapes, N = 14336, K = 4096, and the
+ * 2048 x 4096 x 4096 linear): SKINNY for M <= CURVEFP_AUTO_SKINNY_M;
+ * TENSOR_NARROW for same-format pairs, and for the mixed pairs up to
+ * CURVEFP_AUTO_NARROW_M; TENSOR above; SKINNY up to CURVEFP_SKINNY_MAX_M for
+ * pairs without a tensor-core kernel. */
 typedef enum {
   CURVEFP_GEMM_EXACT = 0,
   CURVEFP_GEMM_TENSOR = 1,

@@ -53,9 +53,21 @@ struct TcnCfg {
   static constexpr int MTMAX = 256 / L;   // tokens per CTA: L Mt <= 256 (MMA N)
   static constexpr int NBLK = 2 * L;      // column blocks of the doubled sequence
   static constexpr int NSB = 4;           // pipeline depth (X stages = W TMEM units)
-  static constexpr int AU_COLS = KW * 8;  // TMEM columns of one step's W planes
+  // Same-format pairs use 2:4-sparse pair planes: weight planes j and j + HB
+  // share one compressed operand (an element sits in one plane), at logical
+  // positions 2k and 2k + 1, with the curve-index bit MBIT as metadata.
+  static constexpr bool SP = FX == FW;
+  static constexpr int HB = KW / 2, MBIT = KW == 8 ? 2 : 1;
+  static constexpr int NJ = SP ? HB : KW;  // A operands (MMAs) per step
+  static constexpr int AU_COLS = NJ * 8;  // TMEM columns of one step's W planes
   static constexpr int ACOL0 = 256;       // W units after the accumulator
-  static_assert(ACOL0 + NSB * AU_COLS <= 512, "TMEM budget");
+  static constexpr int MCOL0 = ACOL0 + NSB * AU_COLS;  // metadata of unit u at MCOL0 + 8 u (2 used)
+  static_assert(MCOL0 + (SP ? NSB * 8 : 0) <= 512, "TMEM budget");
+  // sparse form: R blocks RB0 .. 2L-1 of 64-byte rows, R_b[2k] = Q_b[k],
+  // R_b[2k + 1] = Q_{b - HB}[k]; the operand of pair j is the window of L
+  // blocks from block L - j
+  static constexpr int RB0 = L - HB + 1, NRB = L + HB - 1;
+  static constexpr int ROWB = SP ? 64 : 32;  // bytes of one operand row
   static_assert(L % 4 == 0 && KW % 2 == 0, "epilogue phase groups, plane pairs");
   // Producer groups take turns: W group g % NGW and X group g % NGX produce
   // step g, so each producer thread has NGW (NGX) steps of time per step.
@@ -66,7 +78,7 @@ struct TcnCfg {
   static constexpr int NXT = NGX * XPG * 32;    // X threads
   static constexpr int THREADS = NWT + NXT + 32;
   static constexpr int MMA_WARP = (NWT + NXT) / 32;
-  static constexpr int BSTAGE = NBLK * MTMAX * 32;  // bytes of one step's X planes
+  static constexpr int BSTAGE = (SP ? NRB : NBLK) * MTMAX * ROWB;  // bytes of one step's X operand rows
   static constexpr int PBX = FX == CURVEFP_E5C2 ? 1 : 0;  // plane exponent bias
   static constexpr int PBW = FW == CURVEFP_E5C2 ? 1 : 0;
   static constexpr int PFW = 4;  // own steps of weight codes in flight per W thread
@@ -101,6 +113,36 @@ __device__ __forceinline__ int row_ref(const int8_t* s, int nb) {
     for (int b = 0; b < nb; ++b) ref = max(ref, (int)__ldg(s + b));
   }
   return ref;
+}
+
+// Metadata word of 16 codes (four code words) of a 2:4 operand with 8-bit
+// elements: per chunk of two elements, position bit(2c) and 2 + bit(2c + 1),
+// where bit is the curve-index bit MBIT that selects the partner plane.
+template <int MBIT>
+__device__ __forceinline__ uint32_t pair_meta(uint32_t w0, uint32_t w1, uint32_t w2, uint32_t w3) {
+  const uint32_t w[4] = {w0, w1, w2, w3};
+  uint32_t m = 0;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const uint32_t t = (w[q] >> MBIT) & 0x01010101u;  // bit of element i at 8 i
+    m |= (((t * 0x01041040u) >> 24) | 0x88u) << (8 * q);  // ... at 2 i, plus bit 3 of each nibble
+  }
+  return m;
+}
+
+// 2:4-sparse MMA (kind::f8f6f4), A and metadata in TMEM, issued by `leader`.
+__device__ __forceinline__ void mma_sp_if(uint32_t leader, uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                          uint32_t meta_tmem, uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.b32 p, %5, 0;\n setp.ne.b32 q, %6, 0;\n"
+      "@q tcgen05.mma.sp.cta_group::1.kind::f8f6f4 [%0], [%1], %2, [%3], %4, p;\n}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(meta_tmem), "r"(idesc), "r"(accumulate), "r"(leader)
+      : "memory");
+}
+
+// Interleave two words (elements 4q..4q+3 each) into X0 Y0 X1 Y1 | X2 Y2 X3 Y3.
+__device__ __forceinline__ uint2 interleave2(uint32_t x, uint32_t y) {
+  return make_uint2(__byte_perm(x, y, 0x5140), __byte_perm(x, y, 0x7362));
 }
 
 __device__ __forceinline__ bool wait_all(uint64_t* bar, uint32_t parity) {
@@ -151,7 +193,8 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
   // for each other's accumulation, so where the accumulator is at most 128
   // columns the weight planes rotate over 2 or 4 copies (NP columns each)
   // that the epilogue adds up.
-  const int NP = L * Mt, nacc = NP <= 64 ? 4 : (NP <= 128 ? 2 : 1);
+  const int NP = L * Mt, nacc0 = NP <= 64 ? 4 : (NP <= 128 ? 2 : 1);
+  const int nacc = nacc0 < Cfg::NJ ? nacc0 : Cfg::NJ;  // every copy receives an MMA each step
 
   if (tid == 0) {
     for (int s = 0; s < NSB; ++s) {
@@ -251,17 +294,31 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
           return false;
         }
       }
-      // planes 2jp and 2jp + 1: 16 consecutive columns of the unit
+      // operands 2jp and 2jp + 1 of the step: 16 consecutive columns of the
+      // unit.  Dense: plane j.  Sparse: pair plane j = the elements whose
+      // curve index is j or j + HB (low bits of k equal to j), plus the
+      // metadata words of codes 0-15 and 16-31.
 #pragma unroll
-      for (int jp = 0; jp < Cfg::KW / 2; ++jp) {
+      for (int jp = 0; jp < Cfg::NJ / 2; ++jp) {
         uint32_t r[16];
 #pragma unroll
         for (int e = 0; e < 2; ++e) {
           const int j = 2 * jp + e;
 #pragma unroll
-          for (int w = 0; w < 8; ++w) r[e * 8 + w] = p[w][j & 3] & ((j & 4) ? m2[w] : ~m2[w]);
+          for (int w = 0; w < 8; ++w) {
+            if constexpr (!Cfg::SP)
+              r[e * 8 + w] = p[w][j & 3] & ((j & 4) ? m2[w] : ~m2[w]);
+            else if constexpr (Cfg::KW == 8)
+              r[e * 8 + w] = p[w][j];
+            else
+              r[e * 8 + w] = p[w][j] | p[w][j + 2];
+          }
         }
         tmem_st16(lane_base + Cfg::ACOL0 + st * Cfg::AU_COLS + jp * 16, r);
+      }
+      if constexpr (Cfg::SP) {
+        const uint32_t mt[2] = {pair_meta<Cfg::MBIT>(lo.x, lo.y, lo.z, lo.w), pair_meta<Cfg::MBIT>(hi.x, hi.y, hi.z, hi.w)};
+        tc::tmem_st2(lane_base + Cfg::MCOL0 + st * 8, mt);
       }
       pend = st;
       return true;
@@ -361,7 +418,11 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
       xsrc[i] = X + row * K + (kc * 4 + sub) * 4;
       xsc[i] = sX + row * nb;
       xref[i] = act[i] ? sh.refB[tok] : 0;
-      xbase[i] = core_off(act[i] ? tok : 0, kc) + sub * 4;  // block b adds b Mt 32 bytes
+      // dense: word sub of 16-byte chunk kc of a 32-byte row; sparse: the
+      // word's 8 interleaved bytes in 16-byte chunk j >> 1 of a 64-byte row
+      const int j = kc * 4 + sub, t0 = act[i] ? tok : 0;
+      xbase[i] = Cfg::SP ? (uint32_t)((t0 >> 3) * 512 + (j >> 1) * 128 + (t0 & 7) * 16 + (j & 1) * 8)
+                         : core_off(t0, kc) + sub * 4;  // block b adds b Mt ROWB bytes
     }
     auto load = [&](int i, uint32_t (&cw)[XI], int (&raw)[XI]) {
       const int g = gx + i * NGX;
@@ -376,7 +437,7 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
         }
       }
     };
-    const uint32_t bstride = (uint32_t)Mt * 32;  // bytes per column block
+    const uint32_t bstride = (uint32_t)Mt * Cfg::ROWB;  // bytes per column block
     auto step = [&](const int g, const uint32_t (&cw)[XI], const int (&raw)[XI]) -> bool {
       const int st = g % NSB;
       if (g >= NSB) {
@@ -397,11 +458,22 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
         uint32_t pv[8], pc[8];
         PlaneFmt<FX>::planes(v[0], mk[0], pv);
         PlaneFmt<FX>::planes(vc[0], mk[0], pc);
-        // lattice position u holds plane u / WX where WX divides u
+        if constexpr (Cfg::SP) {
+          // R block b interleaves Q block b (plane partner) with Q block b - HB;
+          // Q block u < L is the carry copy of plane u, u >= L plane u - L
 #pragma unroll
-        for (int u = 0; u < L; u += Cfg::WX) {
-          *reinterpret_cast<uint32_t*>(stg + xbase[e] + u * bstride) = pc[u / Cfg::WX];
-          *reinterpret_cast<uint32_t*>(stg + xbase[e] + (L + u) * bstride) = pv[u / Cfg::WX];
+          for (int b = Cfg::RB0; b < 2 * L; ++b) {
+            const uint32_t x = b < L ? pc[b] : pv[b - L];
+            const uint32_t y = b - Cfg::HB < L ? pc[b - Cfg::HB] : pv[b - Cfg::HB - L];
+            *reinterpret_cast<uint2*>(stg + xbase[e] + (b - Cfg::RB0) * bstride) = interleave2(x, y);
+          }
+        } else {
+          // lattice position u holds plane u / WX where WX divides u
+#pragma unroll
+          for (int u = 0; u < L; u += Cfg::WX) {
+            *reinterpret_cast<uint32_t*>(stg + xbase[e] + u * bstride) = pc[u / Cfg::WX];
+            *reinterpret_cast<uint32_t*>(stg + xbase[e] + (L + u) * bstride) = pv[u / Cfg::WX];
+          }
         }
       }
       tc::fence_proxy_async_smem();
@@ -428,9 +500,10 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
   } else {
     // ------------------------------ MMA issuer -------------------------------
     const uint32_t leader = tc::elect_one();
-    const uint64_t bdesc0 = tc::smem_desc(tc::smem_u32(xstage), 128, 256);
-    const uint32_t idesc = tc::idesc_bf16_f32(Cfg::BM, NP);  // E5M2 x E5M2 -> F32, N = L Mt
-    const int gbytes = Mt * 32;                                   // bytes of one column block
+    const uint64_t bdesc0 = tc::smem_desc(tc::smem_u32(xstage), 128, Cfg::SP ? 512 : 256);
+    // E5M2 x E5M2 -> F32, N = L Mt (bit 2: 2:4-sparse A)
+    const uint32_t idesc = tc::idesc_bf16_f32(Cfg::BM, NP) | (Cfg::SP ? (1u << 2) : 0u);
+    const int gbytes = Mt * Cfg::ROWB;  // bytes of one column block
     bool ok = true;
     for (int g = 0; g < total && ok; ++g) {
       const int st = g % NSB;
@@ -439,12 +512,17 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
       if (!ok) break;
       tc::fence_after_sync();
 #pragma unroll
-      for (int kw = 0; kw < Cfg::KW; ++kw) {
-        // weight plane k_w against the window of column blocks from L - k_w WW
+      for (int kw = 0; kw < Cfg::NJ; ++kw) {
+        // weight plane (pair plane) k_w against the window of column blocks
+        // from L - k_w WW (R block L - k_w)
         const uint32_t a_t = tmem + Cfg::ACOL0 + st * Cfg::AU_COLS + kw * 8;
-        const uint32_t boff = (uint32_t)(st * Cfg::BSTAGE + (L - kw * Cfg::WW) * gbytes);
+        const uint32_t boff = (uint32_t)(st * Cfg::BSTAGE + (Cfg::SP ? L - kw - Cfg::RB0 : L - kw * Cfg::WW) * gbytes);
         const uint32_t d_t = tmem + (uint32_t)((kw & (nacc - 1)) * NP);
-        tc::mma_f8_ts_if(leader, d_t, a_t, bdesc0 + (uint64_t)(boff >> 4), idesc, (g == 0 && kw < nacc) ? 0u : 1u);
+        const uint32_t acc = (g == 0 && kw < nacc) ? 0u : 1u;
+        if constexpr (Cfg::SP)
+          mma_sp_if(leader, d_t, a_t, bdesc0 + (uint64_t)(boff >> 4), tmem + Cfg::MCOL0 + st * 8, idesc, acc);
+        else
+          tc::mma_f8_ts_if(leader, d_t, a_t, bdesc0 + (uint64_t)(boff >> 4), idesc, acc);
       }
       tc::mma_commit_if(leader, &sh.empty[st]);
       if (g == total - 1) tc::mma_commit_if(leader, &sh.acc_full);

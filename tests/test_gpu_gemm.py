@@ -255,13 +255,15 @@ def test_llama7b_linear_full_size(torch):
     check_exact(torch, ra, rsa, rb, rsb, "E3C3", "E3C3", 32, rows=rows)
     check_tensor(torch, ra, rsa, rb, rsb, "E3C3", "E3C3", 32, rows=rows)
     check_tensor(torch, ra, rsa, rb, rsb, "E3C3", "E3C3", 32, rows=rows, algo="tensor_sparse")
+    # the benchmark's GEMM: phases along N, 2:4-sparse pair planes (64 token groups x 32 weight tiles)
+    check_tensor(torch, ra, rsa, rb, rsb, "E3C3", "E3C3", 32, rows=rows, algo="tensor_narrow")
 
 
 @pytest.mark.parametrize("which", ["fwd", "dgrad", "wgrad"])
 def test_training_triplet_full_size(torch, which):
     """CurveFP8 training GEMMs (E4C3 X, W; E5C2 dY = 1e-3 t_3), each operand
-    quantized along its own GEMM's reduction axis; tensor kernel on the full
-    problem, parity on sampled rows."""
+    quantized along its own GEMM's reduction axis; the tile and the narrow
+    tensor-core kernels on the full problem, parity on sampled rows."""
     X, W, dY = inputs.training_triplet()
     if which == "fwd":  # Y = X W: M = tokens, N = out, K = in
         a, sa = quantized(X, "E4C3", 32, 0)
@@ -276,6 +278,7 @@ def test_training_triplet_full_size(torch, which):
         b, sb = quantized(X, "E4C3", 32, 1)
         fa, fb = "E5C2", "E4C3"
     check_tensor(torch, a, sa, b, sb, fa, fb, 32, rows=_sample(a.shape[0], 1))
+    check_tensor(torch, a, sa, b, sb, fa, fb, 32, rows=_sample(a.shape[0], 1), algo="tensor_narrow")
 
 
 @pytest.mark.parametrize("M", [1, 16, 128])
