@@ -64,6 +64,19 @@ def test_random_codes_within_tolerance(torch, fa, fb, M):
     check(torch, a, sa, b, sb, fa, fb, 32)
 
 
+@pytest.mark.parametrize("fa,fb", [("E3C3", "E3C3"), ("E4C3", "E4C3"), ("E5C2", "E5C2"), ("E5C2", "E4C3")])
+@pytest.mark.parametrize("M", [512, 601])
+def test_two_token_groups_per_cta(torch, fa, fb, M):
+    """From 512 rows the same-format pairs take two token groups per CTA
+    (accumulators side by side): M = 601 leaves a last CTA whose second group
+    is partly padding; N = 260 a ragged weight tile; the mixed pair keeps one
+    group and checks the same sizes."""
+    rng = np.random.default_rng(M)
+    a, sa = rand_operand(rng, fa, M, 256, 32)
+    b, sb = rand_operand(rng, fb, 260, 256, 32)
+    check(torch, a, sa, b, sb, fa, fb, 32)
+
+
 @pytest.mark.parametrize("fa,fb", [("E3C3", "E3C3"), ("E5C2", "E4C3")])
 @pytest.mark.parametrize("G", [64, 128, 512])
 def test_larger_blocks(torch, fa, fb, G):
