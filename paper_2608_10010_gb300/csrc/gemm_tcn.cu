@@ -1,5 +1,5 @@
-// Tensor-core closed-product GEMM for few activation rows (algo
-// TENSOR_NARROW): the phases of Eq. 5 run along the MMA's N dimension.
+// Tensor-core closed-product GEMM with the phases along the MMA's N dimension
+// (algo TENSOR_NARROW): Sec. 3.2, Eq. 2, Eq. 5.
 //
 // C = X_hat W_hat^T with X the M activation rows (the API's A operand, format
 // FX) and W the N weight rows (the API's B operand, format FW).  As in the
@@ -9,35 +9,48 @@
 // c = floor((k_x WX + k_w WW) / L) (Eq. 2 on the shared lattice L).
 //
 // Here the weight rows are the MMA's 128-row TMEM operand and the phase is a
-// column index: the accumulator of a CTA is D[w][h Mt + m] (weight row w,
-// phase h, token m of the CTA's Mt tokens), the per-phase sums S_h of Eq. 5
-// for every token side by side.  For weight plane k_w the shared-memory
-// operand must hold, in column block h, the X plane with k_x WX =
-// (h - k_w WW) mod L, doubled where the sum wrapped (carry).  Lay out the
-// sequence of 2L column blocks
+// column index: the accumulator of a token group is D[w][h Mt + m] (weight
+// row w, phase h, token m of the group's Mt tokens), the per-phase sums S_h
+// of Eq. 5 for every token side by side.  For weight plane k_w the
+// shared-memory operand must hold, in column block h, the X plane with
+// k_x WX = (h - k_w WW) mod L, doubled where the sum wrapped (carry).  Lay
+// out the sequence of 2L column blocks
 //   Q = [ 2 X_0 ... (lattice positions 0 .. L-1, carry copies) |
 //           X_0 ... (lattice positions 0 .. L-1, plain) ]
 // (block u of each half holds the plane with k_x WX = u, zero where no plane
 // sits on u); then the operand of weight plane k_w is the window of L blocks
 // that starts at block L - k_w WW: its block h is plain for h >= k_w WW and
 // the carry copy of position L - k_w WW + h otherwise.  A window is a start
-// address of the MMA's shared-memory descriptor, so each pipeline step of 32
-// codes costs K_W MMAs of 128 x (L Mt) x 32 (8 for 8-curve weights) on 2L Mt
-// rows of staged X planes, against K_X K_W MMAs of the tile kernel, whose
-// 128-row activation tile is mostly empty when M is small.
+// address of the MMA's shared-memory descriptor, so a pipeline step of 32
+// codes costs K_W MMAs of 128 x (L Mt) x 32 on 2L Mt staged rows, against
+// K_X K_W MMAs of the tile kernel.
 //
-// Roles (8 + NXT/32 + 1 warps):
-//   warps 0-7   W producers, two threads per weight row (16 codes each per
-//               step): codes -> planes -> TMEM (as the tile kernel's A
-//               producers), prefetching PF steps ahead (the weights stream
-//               from HBM); after the last step they run the epilogue.
-//   next warps  X producers, two threads per token: codes -> plane and
-//               carry-plane words -> the 2L blocks of the step's stage.
+// Same-format pairs (WX = WW = 1) use 2:4-sparse pair planes: an element sits
+// in one plane, so weight planes j and j + K/2 share one compressed operand at
+// logical positions 2k and 2k + 1, with one curve-index bit as metadata; the
+// activation side stores R_b[2k] = Q_b[k], R_b[2k + 1] = Q_{b - K/2}[k] and
+// the operand of pair j is the window from R block L - j: K/2 sparse MMAs of
+// logical K 64 per step, half the MMAs and half the TMEM bytes.  From 512
+// activation rows a CTA takes two token groups (accumulators side by side,
+// a three-step ring), so each decoded weight step serves twice the tokens.
+//
+// Roles (15 warps for 8-phase pairs, 17 for E5C2 x E5C2; a step is short,
+// so producer groups take turns):
+//   warps 0-7   W producers: two groups of 4 warps taking alternate steps,
+//               one thread per weight row (all 32 codes of its steps): codes
+//               -> planes (pair planes and metadata) -> TMEM, prefetching
+//               PFW own steps ahead; after the last step they run the
+//               epilogue.
+//   next warps  X producers: groups taking every NGX-th step, one 4-code word
+//               of one token per work item -> the step's blocks (Q or R),
+//               conflict-free stores; padding tokens are never written (the
+//               stages start at zero).
 //   last warp   TMEM allocation and MMA issue (one elected lane).
-// With fewer weight tiles than SMs every tile is split in K into two pieces
-// (chosen by the same greedy-dispatch simulation as the tile kernel's tail);
-// a piece adds its outputs to zeroed C atomically, two additions per output,
-// so the result does not depend on their order.  Every wait is bounded.
+// With fewer weight tiles than fill the SMs' last wave, tiles are split in K
+// into two pieces (the tile kernel's greedy-dispatch simulation, extended to
+// grids smaller than the SM count); a piece adds its outputs to zeroed C
+// atomically, two additions per output, so the result does not depend on
+// their order.  Every wait is bounded.
 #include "gemm_tc.cuh"
 
 namespace cfp {
@@ -80,7 +93,7 @@ struct TcnCfg {
   // Producer groups take turns: W group g % NGW and X group g % NGX produce
   // step g, so each producer thread has NGW (NGX) steps of time per step.
   static constexpr int NGW = 2;                 // W groups of 4 warps (one thread per weight row)
-  static constexpr int XPG = MTMAX / 16;        // X warps per group (two threads per token)
+  static constexpr int XPG = MTMAX / 16;        // X warps per group
   static constexpr int NGX = L == 8 ? 3 : 2;    // X groups
   static constexpr int NWT = NGW * 128;         // W threads
   static constexpr int NXT = NGX * XPG * 32;    // X threads
