@@ -1,95 +1,90 @@
 // Tensor-core closed-product GEMM with the phases along the MMA's N dimension
 // (algo TENSOR_NARROW): Sec. 3.2, Eq. 2, Eq. 5.
 //
-// C = X_hat W_hat^T with X the M activation rows (the API's A operand, format
-// FX) and W the N weight rows (the API's B operand, format FW).  As in the
-// tile kernel, every operand splits into curve planes of exact powers of two
-// (plane k holds the elements of curve index k), and plane k_x of X times
-// plane k_w of W lands on phase h = (k_x WX + k_w WW) mod L with carry
-// c = floor((k_x WX + k_w WW) / L) (Eq. 2 on the shared lattice L).
+// C = X_hat W_hat^T with X the activation ("token") operand, format FX, and
+// W the weight operand, format FW.  Every operand splits into curve planes of
+// exact powers of two (plane k holds the elements of curve index k), and
+// plane k_x of X times plane k_w of W lands on phase h = (k_x WX + k_w WW)
+// mod L with carry c = floor((k_x WX + k_w WW) / L) (Eq. 2 on the shared
+// lattice L).
+//
+// Block scales.  A plane value is the power of two 2^e of the code alone
+// (tc_mx.cuh); the block scale of every 32-code step enters the MMA as a
+// UE8M0 scale factor (tcgen05.mma .kind::mxf8f6f4 .block_scale), relative to
+// the row's largest block scale, so every product of the step is exact
+// whatever the spread of the block scales along the row.
 //
 // Here the weight rows are the MMA's 128-row TMEM operand and the phase is a
-// column index: the accumulator of a token group is D[w][h Mt + m] (weight
-// row w, phase h, token m of the group's Mt tokens), the per-phase sums S_h
-// of Eq. 5 for every token side by side.  For weight plane k_w the
-// shared-memory operand must hold, in column block h, the X plane with
+// column index: the accumulator of a tile is D[w][h Mt + m] (weight row w,
+// phase h, token m of the tile's Mt tokens), the per-phase sums S_h of Eq. 5
+// for every token side by side.  For weight plane k_w the shared-memory
+// operand must hold, in column block h, the X plane with
 // k_x WX = (h - k_w WW) mod L, doubled where the sum wrapped (carry).  Lay
 // out the sequence of 2L column blocks
 //   Q = [ 2 X_0 ... (lattice positions 0 .. L-1, carry copies) |
 //           X_0 ... (lattice positions 0 .. L-1, plain) ]
-// (block u of each half holds the plane with k_x WX = u, zero where no plane
-// sits on u); then the operand of weight plane k_w is the window of L blocks
-// that starts at block L - k_w WW: its block h is plain for h >= k_w WW and
-// the carry copy of position L - k_w WW + h otherwise.  A window is a start
-// address of the MMA's shared-memory descriptor, so a pipeline step of 32
-// codes costs K_W MMAs of 128 x (L Mt) x 32 on 2L Mt staged rows, against
-// K_X K_W MMAs of the tile kernel.
+// then the operand of weight plane k_w is the window of L blocks that starts
+// at block L - k_w WW: a start address of the MMA's shared-memory descriptor.
 //
-// Same-format pairs (WX = WW = 1) use 2:4-sparse pair planes: an element sits
-// in one plane, so weight planes j and j + K/2 share one compressed operand at
-// logical positions 2k and 2k + 1, with one curve-index bit as metadata; the
-// activation side stores R_b[2k] = Q_b[k], R_b[2k + 1] = Q_{b - K/2}[k] and
-// the operand of pair j is the window from R block L - j: K/2 sparse MMAs of
-// logical K 64 per step, half the MMAs and half the TMEM bytes.  From 512
-// activation rows a CTA takes two token groups (accumulators side by side,
-// a three-step ring), so each decoded weight step serves twice the tokens.
+// 2:4-sparse pair planes: an element sits in one plane, so weight planes j
+// and j + K_W/2 share one compressed operand at logical positions 2k and
+// 2k + 1, with one curve-index bit as metadata.  The activation side stores
+// R blocks R_b[2k] = Q_b[k], R_b[2k + 1] = Q_{b - PO}[k] (PO = K_W/2 WW, the
+// lattice distance of the partner plane) and the operand of pair j is the
+// window from R block L - j WW: K_W/2 sparse MMAs of logical K 64 per step.
 //
-// Roles (15 warps for 8-phase pairs, 17 for E5C2 x E5C2; a step is short,
-// so producer groups take turns):
+// Orientation.  X takes the carry copies, so its planes need one binade more
+// than W's; an E5C2 operand goes on the weight side (its 32 binades fill
+// E5M2): E5C2 x E4C3 runs transposed (X = the E4C3 operand, C stored as
+// C[w][m]).  E5C2 x E5C2 stores the X planes one binade low (its lowest
+// binade's plain copy, 2^-17, has no E5M2 value and is dropped: an element
+// at least 2^30 below the top binade of its block).
+//
+// Roles (15 warps for 8-phase pairs, 17 for E5C2 x E5C2):
 //   warps 0-7   W producers: two groups of 4 warps taking alternate steps,
 //               one thread per weight row (all 32 codes of its steps): codes
-//               -> planes (pair planes and metadata) -> TMEM, prefetching
-//               PFW own steps ahead; after the last step they run the
-//               epilogue.
+//               -> pair planes, metadata and the row's scale factor -> TMEM;
+//               after the last step they run the epilogue.
 //   next warps  X producers: groups taking every NGX-th step, one 4-code word
-//               of one token per work item -> the step's blocks (Q or R),
-//               conflict-free stores; padding tokens are never written (the
-//               stages start at zero).
-//   last warp   TMEM allocation and MMA issue (one elected lane).
+//               of one token per work item -> the step's R blocks; the
+//               token's scale factors -> the stage's factor block (copied to
+//               TMEM by the MMA warp).
+//   last warp   TMEM allocation, factor copies and MMA issue (one elected
+//               lane).
 // With fewer weight tiles than fill the SMs' last wave, tiles are split in K
-// into two pieces (the tile kernel's greedy-dispatch simulation, extended to
-// grids smaller than the SM count); a piece adds its outputs to zeroed C
-// atomically, two additions per output, so the result does not depend on
-// their order.  Every wait is bounded.
+// into two pieces (greedy-dispatch simulation); a piece adds its outputs to
+// zeroed C atomically, two additions per output, so the result does not
+// depend on their order.  Every wait is bounded.
 #include "gemm_tc.cuh"
+#include "tc_mx.cuh"
 
 namespace cfp {
 
 namespace {
 
-template <int FX, int FW, bool T2>
+template <int FX, int FW>
 struct TcnCfg {
   using P = Pair<FX, FW>;
   static constexpr int KW = Fmt<FW>::K, L = P::L, WX = P::WA, WW = P::WB;
+  static_assert(WX == 1, "X planes sit on every lattice position");
   static constexpr int BM = 128;          // weight rows per CTA (TMEM lanes)
-  static constexpr int KS = 32;           // codes per pipeline step (K of one FP8 MMA)
+  static constexpr int KS = 32;           // codes per pipeline step (one scale factor)
   static constexpr int MTMAX = 256 / L;   // tokens per CTA: L Mt <= 256 (MMA N)
-  static constexpr int NBLK = 2 * L;      // column blocks of the doubled sequence
-  static constexpr bool SP = FX == FW;     // 2:4-sparse pair planes (below)
-  static constexpr bool TWO = SP && T2;    // two token groups per CTA (below)
-  // pipeline depth (X stages = W TMEM units): three where TMEM also holds two
-  // token groups' accumulators
-  static constexpr int NSB = TWO ? 3 : 4;
-  // Same-format pairs use 2:4-sparse pair planes: weight planes j and j + HB
-  // share one compressed operand (an element sits in one plane), at logical
-  // positions 2k and 2k + 1, with the curve-index bit MBIT as metadata.
+  static constexpr int NSB = 4;           // pipeline depth (X stages = W TMEM units)
   static constexpr int HB = KW / 2, MBIT = KW == 8 ? 2 : 1;
-  static constexpr int NJ = SP ? HB : KW;  // A operands (MMAs) per step
-  static constexpr int AU_COLS = NJ * 8;  // TMEM columns of one step's W planes
-  // A CTA takes one token group of Mt <= MTMAX tokens or (TWO: sparse form,
-  // large M) two groups of Mt <= MT2 with their accumulators side by side, so
-  // each decoded weight step serves up to 2 MT2 tokens.
-  static constexpr int MT2 = TWO ? 192 / L : 0;
-  static constexpr int MTOK = TWO ? 2 * MT2 : MTMAX;  // tokens per CTA at most
-  static constexpr int ACOL0 = TWO ? 384 : 256;       // W units after the accumulators
-  static constexpr int MCOL0 = ACOL0 + NSB * AU_COLS;  // metadata of unit u at MCOL0 + 8 u (2 used)
-  static_assert(MCOL0 + (SP ? NSB * 8 : 0) <= 512, "TMEM budget");
-  // sparse form: R blocks RB0 .. 2L-1 of 64-byte rows, R_b[2k] = Q_b[k],
-  // R_b[2k + 1] = Q_{b - HB}[k]; the operand of pair j is the window of L
-  // blocks from block L - j
-  static constexpr int RB0 = L - HB + 1, NRB = L + HB - 1;
-  static constexpr int ROWB = SP ? 64 : 32;  // bytes of one operand row
-  static_assert(L % 4 == 0 && KW % 2 == 0, "epilogue phase groups, plane pairs");
+  static constexpr int NJ = HB;           // sparse MMAs per step
+  static constexpr int PO = HB * WW;      // lattice distance of the partner plane
+  static constexpr int RB0 = L - (NJ - 1) * WW, NRB = 2 * L - RB0;
+  static constexpr int ROWB = 64;         // bytes of one operand row (logical K 64)
+  static constexpr int PBX = FX == CURVEFP_E5C2 ? 1 : 0;  // X planes one binade low
+  // TMEM columns: accumulators, W units, metadata (8 per unit, 2 used), A
+  // factors (4 per unit: quadrant q reads column q), B factors (8 per unit)
+  static constexpr int AU_COLS = NJ * 8;
+  static constexpr int ACOL0 = 256;
+  static constexpr int MCOL0 = ACOL0 + NSB * AU_COLS;
+  static constexpr int SFA0 = MCOL0 + NSB * 8;
+  static constexpr int SFB0 = (SFA0 + NSB * 4 + 31) / 32 * 32;
+  static_assert(SFB0 + NSB * 8 <= 512, "TMEM budget");
   // Producer groups take turns: W group g % NGW and X group g % NGX produce
   // step g, so each producer thread has NGW (NGX) steps of time per step.
   static constexpr int NGW = 2;                 // W groups of 4 warps (one thread per weight row)
@@ -99,25 +94,18 @@ struct TcnCfg {
   static constexpr int NXT = NGX * XPG * 32;    // X threads
   static constexpr int THREADS = NWT + NXT + 32;
   static constexpr int MMA_WARP = (NWT + NXT) / 32;
-  static constexpr int BSTAGE = (SP ? NRB * MTOK : NBLK * MTMAX) * ROWB;  // bytes of one step's X operand rows
-  static constexpr int PBX = FX == CURVEFP_E5C2 ? 1 : 0;  // plane exponent bias
-  static constexpr int PBW = FW == CURVEFP_E5C2 ? 1 : 0;
+  static constexpr int BSTAGE = NRB * MTMAX * ROWB;  // bytes of one step's X operand rows
+  static constexpr int SFSTAGE = 1024;               // factor block of a step (two copy sources)
   static constexpr int PFW = 4;  // own steps of weight codes in flight per W thread
   static constexpr int PFX = 2;  // own steps of activation codes in flight per X thread
-  static constexpr int XI = MTOK * 8 / (XPG * 32);  // X work items (4-code words) per thread and step
+  static constexpr int XI = MTMAX * 8 / (XPG * 32);  // X work items (4-code words) per thread and step
   // more than half of the SM's shared memory: one CTA per SM (the split plan
   // assumes it, and the CTA allocates all of TMEM)
-  static constexpr size_t SMEM_USED = (size_t)NSB * BSTAGE + 2048;
+  static constexpr size_t SMEM_USED = (size_t)NSB * (BSTAGE + SFSTAGE) + 2048;
   static constexpr size_t SMEM = SMEM_USED > 120 * 1024 ? SMEM_USED : 120 * 1024;
 };
 
-// Byte offset of row `row`, 16-byte chunk `kc` (of two) in a K-major
-// no-swizzle stage: 8-row core-matrix groups of 256 bytes.
-__device__ __forceinline__ uint32_t core_off(int row, int kc) {
-  return (uint32_t)((row >> 3) * 256 + kc * 128 + (row & 7) * 16);
-}
-
-// Largest block scale of a row (the row reference of the plane values).
+// Largest block scale of a row (the row reference of the scale factors).
 __device__ __forceinline__ int row_ref(const int8_t* s, int nb) {
   int ref = -128;
   if ((nb & 15) == 0 && (reinterpret_cast<uintptr_t>(s) & 15) == 0) {
@@ -151,16 +139,6 @@ __device__ __forceinline__ uint32_t pair_meta(uint32_t w0, uint32_t w1, uint32_t
   return m;
 }
 
-// 2:4-sparse MMA (kind::f8f6f4), A and metadata in TMEM, issued by `leader`.
-__device__ __forceinline__ void mma_sp_if(uint32_t leader, uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
-                                          uint32_t meta_tmem, uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n .reg .pred p, q;\n setp.ne.b32 p, %5, 0;\n setp.ne.b32 q, %6, 0;\n"
-      "@q tcgen05.mma.sp.cta_group::1.kind::f8f6f4 [%0], [%1], %2, [%3], %4, p;\n}\n" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(b_desc), "r"(meta_tmem), "r"(idesc), "r"(accumulate), "r"(leader)
-      : "memory");
-}
-
 // Interleave two words (elements 4q..4q+3 each) into X0 Y0 X1 Y1 | X2 Y2 X3 Y3.
 __device__ __forceinline__ uint2 interleave2(uint32_t x, uint32_t y) {
   return make_uint2(__byte_perm(x, y, 0x5140), __byte_perm(x, y, 0x7362));
@@ -181,17 +159,20 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16
 
 }  // namespace
 
-template <int FX, int FW, bool T2>
-__global__ void __launch_bounds__(TcnCfg<FX, FW, T2>::THREADS, 1)
+// X: [Mx x K] token codes, W: [Nw x K] weight codes (K contiguous), scales
+// [rows x K/G].  C: [Mx x Nw] (TR = false) or [Nw x Mx] (TR = true), row-major.
+template <int FX, int FW, bool TR>
+__global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
     gemm_tcn_kernel(const uint8_t* __restrict__ X, const int8_t* __restrict__ sX, const uint8_t* __restrict__ W,
-                    const int8_t* __restrict__ sW, int M, int N, int K, int G, int gshift, int Mt, int ntg,
+                    const int8_t* __restrict__ sW, int M, int N, int K, int G, int gshift, int Mt,
                     float* __restrict__ C, uint32_t* status, const TailPlan plan) {
-  using Cfg = TcnCfg<FX, FW, T2>;
+  using Cfg = TcnCfg<FX, FW>;
   constexpr int L = Cfg::L, NSB = Cfg::NSB;
-  static_assert(NSB <= TC_MAX_RING && Cfg::MTOK <= 128, "barrier rings, row references");
+  static_assert(NSB <= TC_MAX_RING && Cfg::MTMAX <= 128, "barrier rings, row references");
   extern __shared__ __align__(1024) uint8_t smem[];
   uint8_t* xstage = smem;
-  TcShared& sh = *reinterpret_cast<TcShared*>(smem + (size_t)NSB * Cfg::BSTAGE);
+  uint8_t* sfstage = smem + (size_t)NSB * Cfg::BSTAGE;
+  TcShared& sh = *reinterpret_cast<TcShared*>(smem + (size_t)NSB * (Cfg::BSTAGE + Cfg::SFSTAGE));
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   // this CTA's job: a whole tile (128 weight rows x Mt tokens) or one K piece
@@ -208,14 +189,13 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW, T2>::THREADS, 1)
       s0 = plan.split_step;
     }
   }
-  const int ntok = ntg * Mt;  // tokens of the CTA: ntg groups of Mt
-  const int x0 = (tile / ntw) * ntok, w0 = (tile % ntw) * Cfg::BM;
+  const int x0 = (tile / ntw) * Mt, w0 = (tile % ntw) * Cfg::BM;
   const int nb = K / G, total = s1 - s0;
   // Accumulator copies: consecutive MMAs of a step into one accumulator wait
   // for each other's accumulation, so where the accumulator is at most 128
-  // columns the weight planes rotate over 2 or 4 copies (NP columns each)
-  // that the epilogue adds up.
-  const int NP = L * Mt, nacc0 = ntg > 1 ? 1 : (NP <= 64 ? 4 : (NP <= 128 ? 2 : 1));
+  // columns the pair planes rotate over 2 or 4 copies (NP columns each) that
+  // the epilogue adds up.
+  const int NP = L * Mt, nacc0 = NP <= 64 ? 4 : (NP <= 128 ? 2 : 1);
   const int nacc = nacc0 < Cfg::NJ ? nacc0 : Cfg::NJ;  // every copy receives an MMA each step
 
   if (tid == 0) {
@@ -232,21 +212,21 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW, T2>::THREADS, 1)
     tc::tmem_relinquish();
   }
   const bool is_w = tid < Cfg::NWT, is_x = !is_w && warp < Cfg::MMA_WARP;
-  // W threads: weight row (TMEM lane) and group; X threads: group.  The
-  // row references: a weight row per W thread, a token per thread of the
-  // first X group.  The X stages start at zero (padding tokens and empty
-  // lattice positions are never written).
+  // W threads: weight row (TMEM lane) and group; X threads: group.  The row
+  // references: a weight row per W thread, a token per thread of the first X
+  // group.  The X stages and factor blocks start at zero (padding tokens and
+  // empty lattice positions are never written).
   const int wrow = w0 + (warp & 3) * 32 + lane, gw = warp >> 2;
   const int t_x = tid - Cfg::NWT, gx = t_x / (Cfg::XPG * 32);
   int ref = -128;
   if (is_w && wrow < N) ref = row_ref(sW + (int64_t)wrow * nb, nb);
-  if (is_x && t_x < Cfg::MTOK) {
+  if (is_x && t_x < Cfg::MTMAX) {
     int rx = -128;
-    if (t_x < ntok && x0 + t_x < M) rx = row_ref(sX + (int64_t)(x0 + t_x) * nb, nb);
+    if (t_x < Mt && x0 + t_x < M) rx = row_ref(sX + (int64_t)(x0 + t_x) * nb, nb);
     sh.refB[t_x] = rx;
   }
-  for (int o = tid * 16; o < NSB * Cfg::BSTAGE; o += Cfg::THREADS * 16)
-    *reinterpret_cast<uint4*>(xstage + o) = make_uint4(0, 0, 0, 0);
+  for (int o = tid * 16; o < NSB * (Cfg::BSTAGE + Cfg::SFSTAGE); o += Cfg::THREADS * 16)
+    *reinterpret_cast<uint4*>(smem + o) = make_uint4(0, 0, 0, 0);
   tc::fence_proxy_async_smem();
   tc::fence_before_sync();
   __syncthreads();
@@ -286,24 +266,24 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW, T2>::THREADS, 1)
       if (lane == 0) tc::mbar_arrive(&sh.full[pend]);
       pend = -1;
     };
-    auto step = [&](const int g, const uint4 lo, const uint4 hi, const int raw) -> bool {
-      const int st = g % NSB, off = raw - ref - Cfg::PBW;
-      // the 32 codes of the row's step: value words and curve-index masks;
-      // plane j of word w = p[w][j & 3] & (bit 2 of k set ? mk2 : ~mk2)
-      uint32_t p[8][4], m2[8];
+    auto step = [&](const int g, uint4 lo, uint4 hi, const int raw) -> bool {
+      const int st = g % NSB;
+      bool keep;
+      const uint32_t sf = mx_sf(raw - ref, 0, keep) * 0x01010101u;
+      if (!keep) lo = hi = make_uint4(0, 0, 0, 0);
+      // the 32 codes of the row's step: plane words and curve-index masks;
+      // pair plane j of word w = the elements whose low curve-index bits are j
+      uint32_t p[8][4];
+      const uint32_t cw[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        uint32_t v[4], vc[4], mk[4][4];
-        PlaneFmt<FW>::template decode<PLANE_E5M2, 4>(h ? hi : lo, off, v, vc, mk, false);
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          const int w = h * 4 + c;
-          p[w][0] = v[c] & ~mk[c][0] & ~mk[c][1];
-          p[w][1] = v[c] & mk[c][0] & ~mk[c][1];
-          p[w][2] = v[c] & ~mk[c][0] & mk[c][1];
-          p[w][3] = v[c] & mk[c][0] & mk[c][1];
-          m2[w] = mk[c][2];
-        }
+      for (int w = 0; w < 8; ++w) {
+        uint32_t v, vc, mk[4];
+        mx_word<FW, 0>(cw[w], v, vc);
+        k_masks<PLANE_E5M2, Fmt<FW>::C>(cw[w], mk);
+        p[w][0] = v & ~mk[0] & ~mk[1];
+        p[w][1] = v & mk[0] & ~mk[1];
+        p[w][2] = v & ~mk[0] & mk[1];
+        p[w][3] = v & mk[0] & mk[1];
       }
       hand_over();
       if (g >= NSB) {
@@ -316,10 +296,8 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW, T2>::THREADS, 1)
           return false;
         }
       }
-      // operands 2jp and 2jp + 1 of the step: 16 consecutive columns of the
-      // unit.  Dense: plane j.  Sparse: pair plane j = the elements whose
-      // curve index is j or j + HB (low bits of k equal to j), plus the
-      // metadata words of codes 0-15 and 16-31.
+      // pair planes 2jp and 2jp + 1 of the step: 16 consecutive columns of
+      // the unit, then the metadata of codes 0-15 and 16-31 and the factor
 #pragma unroll
       for (int jp = 0; jp < Cfg::NJ / 2; ++jp) {
         uint32_t r[16];
@@ -327,21 +305,14 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW, T2>::THREADS, 1)
         for (int e = 0; e < 2; ++e) {
           const int j = 2 * jp + e;
 #pragma unroll
-          for (int w = 0; w < 8; ++w) {
-            if constexpr (!Cfg::SP)
-              r[e * 8 + w] = p[w][j & 3] & ((j & 4) ? m2[w] : ~m2[w]);
-            else if constexpr (Cfg::KW == 8)
-              r[e * 8 + w] = p[w][j];
-            else
-              r[e * 8 + w] = p[w][j] | p[w][j + 2];
-          }
+          for (int w = 0; w < 8; ++w) r[e * 8 + w] = Cfg::KW == 8 ? p[w][j] : (p[w][j] | p[w][j + 2]);
         }
         tmem_st16(lane_base + Cfg::ACOL0 + st * Cfg::AU_COLS + jp * 16, r);
       }
-      if constexpr (Cfg::SP) {
-        const uint32_t mt[2] = {pair_meta<Cfg::MBIT>(lo.x, lo.y, lo.z, lo.w), pair_meta<Cfg::MBIT>(hi.x, hi.y, hi.z, hi.w)};
-        tc::tmem_st2(lane_base + Cfg::MCOL0 + st * 8, mt);
-      }
+      const uint32_t mt[2] = {pair_meta<Cfg::MBIT>(lo.x, lo.y, lo.z, lo.w),
+                              pair_meta<Cfg::MBIT>(hi.x, hi.y, hi.z, hi.w)};
+      tc::tmem_st2(lane_base + Cfg::MCOL0 + st * 8, mt);
+      tc::tmem_st1(lane_base + Cfg::SFA0 + st * 4 + (warp & 3), sf);
       pend = st;
       return true;
     };
@@ -371,16 +342,16 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW, T2>::THREADS, 1)
     if (!failed) hand_over();
     // Epilogue (after the last MMA): chunks of 8 tokens, chunk ch taken by
     // group ch % NGW; per token the phase sums D[w][h Mt + m] are combined as
-    // sum_h 2^{h/L} S_h (FP32, phase order) and scaled by 2^{ref_w + ref_m}.
-    // A whole tile stores C, a K piece adds to zeroed C.
+    // sum_h 2^{h/L} S_h (FP32, phase order) and scaled by
+    // 2^{ref_w + ref_m - 2 MX_OFF}.  A whole tile stores C, a K piece adds to
+    // zeroed C.
     const bool aborted = __any_sync(0xffffffffu, read_abort(&sh.abort_flag) != 0);
     const bool ok = !aborted && wait_all(&sh.acc_full, 0);
     if (!ok && lane == 0) raise_flag(status, CURVEFP_DEV_TIMEOUT);
     tc::fence_after_sync();
 #pragma unroll 1
-    for (int ch = gw; ch < (ntok >> 3); ch += NGW) {
-      // chunk ch: tokens 8 ch .. 8 ch + 7 of token group tgp (local lt ..)
-      const int tgp = (ch * 8) / Mt, lt = ch * 8 - tgp * Mt;
+    for (int ch = gw; ch < (Mt >> 3); ch += NGW) {
+      const int lt = ch * 8;  // tokens lt .. lt + 7 of the tile
       float t[8];
 #pragma unroll
       for (int j = 0; j < 8; ++j) t[j] = 0.f;
@@ -392,7 +363,7 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW, T2>::THREADS, 1)
         for (int a = 0; a < nacc; ++a) {
           uint32_t acc[4][8];
 #pragma unroll
-          for (int h = 0; h < 4; ++h) tc::tmem_ld8(lane_base + (tgp + a) * NP + (h0 + h) * Mt + lt, acc[h]);
+          for (int h = 0; h < 4; ++h) tc::tmem_ld8(lane_base + a * NP + (h0 + h) * Mt + lt, acc[h]);
           tc::tmem_wait_ld();
 #pragma unroll
           for (int h = 0; h < 4; ++h)
@@ -405,16 +376,36 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW, T2>::THREADS, 1)
           for (int h = 0; h < 4; ++h) t[j] = fmaf(phase_const(L, h0 + h), sh4[h][j], t[j]);
       }
       if (rowok && ok) {
+        float y[8];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const int tok = ch * 8 + j, m = x0 + tok;
-          if (m < M) {
-            const float y = scalbnf(t[j], ref + Cfg::PBW + sh.refB[tok] + Cfg::PBX);
-            float* dst = C + (int64_t)m * N + wrow;
-            if (split)
-              atomicAdd(dst, y);
-            else
-              *dst = y;
+        for (int j = 0; j < 8; ++j) y[j] = scalbnf(t[j], ref + sh.refB[lt + j] - 2 * MX_OFF);
+        const int m0 = x0 + lt;
+        if constexpr (TR) {
+          // C[w][m]: the thread's 8 consecutive tokens
+          float* dst = C + (int64_t)wrow * M + m0;
+          if (split) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+              if (m0 + j < M) atomicAdd(dst + j, y[j]);
+          } else if (m0 + 8 <= M && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
+            reinterpret_cast<float4*>(dst)[0] = make_float4(y[0], y[1], y[2], y[3]);
+            reinterpret_cast<float4*>(dst)[1] = make_float4(y[4], y[5], y[6], y[7]);
+          } else {
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+              if (m0 + j < M) dst[j] = y[j];
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int m = m0 + j;
+            if (m < M) {
+              float* dst = C + (int64_t)m * N + wrow;
+              if (split)
+                atomicAdd(dst, y[j]);
+              else
+                *dst = y[j];
+            }
           }
         }
       }
@@ -422,31 +413,30 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW, T2>::THREADS, 1)
   } else if (is_x) {
     // ---------------------------- X producers -----------------------------
     // Work item wi of a group covers one 4-code word: lane bits of wi give 8
-    // tokens x 4 words of a 16-code chunk kc, so a warp's 4-byte stores fill
-    // 128 consecutive bytes of a column block.  Items of padding tokens (and
+    // tokens x 4 words of a 16-code chunk kc, so a warp's 8-byte stores fill
+    // 256 consecutive bytes of an R block.  Items of padding tokens (and
     // lattice positions that hold no plane) write nothing: the stages were
-    // zeroed at the start.
+    // zeroed at the start.  The item of a token's first word also writes the
+    // token's scale factor into the factor block: one word per column n =
+    // h Mt + m of the MMA (the factor ids read bytes 0 and 1).
     constexpr int PF = Cfg::PFX, XI = Cfg::XI, NGX = Cfg::NGX;
     const int tg = t_x % (Cfg::XPG * 32);  // thread of the group
-    // per item: activation row (-1: padding), its row reference and the
-    // byte offset of its word in a stage (block b adds b Mt ROWB bytes)
-    int xrow[XI], xref[XI];
+    // per item: activation row (-1: padding), its row reference, its token
+    // and the byte offset of its word in a stage (block b adds b Mt 64 bytes)
+    int xrow[XI], xref[XI], xtok[XI];
     uint32_t xbase[XI];
     auto word_of = [&](int wi) { return ((wi >> 5) & 1) * 4 + ((wi & 31) >> 3); };  // 4-code word of the step
 #pragma unroll
     for (int i = 0; i < XI; ++i) {
-      const int wi = tg + i * Cfg::XPG * 32, xl = wi & 31, kc = (wi >> 5) & 1;
-      const int tokc = (wi >> 6) * 8 + (xl & 7), sub = xl >> 3;  // token of the CTA
-      const bool act = wi < ntok * 8 && x0 + tokc < M;
-      xrow[i] = act ? x0 + tokc : -1;
-      xref[i] = act ? sh.refB[tokc] : 0;
-      // token group and local token; dense: word sub of 16-byte chunk kc of
-      // a 32-byte row; sparse: the word's 8 interleaved bytes in 16-byte
-      // chunk j >> 1 of a 64-byte row, group t's R blocks after group t - 1's
-      const int t = act ? tokc / Mt : 0, tok = act ? tokc - t * Mt : 0, j = kc * 4 + sub;
-      xbase[i] = Cfg::SP ? (uint32_t)(t * Cfg::NRB * Mt * 64 + (tok >> 3) * 512 + (j >> 1) * 128 + (tok & 7) * 16 +
-                                      (j & 1) * 8)
-                         : core_off(tok, kc) + sub * 4;
+      const int wi = tg + i * Cfg::XPG * 32, xl = wi & 31;
+      const int tok = (wi >> 6) * 8 + (xl & 7);  // token of the tile
+      const bool act = tok < Mt && x0 + tok < M;
+      xrow[i] = act ? x0 + tok : -1;
+      xref[i] = act ? sh.refB[tok] : 0;
+      xtok[i] = word_of(wi) == 0 ? tok : -1;  // writes the token's factors
+      // the word's 8 interleaved bytes in 16-byte chunk j >> 1 of a 64-byte row
+      const int j = word_of(wi);
+      xbase[i] = (uint32_t)((tok >> 3) * 512 + (j >> 1) * 128 + (tok & 7) * 16 + (j & 1) * 8);
     }
     auto load = [&](int i, uint32_t (&cw)[XI], int (&raw)[XI]) {
       const int g = gx + i * NGX;
@@ -475,31 +465,30 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW, T2>::THREADS, 1)
         }
       }
       uint8_t* stg = xstage + (size_t)st * Cfg::BSTAGE;
+      uint8_t* sfs = sfstage + (size_t)st * Cfg::SFSTAGE;
 #pragma unroll
       for (int e = 0; e < XI; ++e) {
         if (xrow[e] < 0) continue;
-        uint32_t v[1], vc[1], mk[1][4];
-        PlaneFmt<FX>::template decode<PLANE_E5M2, 1>(make_uint4(cw[e], 0u, 0u, 0u), raw[e] - xref[e] - Cfg::PBX, v,
-                                                     vc, mk, true);
+        bool keep;
+        const uint32_t sf = mx_sf(raw[e] - xref[e], Cfg::PBX, keep);
+        uint32_t v, vc, mk[4];
+        mx_word<FX, Cfg::PBX>(keep ? cw[e] : 0u, v, vc);
+        k_masks<PLANE_E5M2, Fmt<FX>::C>(cw[e], mk);
         uint32_t pv[8], pc[8];
-        PlaneFmt<FX>::planes(v[0], mk[0], pv);
-        PlaneFmt<FX>::planes(vc[0], mk[0], pc);
-        if constexpr (Cfg::SP) {
-          // R block b interleaves Q block b (plane partner) with Q block b - HB;
-          // Q block u < L is the carry copy of plane u, u >= L plane u - L
+        planes_of<Fmt<FX>::C>(v, mk, pv);
+        planes_of<Fmt<FX>::C>(vc, mk, pc);
+        // R block b interleaves Q block b with Q block b - PO; Q block u < L
+        // is the carry copy of plane u, u >= L plane u - L
 #pragma unroll
-          for (int b = Cfg::RB0; b < 2 * L; ++b) {
-            const uint32_t x = b < L ? pc[b] : pv[b - L];
-            const uint32_t y = b - Cfg::HB < L ? pc[b - Cfg::HB] : pv[b - Cfg::HB - L];
-            *reinterpret_cast<uint2*>(stg + xbase[e] + (b - Cfg::RB0) * bstride) = interleave2(x, y);
-          }
-        } else {
-          // lattice position u holds plane u / WX where WX divides u
+        for (int b = Cfg::RB0; b < 2 * L; ++b) {
+          const uint32_t x = b < L ? pc[b] : pv[b - L];
+          const uint32_t y = b - Cfg::PO < L ? pc[b - Cfg::PO] : pv[b - Cfg::PO - L];
+          *reinterpret_cast<uint2*>(stg + xbase[e] + (b - Cfg::RB0) * bstride) = interleave2(x, y);
+        }
+        if (xtok[e] >= 0) {
+          const uint32_t sw = sf * 0x01010101u;
 #pragma unroll
-          for (int u = 0; u < L; u += Cfg::WX) {
-            *reinterpret_cast<uint32_t*>(stg + xbase[e] + u * bstride) = pc[u / Cfg::WX];
-            *reinterpret_cast<uint32_t*>(stg + xbase[e] + (L + u) * bstride) = pv[u / Cfg::WX];
-          }
+          for (int h = 0; h < L; ++h) *reinterpret_cast<uint32_t*>(sfs + sfb_off(h * Mt + xtok[e])) = sw;
         }
       }
       tc::fence_proxy_async_smem();
@@ -526,9 +515,8 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW, T2>::THREADS, 1)
   } else {
     // ------------------------------ MMA issuer -------------------------------
     const uint32_t leader = tc::elect_one();
-    const uint64_t bdesc0 = tc::smem_desc(tc::smem_u32(xstage), 128, Cfg::SP ? 512 : 256);
-    // E5M2 x E5M2 -> F32, N = L Mt (bit 2: 2:4-sparse A)
-    const uint32_t idesc = tc::idesc_bf16_f32(Cfg::BM, NP) | (Cfg::SP ? (1u << 2) : 0u);
+    const uint64_t bdesc0 = tc::smem_desc(tc::smem_u32(xstage), 128, 512);
+    const uint32_t idesc = idesc_mx_e5m2(NP, true);
     const int gbytes = Mt * Cfg::ROWB;  // bytes of one column block
     bool ok = true;
     for (int g = 0; g < total && ok; ++g) {
@@ -537,21 +525,19 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW, T2>::THREADS, 1)
       if ((g & 7) == 0) ok = ok && !read_abort(&sh.abort_flag);
       if (!ok) break;
       tc::fence_after_sync();
-#pragma unroll 1
-      for (int tg2 = 0; tg2 < ntg; ++tg2)
+      // the step's B factors: columns 0..127 and, for N > 128, 128..255
+      const uint8_t* sfs = sfstage + (size_t)st * Cfg::SFSTAGE;
+      tmem_cp_sf_if(leader, tmem + Cfg::SFB0 + st * 8, sfs);
+      if (NP > 128) tmem_cp_sf_if(leader, tmem + Cfg::SFB0 + st * 8 + 4, sfs + 512);
 #pragma unroll
       for (int kw = 0; kw < Cfg::NJ; ++kw) {
-        // weight plane (pair plane) k_w against the window of column blocks
-        // from L - k_w WW (R block L - k_w) of token group tg2
+        // pair plane kw against the window of R blocks from L - kw WW
         const uint32_t a_t = tmem + Cfg::ACOL0 + st * Cfg::AU_COLS + kw * 8;
-        const uint32_t boff = (uint32_t)(st * Cfg::BSTAGE + tg2 * Cfg::NRB * gbytes +
-                                         (Cfg::SP ? L - kw - Cfg::RB0 : L - kw * Cfg::WW) * gbytes);
-        const uint32_t d_t = tmem + (uint32_t)((tg2 + (kw & (nacc - 1))) * NP);
+        const uint32_t boff = (uint32_t)(st * Cfg::BSTAGE + (L - kw * Cfg::WW - Cfg::RB0) * gbytes);
+        const uint32_t d_t = tmem + (uint32_t)((kw & (nacc - 1)) * NP);
         const uint32_t acc = (g == 0 && kw < nacc) ? 0u : 1u;
-        if constexpr (Cfg::SP)
-          mma_sp_if(leader, d_t, a_t, bdesc0 + (uint64_t)(boff >> 4), tmem + Cfg::MCOL0 + st * 8, idesc, acc);
-        else
-          tc::mma_f8_ts_if(leader, d_t, a_t, bdesc0 + (uint64_t)(boff >> 4), idesc, acc);
+        mma_sp_mx_if(leader, d_t, a_t, bdesc0 + (uint64_t)(boff >> 4), tmem + Cfg::MCOL0 + st * 8, idesc,
+                     tmem + Cfg::SFA0 + st * 4, tmem + Cfg::SFB0 + st * 8, acc);
       }
       tc::mma_commit_if(leader, &sh.empty[st]);
       if (g == total - 1) tc::mma_commit_if(leader, &sh.acc_full);
@@ -613,34 +599,38 @@ inline TailPlan tcn_plan(int64_t tiles, int sms, int nsub) {
   return t;
 }
 
-template <int FX, int FW, bool T2>
-cudaError_t launch_tcn_t(int G, const uint8_t* x, const int8_t* sx, const uint8_t* w, const int8_t* sw, int64_t M,
-                         int64_t N, int64_t K, float* c, uint32_t* st, cudaStream_t s, int sms) {
-  using Cfg = TcnCfg<FX, FW, T2>;
+// x: [Mx x K] token codes, w: [Nw x K] weight codes; c: [Mx x Nw], or
+// [Nw x Mx] with TR.
+template <int FX, int FW, bool TR>
+cudaError_t launch_tcn_t(int G, const uint8_t* x, const int8_t* sx, const uint8_t* w, const int8_t* sw, int64_t Mx,
+                         int64_t Nw, int64_t K, float* c, uint32_t* st, cudaStream_t s, int sms) {
+  using Cfg = TcnCfg<FX, FW>;
   static_assert(sizeof(TcShared) <= 2048, "shared tail");
   static_assert(Cfg::SMEM <= 227 * 1024, "shared memory");
-  auto kern = gemm_tcn_kernel<FX, FW, T2>;
+  auto kern = gemm_tcn_kernel<FX, FW, TR>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg::SMEM);
   if (e != cudaSuccess) return e;
-  // token groups of equal size Mt (a multiple of 8): one per CTA of at most
-  // MTMAX tokens, or (sparse form, larger M) two per CTA of at most MT2
-  const int ntg = Cfg::TWO ? 2 : 1;
-  const int64_t cap = ntg == 2 ? 2 * Cfg::MT2 : Cfg::MTMAX;
-  int64_t ng = (M + cap - 1) / cap;
-  const int Mt = (int)(((M + ng * ntg - 1) / (ng * ntg) + 7) / 8 * 8);
-  ng = (M + (int64_t)ntg * Mt - 1) / ((int64_t)ntg * Mt);
-  const int64_t ntw = (N + Cfg::BM - 1) / Cfg::BM, tiles = ntw * ng;
+  // token groups of equal size Mt (a multiple of 8) of at most MTMAX tokens
+  int64_t ng = (Mx + Cfg::MTMAX - 1) / Cfg::MTMAX;
+  const int Mt = (int)(((Mx + ng - 1) / ng + 7) / 8 * 8);
+  ng = (Mx + Mt - 1) / Mt;
+  const int64_t ntw = (Nw + Cfg::BM - 1) / Cfg::BM, tiles = ntw * ng;
   const TailPlan plan = tcn_plan(tiles, sms, (int)(K / Cfg::KS));
   if (plan.nsplit > 0) {
-    // C of the split tiles starts at zero: whole token groups from the first one
-    const int64_t row0 = (plan.ntiles_full / ntw) * ntg * Mt;
-    e = cudaMemsetAsync(c + row0 * N, 0, (size_t)((M - row0) * N) * sizeof(float), s);
+    // C of the split tiles starts at zero: for C[m][w], the token rows from
+    // the first split tile's group on; for C[w][m], all of C
+    if (TR) {
+      e = cudaMemsetAsync(c, 0, (size_t)(Mx * Nw) * sizeof(float), s);
+    } else {
+      const int64_t row0 = (plan.ntiles_full / ntw) * Mt;
+      e = cudaMemsetAsync(c + row0 * Nw, 0, (size_t)((Mx - row0) * Nw) * sizeof(float), s);
+    }
     if (e != cudaSuccess) return e;
   }
   const unsigned grid = (unsigned)(plan.ntiles_full + 2 * plan.nsplit);
   int gshift = 0;  // scale block of step s is s >> gshift
   while ((Cfg::KS << gshift) < G) ++gshift;
-  kern<<<grid, Cfg::THREADS, Cfg::SMEM, s>>>(x, sx, w, sw, (int)M, (int)N, (int)K, G, gshift, Mt, ntg, c, st, plan);
+  kern<<<grid, Cfg::THREADS, Cfg::SMEM, s>>>(x, sx, w, sw, (int)Mx, (int)Nw, (int)K, G, gshift, Mt, c, st, plan);
   return cudaGetLastError();
 }
 
@@ -652,23 +642,23 @@ bool gemm_narrow_supported(int fa, int fb) {
          (fa == CURVEFP_E5C2 && fb == CURVEFP_E5C2);
 }
 
+// C = A_hat B_hat^T, A [M x K] (format fa), B [N x K] (format fb).  The
+// tokens are A's rows and the weights B's, except for E5C2 x E4C3, which runs
+// transposed (tokens = B's rows, weights = A's rows, C written as C[m][n]
+// with m the weight index) so that the E5C2 operand is on the weight side.
 cudaError_t launch_gemm_tensor_narrow(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
                                       const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, uint32_t* status,
                                       cudaStream_t s, int sms) {
-  // same-format pairs from 512 activation rows: two token groups per CTA
-  // (measured: 2048 x 4096 x 4096 0.861 -> 0.837 ms, FFN M = 4096 5.94 ->
-  // 5.54 ms; at M <= 256 the deeper one-group ring and its waves are faster)
-  const bool two = fa == fb && M >= 512;
-#define CFP_T(X, Y)                                                                                  \
-  if (fa == X && fb == Y)                                                                           \
-    return two ? launch_tcn_t<X, Y, true>(G, a, sa, b, sb, M, N, K, c, status, s, sms)             \
-               : launch_tcn_t<X, Y, false>(G, a, sa, b, sb, M, N, K, c, status, s, sms);
-  CFP_T(CURVEFP_E3C3, CURVEFP_E3C3)
-  CFP_T(CURVEFP_E4C3, CURVEFP_E4C3)
-  CFP_T(CURVEFP_E5C2, CURVEFP_E4C3)
-  CFP_T(CURVEFP_E4C3, CURVEFP_E5C2)
-  CFP_T(CURVEFP_E5C2, CURVEFP_E5C2)
-#undef CFP_T
+  if (fa == CURVEFP_E3C3 && fb == CURVEFP_E3C3)
+    return launch_tcn_t<CURVEFP_E3C3, CURVEFP_E3C3, false>(G, a, sa, b, sb, M, N, K, c, status, s, sms);
+  if (fa == CURVEFP_E4C3 && fb == CURVEFP_E4C3)
+    return launch_tcn_t<CURVEFP_E4C3, CURVEFP_E4C3, false>(G, a, sa, b, sb, M, N, K, c, status, s, sms);
+  if (fa == CURVEFP_E4C3 && fb == CURVEFP_E5C2)
+    return launch_tcn_t<CURVEFP_E4C3, CURVEFP_E5C2, false>(G, a, sa, b, sb, M, N, K, c, status, s, sms);
+  if (fa == CURVEFP_E5C2 && fb == CURVEFP_E4C3)
+    return launch_tcn_t<CURVEFP_E4C3, CURVEFP_E5C2, true>(G, b, sb, a, sa, N, M, K, c, status, s, sms);
+  if (fa == CURVEFP_E5C2 && fb == CURVEFP_E5C2)
+    return launch_tcn_t<CURVEFP_E5C2, CURVEFP_E5C2, false>(G, a, sa, b, sb, M, N, K, c, status, s, sms);
   return cudaErrorInvalidValue;
 }
 

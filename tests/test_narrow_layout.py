@@ -2,15 +2,21 @@
 the oracle's closed-product GEMM (Eq. 2, Eq. 5).
 
 A numpy model of what the kernel's MMAs compute, at the level of plane values
-(not bytes): weight plane k_w (the 128-row operand) against the window of L
-column blocks from block L - k_w WW of Q = [carry copies of the activation
-planes on lattice positions 0..L-1 | plain copies], accumulating
-D[w][h Mt + m] = S_h; for same-format pairs the 2:4-sparse form, where pair
-plane j (planes j and j + K/2 at logical positions 2k, 2k + 1) meets the
-window of R blocks from L - j with R_b[2k] = Q_b[k], R_b[2k + 1] = Q_{b-K/2}[k].
-The phase combine sum_h 2^{h/L} S_h then has to reproduce the oracle's C for
-every format pair; a wrong window start, a missing carry copy or a swapped
-interleave fails it."""
+and scale factors (not bytes): every element's plane value is the power of
+two 2^e of its code (one binade low on an E5C2 token operand, whose carry
+copies need the room), every 32-code step of a row carries the scale factor
+2^{a_b - ref + 32}, and weight pair plane j (planes j and j + K_W/2 at
+logical positions 2k, 2k + 1) meets the window of L column blocks from R
+block L - j WW, with R_b[2k] = Q_b[k], R_b[2k + 1] = Q_{b - PO}[k],
+PO = K_W/2 WW, and Q = [carry copies of the token planes on lattice
+positions 0..L-1 | plain copies].  D[w][h Mt + m] = S_h, and the phase
+combine sum_h 2^{h/L} S_h 2^{ref_w + ref_m - 64} has to reproduce the
+oracle's C for every format pair, E5C2 x E4C3 in its transposed orientation
+(the E5C2 operand on the weight side); a wrong window start, a missing carry
+copy, a swapped interleave or a scale factor on the wrong block fails it.
+
+The byte-level arithmetic that forms the E5M2 plane bytes four codes at a
+time (tc_mx.cuh mx_word) is emulated on every code byte in every lane."""
 import numpy as np
 import pytest
 
@@ -18,104 +24,211 @@ import oracle
 
 FMTS = {"E3C3": (3, 3), "E4C3": (4, 3), "E5C2": (5, 2)}
 PAIRS = [("E3C3", "E3C3"), ("E4C3", "E4C3"), ("E5C2", "E4C3"), ("E4C3", "E5C2"), ("E5C2", "E5C2")]
+MX_OFF = 32
 
 
-def planes(codes, scales, fmt, G):
-    """Per element: curve index k and the power-of-two plane value
-    +-2^{e + a_b - ref} (ref = the row's largest block scale), the code
-    layout of the oracle's reading R1; zero codes have value 0."""
+def fields(codes, fmt):
     E, C = FMTS[fmt]
     K, B = 1 << C, 1 << (E + C - 1)
     m = (codes & (0x3F if fmt == "E3C3" else 0x7F)).astype(np.int64)
     n = m - B
     e = np.floor_divide(n, K)
-    k = n - e * K
-    a = np.repeat(scales.astype(np.int64), G, axis=1)
+    return m, e, n - e * K
+
+
+def planes(codes, scales, fmt, G, bias):
+    """Per element: curve index k, the plane value +-2^{e - bias} (0 for zero
+    codes and, with bias 1, for the plain copy of e = -16, which E5M2 cannot
+    hold), the carry value +-2^{e - bias + 1}, the per-element scale factor
+    exponent a_b - ref + 32 + bias, and the row reference."""
+    m, e, k = fields(codes, fmt)
+    sgn = np.where(codes & 0x80, -1.0, 1.0)
+    v = np.where((m != 0) & (e - bias >= -16), sgn * np.exp2((e - bias).astype(float)), 0.0)
+    vc = np.where(m != 0, sgn * np.exp2((e - bias + 1).astype(float)), 0.0)
     ref = scales.max(axis=1).astype(np.int64)
-    v = np.where(codes & 0x80, -1.0, 1.0) * np.exp2((e + a - ref[:, None]).astype(float))
-    return k, np.where(m != 0, v, 0.0), ref
+    sf = np.repeat(scales.astype(np.int64), G, axis=1) - ref[:, None] + MX_OFF + bias
+    return k, v, vc, sf, ref
 
 
-def narrow_model(a, sa, b, sb, fx, fw, G, Mt, sparse):
-    M, Kd = a.shape
+def narrow_model(x, sx, w, sw, fx, fw, G, Mt):
+    """C[m][n] = x_hat[m] . w_hat[n] as the kernel forms it (tokens x, weights w)."""
+    M, Kd = x.shape
     KX, KW = 1 << FMTS[fx][1], 1 << FMTS[fw][1]
     L = max(KX, KW)
     WX, WW = L // KX, L // KW
-    kx, vx, rx = planes(a, sa, fx, G)
-    kw, vw, rw = planes(b, sb, fw, G)
-    C = np.zeros((M, b.shape[0]))
+    assert WX == 1
+    bx = 1 if fx == "E5C2" else 0
+    kx, vx, cx, fxs, rx = planes(x, sx, fx, G, bx)
+    kw, vw, _, fws, rw = planes(w, sw, fw, G, 0)
+    hb = KW // 2
+    po = hb * WW
+    C = np.zeros((M, w.shape[0]))
     for x0 in range(0, M, Mt):  # one token group per CTA tile
         toks = np.arange(x0, min(x0 + Mt, M))
-        D = np.zeros((b.shape[0], L * Mt))
-        # Q[u] (u < L: carry copy of position u; u >= L: plain), [Mt x K]
+        D = np.zeros((w.shape[0], L * Mt))
+        # Q[u] (u < L: carry copy of position u; u >= L: plain), [Mt x K],
+        # with the tokens' scale factors applied (the B factors of a column)
         Q = np.zeros((2 * L, Mt, Kd))
+        scale_x = np.exp2(fxs[toks].astype(float))
         for u in range(L):
-            if u % WX == 0:
-                pl = np.where(kx[toks] == u // WX, vx[toks], 0.0)
-                Q[u, : len(toks)] = 2 * pl
-                Q[L + u, : len(toks)] = pl
-        if not sparse:
-            for k in range(KW):
-                window = Q[L - k * WW: 2 * L - k * WW].reshape(L * Mt, Kd)
-                D += np.where(kw == k, vw, 0.0) @ window.T
-        else:
-            hb = KW // 2
-            for j in range(hb):
-                # logical K 2 Kd: A[2k] = plane j, A[2k + 1] = plane j + hb
-                A = np.zeros((b.shape[0], 2 * Kd))
-                A[:, 0::2] = np.where(kw == j, vw, 0.0)
-                A[:, 1::2] = np.where(kw == j + hb, vw, 0.0)
-                R = np.zeros((L, Mt, 2 * Kd))
-                for h in range(L):
-                    R[h, :, 0::2] = Q[L - j + h]
-                    R[h, :, 1::2] = Q[L - j + h - hb]
-                D += A @ R.reshape(L * Mt, 2 * Kd).T
+            Q[u, : len(toks)] = np.where(kx[toks] == u, cx[toks], 0.0) * scale_x
+            Q[L + u, : len(toks)] = np.where(kx[toks] == u, vx[toks], 0.0) * scale_x
+        scale_w = np.exp2(fws.astype(float))
+        for j in range(hb):
+            # logical K 2 Kd: A[2k] = plane j, A[2k + 1] = plane j + hb (the A factors)
+            A = np.zeros((w.shape[0], 2 * Kd))
+            A[:, 0::2] = np.where(kw == j, vw, 0.0) * scale_w
+            A[:, 1::2] = np.where(kw == j + hb, vw, 0.0) * scale_w
+            R = np.zeros((L, Mt, 2 * Kd))
+            for h in range(L):
+                R[h, :, 0::2] = Q[L - j * WW + h]
+                R[h, :, 1::2] = Q[L - j * WW + h - po]
+            D += A @ R.reshape(L * Mt, 2 * Kd).T
         ph = np.exp2(np.arange(L) / L)
         S = D.reshape(-1, L, Mt)  # [w, h, m]
         Ct = np.einsum("h,whm->mw", ph, S)[: len(toks)]
-        C[toks] = Ct * np.exp2((rx[toks][:, None] + rw[None, :]).astype(float))
+        C[toks] = Ct * np.exp2((rx[toks][:, None] + rw[None, :] - 2 * MX_OFF).astype(float))
     return C
 
 
-def _operand(rng, fmt, rows, K, G):
+def kernel_model(a, sa, b, sb, fa, fb, G, Mt):
+    """The launcher's orientation: E5C2 x E4C3 runs with the E4C3 operand as
+    the tokens and C written transposed."""
+    if fa == "E5C2" and fb == "E4C3":
+        return narrow_model(b, sb, a, sa, fb, fa, G, Mt).T
+    return narrow_model(a, sa, b, sb, fa, fb, G, Mt)
+
+
+def _operand(rng, fmt, rows, K, G, spread=4):
     codes = rng.integers(0, 256, size=(rows, K), dtype=np.uint8)
     if fmt == "E3C3":
         codes &= 0xBF
-    return codes, rng.integers(-4, 5, size=(rows, K // G)).astype(np.int8)
+    return codes, rng.integers(-spread, spread + 1, size=(rows, K // G)).astype(np.int8)
 
 
-@pytest.mark.parametrize("fx,fw", PAIRS)
-@pytest.mark.parametrize("sparse", [False, True])
-def test_windows_reproduce_the_oracle(fx, fw, sparse):
-    if sparse and fx != fw:
-        pytest.skip("the sparse form is for same-format pairs")
-    rng = np.random.default_rng(len(fx) + 7 * len(fw) + sparse)
+@pytest.mark.parametrize("fa,fb", PAIRS)
+def test_windows_reproduce_the_oracle(fa, fb):
+    rng = np.random.default_rng(len(fa) + 7 * len(fb))
     G = 32
-    a, sa = _operand(rng, fx, 21, 128, G)  # 21 tokens: groups of 8, 8 and 5 (padding)
-    b, sb = _operand(rng, fw, 40, 128, G)
-    ref = oracle.gemm(a, sa, b, sb, fx, fw, G, phases=False)["C"]
-    got = narrow_model(a, sa, b, sb, fx, fw, G, 8, sparse)
+    a, sa = _operand(rng, fa, 21, 128, G)  # 21 tokens: groups of 8, 8 and 5 (padding)
+    b, sb = _operand(rng, fb, 40, 128, G)
+    if fa == "E5C2" and fb == "E5C2":
+        a[:, :] = np.where((fields(a, fa)[1] == -16) & (a & 0x7F != 0), a + 4, a)  # no lowest-binade tokens
+    ref = oracle.gemm(a, sa, b, sb, fa, fb, G, phases=False)["C"]
+    got = kernel_model(a, sa, b, sb, fa, fb, G, 8)
     assert np.abs(got - ref).max() <= 1e-12 * np.abs(ref).max()
 
 
+@pytest.mark.parametrize("fa,fb", PAIRS)
+def test_scale_spread_is_carried_by_the_factors(fa, fb):
+    """Block scales up to 30 binades apart along a row (beyond any FP8 plane range):
+    the factors carry them, and the model still matches the oracle."""
+    rng = np.random.default_rng(11 + len(fa))
+    G = 32
+    a, sa = _operand(rng, fa, 9, 256, G, spread=15)
+    b, sb = _operand(rng, fb, 24, 256, G, spread=15)
+    if fa == "E5C2" and fb == "E5C2":
+        a[:, :] = np.where((fields(a, fa)[1] == -16) & (a & 0x7F != 0), a + 4, a)
+    ref = oracle.gemm(a, sa, b, sb, fa, fb, G, phases=False)["C"]
+    got = kernel_model(a, sa, b, sb, fa, fb, G, 8)
+    na, nb = oracle.row_norms(a, sa, fa, G), oracle.row_norms(b, sb, fb, G)
+    assert (np.abs(got - ref) / np.outer(na, nb)).max() <= 1e-12
+
+
 def test_a_wrong_window_start_is_caught():
-    """The same model with each weight plane meeting the window one block off
-    (a plausible indexing slip) no longer matches the oracle."""
+    """The same model with each weight pair plane meeting the window one block
+    off (a plausible indexing slip) no longer matches the oracle."""
     rng = np.random.default_rng(3)
     a, sa = _operand(rng, "E4C3", 8, 64, 32)
     b, sb = _operand(rng, "E4C3", 16, 64, 32)
     ref = oracle.gemm(a, sa, b, sb, "E4C3", "E4C3", 32, phases=False)["C"]
-    kx, vx, rx = planes(a, sa, "E4C3", 32)
-    kw, vw, rw = planes(b, sb, "E4C3", 32)
+    kx, vx, cx, fxs, rx = planes(a, sa, "E4C3", 32, 0)
+    kw, vw, _, fws, rw = planes(b, sb, "E4C3", 32, 0)
     L, Mt = 8, 8
     Q = np.zeros((2 * L, Mt, 64))
     for u in range(L):
-        pl = np.where(kx == u, vx, 0.0)
-        Q[u], Q[L + u] = 2 * pl, pl
+        Q[u] = np.where(kx == u, cx, 0.0) * np.exp2(fxs)
+        Q[L + u] = np.where(kx == u, vx, 0.0) * np.exp2(fxs)
     D = np.zeros((16, L * Mt))
-    for k in range(L):
-        start = L - k + (1 if k else 0)  # one block off for every plane but the first
-        D += np.where(kw == k, vw, 0.0) @ Q[start: start + L].reshape(L * Mt, 64).T
+    for j in range(4):
+        A = np.zeros((16, 128))
+        A[:, 0::2] = np.where(kw == j, vw, 0.0) * np.exp2(fws)
+        A[:, 1::2] = np.where(kw == j + 4, vw, 0.0) * np.exp2(fws)
+        R = np.zeros((L, Mt, 128))
+        start = L - j + (1 if j else 0)  # one block off for every pair but the first
+        for h in range(L):
+            R[h, :, 0::2] = Q[(start + h) % (2 * L)]
+            R[h, :, 1::2] = Q[start + h - 4]
+        D += A @ R.reshape(L * Mt, 128).T
     S = D.reshape(-1, L, Mt)
-    C = np.einsum("h,whm->mw", np.exp2(np.arange(L) / L), S) * np.exp2((rx[:, None] + rw[None, :]).astype(float))
+    C = np.einsum("h,whm->mw", np.exp2(np.arange(L) / L), S) * np.exp2(
+        (rx[:, None] + rw[None, :] - 2 * MX_OFF).astype(float))
     assert np.abs(C - ref).max() > 1e-3 * np.abs(ref).max()
+
+
+# ---- byte-level emulation of the plane-byte arithmetic (tc_mx.cuh) ----------
+
+M32 = 0xFFFFFFFF
+
+
+def prmt_sign(v, sel):
+    """prmt.b32 r, v, 0, sel with sign replication (selector nibbles 8..B)."""
+    out = 0
+    for i in range(4):
+        nib = (sel >> (4 * i)) & 0xF
+        byte = (v >> (8 * (nib & 3))) & 0xFF
+        out |= (0xFF if byte & 0x80 else 0) << (8 * i)
+    return out
+
+
+def e5m2_pow2(x):
+    ge2 = prmt_sign((x + 0x7E7E7E7E) & M32, 0xBA98)
+    nrm = (((((x | 0x80808080) - 0x01010101) & 0x1F1F1F1F) << 2) & M32) & ge2
+    return nrm | ((x + 0x01010101) & ~ge2 & M32)
+
+
+def mx_word(w, fmt, bias):
+    E, C = FMTS[fmt]
+    mm = (0x3F if fmt == "E3C3" else 0x7F) * 0x01010101
+    sgn = w & 0x80808080
+    nz = prmt_sign(((w & mm) + 0x7F7F7F7F) & M32, 0xBA98)
+    eb = (w >> C) & (((1 << E) - 1) * 0x01010101)
+    if E < 5:
+        v = (sgn | (((eb + (15 - (1 << (E - 1))) * 0x01010101) << 2) & M32)) & nz
+        return v, (v + (nz & 0x04040404)) & M32
+    if bias == 0:
+        return (sgn | e5m2_pow2(eb)) & nz, 0
+    ge1 = prmt_sign((eb + 0x7F7F7F7F) & M32, 0xBA98)
+    x = ((eb | 0x80808080) - 0x01010101) & 0x1F1F1F1F
+    return (sgn | e5m2_pow2(x)) & nz & ge1, (sgn | e5m2_pow2(eb)) & nz
+
+
+def e5m2_value(byte):
+    s = -1.0 if byte & 0x80 else 1.0
+    ex, man = (byte >> 2) & 31, byte & 3
+    assert ex != 31, "no Inf/NaN plane bytes"
+    return s * (man * 2.0 ** -16 if ex == 0 else (1 + man / 4) * 2.0 ** (ex - 15))
+
+
+@pytest.mark.parametrize("fmt,bias", [("E3C3", 0), ("E4C3", 0), ("E5C2", 0), ("E5C2", 1)])
+def test_plane_bytes_of_every_code_in_every_lane(fmt, bias):
+    """Every code byte in every lane of a word (random neighbours): the plane
+    byte is exactly +-2^{e - bias} (0 for the zero codes and, with bias 1, for
+    e = -16), its carry byte +-2^{e - bias + 1}, and no lane disturbs
+    another."""
+    rng = np.random.default_rng(17)
+    valid = [c for c in range(256) if not (fmt == "E3C3" and c & 0x40)]
+    for c in valid:
+        m, e, _ = fields(np.array([c], np.uint8), fmt)
+        m, e = int(m[0]), int(e[0])
+        s = -1.0 if c & 0x80 else 1.0
+        want_v = 0.0 if m == 0 or e - bias < -16 else s * 2.0 ** (e - bias)
+        want_c = 0.0 if m == 0 else s * 2.0 ** (e - bias + 1)
+        for lane in range(4):
+            nb = rng.choice(valid, size=4)
+            nb[lane] = c
+            w = int(nb[0]) | int(nb[1]) << 8 | int(nb[2]) << 16 | int(nb[3]) << 24
+            v, vc = mx_word(w, fmt, bias)
+            assert e5m2_value((v >> (8 * lane)) & 0xFF) == want_v, (c, lane)
+            if fmt != "E5C2" or bias == 1:
+                assert e5m2_value((vc >> (8 * lane)) & 0xFF) == want_c, (c, lane)
