@@ -81,28 +81,25 @@ typedef enum {
 /* GEMM kernels.  EXACT: integer-ALU kernel whose per-phase sums are exact
  * integers (bit-identical to the definition).  TENSOR: tcgen05 tensor-core
  * kernel over power-of-two phase planes with FP32 per-phase accumulation, one
- * plane pair per dense MMA.  TENSOR_SPARSE: the same method with two plane
- * pairs per 2:4-sparse MMA (half the tensor work, more producer arithmetic;
- * code tiles streamed by TMA).  SKINNY: decode-sized GEMMs (M <=
- * CURVEFP_SKINNY_MAX_M) on the CUDA cores with the same FP32 per-phase
- * accumulation, every product formed from the two codes (the tensor-core
- * tile costs the same for any M up to 128).  TENSOR_NARROW: the tensor-core
- * method with the weight rows (B) as the 128-row operand and the L phases of
- * every token (row of A) along the MMA's N dimension (Sec. 3.2, Eq. 2,
- * Eq. 5): a step of 32 codes takes K_b MMAs of 128 x (L Mt) (Mt <= 256/L
- * tokens per CTA), and for same-format pairs K_b/2 2:4-sparse MMAs (weight
- * planes j and j + K_b/2 share one compressed operand), against K_a K_b MMAs
- * of a 128-row tile; the fastest tensor-core kernel at every M for
- * same-format pairs.
+ * plane pair per dense MMA of a 128-row tile.  SKINNY: decode-sized GEMMs
+ * (M <= CURVEFP_SKINNY_MAX_M) on the CUDA cores with the same FP32 per-phase
+ * accumulation, every product formed from the two codes.  TENSOR_NARROW: the
+ * tensor-core method with the weight rows as the 128-row operand and the L
+ * phases of every token (row) along the MMA's N dimension (Sec. 3.2, Eq. 2,
+ * Eq. 5): a step of 32 codes takes K_w/2 2:4-sparse MMAs of 128 x (L Mt)
+ * (weight curve planes j and j + K_w/2 share one compressed operand; Mt <=
+ * 256/L tokens per CTA), against K_a K_b dense MMAs of a 128-row tile; the
+ * fastest tensor-core kernel at every M.  In both tensor-core kernels the
+ * block scales enter the MMAs as UE8M0 scale factors (block-scaled MMAs), so
+ * the plane values are the codes' own powers of two.
  * AUTO (measured on the FFN shapes, N = 14336, K = 4096, and the
  * 2048 x 4096 x 4096 linear): SKINNY for M <= CURVEFP_AUTO_SKINNY_M;
  * TENSOR_NARROW for same-format pairs, and for the mixed pairs up to
  * CURVEFP_AUTO_NARROW_M; TENSOR above; SKINNY up to CURVEFP_SKINNY_MAX_M for
- * pairs without a tensor-core kernel. */
+ * pairs without a tensor-core kernel.  (Value 2 is not an algorithm.) */
 typedef enum {
   CURVEFP_GEMM_EXACT = 0,
   CURVEFP_GEMM_TENSOR = 1,
-  CURVEFP_GEMM_TENSOR_SPARSE = 2,
   CURVEFP_GEMM_SKINNY = 3,
   CURVEFP_GEMM_AUTO = 4,
   CURVEFP_GEMM_TENSOR_NARROW = 5
@@ -212,13 +209,25 @@ curvefp_status_t curvefp_dequantize(curvefp_format_t fmt, int block, const uint8
  * Requirements: K % block == 0; a, b 16-byte aligned.
  * EXACT: S_h exact, combine in FP64, one FP32 rounding; outputs whose scale
  *   spread leaves the int128 window raise CURVEFP_DEV_RANGE (values undefined).
- * TENSOR, TENSOR_SPARSE, TENSOR_NARROW: S_h accumulated in FP32 on the
- *   tensor cores, combine in FP32; plane values below 2^-14 of a row's largest
- *   block scale flush.  Format pairs: E3C3 x E3C3, E4C3 x E4C3, E5C2 x E4C3,
- *   E4C3 x E5C2, E5C2 x E5C2, and (TENSOR) E4C3_R8_9 x E4C3_R8_9 (others
- *   return CURVEFP_ERR_UNSUPPORTED).  TENSOR and TENSOR_NARROW zero parts of C
- *   with cudaMemsetAsync before adding split-K pieces to them (two additions
- *   per output, so results do not depend on their order).
+ * TENSOR, TENSOR_NARROW: S_h accumulated in FP32 on the tensor cores, combine
+ *   in FP32.  Every product is exact before the FP32 accumulation: a plane
+ *   value is the code's power of two 2^e and the block scale is the MMA's
+ *   scale factor 2^{a_b - ref + 32} (ref = the row's largest block scale),
+ *   so the spread of the block scales along a row costs nothing.  Lost are
+ *   only (1) products below FP32's normal range, i.e. below 2^{-190} of
+ *   2^{ref_a + ref_b}; (2) blocks more than 159 binades below their row's
+ *   largest block scale; (3) TENSOR_NARROW with E5C2 x E5C2: the tokens'
+ *   elements of the lowest binade (e = -16) in the products without carry
+ *   (an element at least 2^30 below its block's top binade).  Within 1e-5 of
+ *   ||a_i|| ||b_j|| whenever, per row, the largest element lies within about
+ *   75 binades of the row's largest block scale on both operands (the
+ *   quantizer writes 0 as the scale of an all-zero block, so this holds
+ *   unless both operands' data lie below about 2^-75).  Format pairs: E3C3 x
+ *   E3C3, E4C3 x E4C3, E5C2 x E4C3, E4C3 x E5C2, E5C2 x E5C2, and (TENSOR)
+ *   E4C3_R8_9 x E4C3_R8_9 (others return CURVEFP_ERR_UNSUPPORTED).  TENSOR and
+ *   TENSOR_NARROW zero parts of C with cudaMemsetAsync before adding split-K
+ *   pieces to them (two additions per output, so results do not depend on
+ *   their order).
  * SKINNY (M <= CURVEFP_SKINNY_MAX_M, else CURVEFP_ERR_UNSUPPORTED), AUTO:
  *   S_h accumulated in FP32 per output (products relative to the output's
  *   largest scale sum; products below the FP32 normal range relative to it
@@ -256,7 +265,8 @@ typedef enum { CURVEFP_LAYOUT_ROWS = 0, CURVEFP_LAYOUT_COLS = 1 } curvefp_layout
 
 /* Bytes of device workspace curvefp_gemm_oriented needs (0 for EXACT and for
  * ROWS x ROWS); for TENSOR with a COLS operand:
- *   sum over operands of [R K (COLS only)] + R K + 4 R, each rounded up to 256. */
+ *   sum over operands of [R K (COLS only)] + R K + R K / 16 + 4 R, each
+ *   rounded up to 256. */
 size_t curvefp_gemm_oriented_workspace_bytes(curvefp_gemm_algo_t algo, curvefp_layout_t layout_a,
                                              curvefp_layout_t layout_b, int64_t M, int64_t N, int64_t K);
 
@@ -267,15 +277,17 @@ size_t curvefp_gemm_oriented_workspace_bytes(curvefp_gemm_algo_t algo, curvefp_l
  *   EXACT : integer ALUs, phase sums bit-identical to the definition;
  *           phase_sums / phase_lsb as curvefp_gemm_phases (both or neither);
  *           c may be NULL when phase_sums is given.  No workspace.
- *   TENSOR: the tensor-core kernel with per-element scales (tolerance and
- *           flush rule as curvefp_gemm TENSOR, the reference exponent of a
- *           row being its largest element scale); phase_sums and phase_lsb
- *           must be NULL; K % 32 == 0; workspace (256-byte aligned, at least
- *           curvefp_gemm_oriented_workspace_bytes) receives the transposed
- *           codes of COLS operands and a relative-scale byte per element,
- *           written by preparation kernels on the same stream.  ROWS x ROWS
- *           is curvefp_gemm (no workspace).
- *   TENSOR_SPARSE: ROWS x ROWS only (CURVEFP_ERR_UNSUPPORTED otherwise).
+ *   TENSOR: the tensor-core kernel with per-element scales: per 32-code step
+ *           of a row the scale factor follows the step's largest element and
+ *           each element's plane value is its power of two relative to it;
+ *           an element more than 31 binades below the largest element of
+ *           its step (2^-31 of it) is dropped, so the error bound is
+ *           2^-31 sqrt(K) ||a_i|| ||b_j|| beyond curvefp_gemm TENSOR's;
+ *           phase_sums and phase_lsb must be NULL; K % 32 == 0; workspace
+ *           (256-byte aligned, at least curvefp_gemm_oriented_workspace_bytes)
+ *           receives the transposed codes of COLS operands, an exponent byte
+ *           per element and a scale per step, written by preparation kernels
+ *           on the same stream.  ROWS x ROWS is curvefp_gemm (no workspace).
  * Codes pointers 16-byte aligned; M, N, K > 0. */
 curvefp_status_t curvefp_gemm_oriented(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, curvefp_format_t fmt_b,
                                        int block, const uint8_t* a, const int8_t* sa, curvefp_layout_t layout_a,

@@ -15,7 +15,7 @@ from . import _build
 # E4C3_R8_9 / E4C3_R3_4: E4C3 codes with the rational radices 2^{8/9}, 2^{3/4}
 FORMATS = {"E3C3": 0, "E4C3": 1, "E5C2": 2, "E4C3_R8_9": 3, "E4C3_R3_4": 4}
 DTYPES = {"f32": 0, "bf16": 1}
-ALGOS = {"exact": 0, "tensor": 1, "tensor_sparse": 2, "skinny": 3, "auto": 4, "tensor_narrow": 5}
+ALGOS = {"exact": 0, "tensor": 1, "skinny": 3, "auto": 4, "tensor_narrow": 5}
 STATUS_BITS = {"nan": 1, "range": 2, "timeout": 4}
 
 _lib = None

@@ -174,10 +174,8 @@ curvefp_status_t curvefp_gemm(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, 
     return from_cuda(cfp::launch_gemm_tensor_narrow(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, device_status, st,
                                                     sm_count()));
   }
-  if (algo == CURVEFP_GEMM_TENSOR || algo == CURVEFP_GEMM_TENSOR_SPARSE) {
+  if (algo == CURVEFP_GEMM_TENSOR) {
     if (!cfp::gemm_tensor_supported(fmt_a, fmt_b)) return CURVEFP_ERR_UNSUPPORTED;
-    if (algo == CURVEFP_GEMM_TENSOR_SPARSE)
-      return from_cuda(cfp::launch_gemm_tensor_sparse(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, device_status, st));
     return from_cuda(cfp::launch_gemm_tensor(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, device_status, st,
                                              sm_count()));
   }
@@ -236,7 +234,6 @@ curvefp_status_t curvefp_gemm_oriented(curvefp_gemm_algo_t algo, curvefp_format_
   if (phase_sums || phase_lsb || !c) return CURVEFP_ERR_INVALID_ARG;
   if (layout_a == CURVEFP_LAYOUT_ROWS && layout_b == CURVEFP_LAYOUT_ROWS)
     return curvefp_gemm(algo, fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, device_status, stream);
-  if (algo == CURVEFP_GEMM_TENSOR_SPARSE) return CURVEFP_ERR_UNSUPPORTED;
   if (algo != CURVEFP_GEMM_TENSOR) return CURVEFP_ERR_INVALID_ARG;
   if (!cfp::gemm_tensor_supported(fmt_a, fmt_b)) return CURVEFP_ERR_UNSUPPORTED;
   if (K % 32 != 0) return CURVEFP_ERR_INVALID_ARG;

@@ -4,13 +4,18 @@
 // A COLS operand is a [K x R] code matrix quantized along R (scales [K x R/G])
 // that the GEMM reads as R rows of K codes: the scale of an element follows
 // the element, so along a GEMM row it changes with k.  The tensor-core path
-// handles that with per-element scales in the producers (gemm_tc.cuh, PES):
-// every operand gets a byte per element holding its scale relative to the row
-// reference, dp = max(a - ref, -64) + 64 (elements 64 binades below the
-// reference flush in any case), and a COLS operand's codes are transposed once
-// into K-contiguous rows.  Both are written into the caller's workspace by the
-// preparation kernels below, which stream the operand once (HBM-bound: R K
-// bytes read, 2 R K written for a COLS operand, R K for a ROWS operand).
+// handles that with per-element exponents (gemm_tc.cuh, PES): for every
+// 32-code step of a GEMM row the preparation kernels below find the largest
+// element exponent x = a + e over the step's nonzero codes, store
+// f = that maximum - 15 as the step's scale (it becomes the step's UE8M0
+// factor 2^{f - ref + 32}, ref = max over the row's steps) and, per element,
+// the plane exponent x - f + 16 in [0, 31] (0x80 for zero codes and for the
+// elements more than 31 binades below the step's largest one, whose plane
+// value 2^{x - f} would leave E5M2).  A COLS operand's codes are transposed
+// once into K-contiguous rows.  Everything goes into the caller's workspace;
+// the kernels stream the operand once (HBM-bound: R K bytes read, 2 R K
+// written for a COLS operand, R K for a ROWS operand, plus 2 R K / 32 bytes
+// of step scales).
 #include "gemm_tc.cuh"
 
 namespace cfp {
@@ -18,61 +23,87 @@ namespace cfp {
 namespace {
 
 constexpr int TT = 64;  // transpose tile (codes), 64 x 64 bytes
+constexpr int16_t NO_STEP = -32768;
 
-// ROWS operand: ref[r] = max_b s[r][b].
-__global__ void pes_ref_rows_kernel(const int8_t* __restrict__ s, int64_t R, int nb, int* __restrict__ ref) {
-  const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (r >= R) return;
-  int m = -128;
-  for (int b = 0; b < nb; ++b) m = max(m, (int)__ldg(s + r * nb + b));
-  ref[r] = m;
+// e + 2^{E-1} of a code byte (zero codes: -1).
+template <int FMT>
+__device__ __forceinline__ int biased_exp(uint32_t code) {
+  const uint32_t m = code & (uint32_t)Fmt<FMT>::MMASK;
+  return m ? (int)(m >> Fmt<FMT>::C) : -1;
 }
 
-// COLS operand: ref[q] = max_k s[k][q] over the block column q < nq (ref is
-// preset to INT_MIN-like 0x80808080).  Block: 32 columns x 8 row lanes, rows
-// [blockIdx.y * KCH, +KCH).
-constexpr int KCH = 256;
-__global__ void pes_ref_cols_kernel(const int8_t* __restrict__ s, int64_t K, int nq, int* __restrict__ ref) {
-  const int q = blockIdx.x * 32 + (threadIdx.x & 31);
-  if (q >= nq) return;
-  const int64_t k0 = (int64_t)blockIdx.y * KCH;
-  const int64_t k1 = min(K, k0 + KCH);
-  int m = -128;
-  for (int64_t k = k0 + (threadIdx.x >> 5); k < k1; k += 8) m = max(m, (int)__ldg(s + k * nq + q));
-  atomicMax(ref + q, m);
-}
-
-__device__ __forceinline__ uint32_t rel_byte(int a, int ref) {
-  const int d = a - ref;
-  return (uint32_t)((d < -64 ? -64 : d) + 64);
-}
-
-// ROWS operand: dp[r][k] = rel(s[r][k >> gsh], ref[r]); 16 bytes per thread
-// (G >= 32, so one scale per 16-byte run).
-__global__ void pes_dp_rows_kernel(const int8_t* __restrict__ s, const int* __restrict__ ref, int64_t R, int64_t K,
-                                   int gsh, uint8_t* __restrict__ dp) {
-  const int64_t per_row = K / 16;
-  const int64_t n = R * per_row;
-  const int64_t nb = K >> gsh;
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t r = i / per_row, k = (i - r * per_row) * 16;
-    const uint32_t v = rel_byte((int)__ldg(s + r * nb + (k >> gsh)), __ldg(ref + r)) * 0x01010101u;
-    *reinterpret_cast<uint4*>(dp + r * K + k) = make_uint4(v, v, v, v);
+// Exponent bytes of the 16 codes of a half step (scales a[i], the step's
+// largest exponent xmax over both halves, exchanged with the partner lane
+// `pmask`), and the step scale f = xmax - 15 (NO_STEP when all 32 are zero).
+template <int FMT>
+__device__ __forceinline__ void half_step_bytes(const uint32_t (&c)[16], const int (&a)[16], unsigned pmask,
+                                                uint32_t (&dp)[4], int& f) {
+  constexpr int EB = 1 << (Fmt<FMT>::E - 1);
+  int x[16], xm = -100000;
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    const int eb = biased_exp<FMT>(c[i]);
+    x[i] = eb < 0 ? -100000 : a[i] + eb - EB;
+    xm = max(xm, x[i]);
+  }
+  xm = max(xm, __shfl_xor_sync(pmask, xm, 1));
+  f = xm < -50000 ? NO_STEP : xm - 15;
+#pragma unroll
+  for (int w = 0; w < 4; ++w) {
+    uint32_t d = 0;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int b = x[4 * w + j] - (xm - 15) + 16;  // plane exponent + 16
+      d |= (uint32_t)(b >= 0 && b <= 31 && x[4 * w + j] > -50000 ? b : 0x80) << (8 * j);
+    }
+    dp[w] = d;
   }
 }
 
-// COLS operand: codes [K x R] -> codesT [R x K] and dp [R x K] with
-// dp[r][k] = rel(s[k][r >> gsh], ref[r >> gsh]).  One 64 x 64 tile per CTA
-// (256 threads, 16 bytes per thread each way); R % 32 == 0 and K % 16 == 0,
-// so every 16-byte run is wholly inside or outside the matrix.
-__global__ void __launch_bounds__(256) pes_transpose_cols_kernel(const uint8_t* __restrict__ codes,
-                                                                 const int8_t* __restrict__ s,
-                                                                 const int* __restrict__ refq, int64_t R, int64_t K,
-                                                                 int gsh, uint8_t* __restrict__ codesT,
-                                                                 uint8_t* __restrict__ dp) {
+// ROWS operand (codes [R x K], scales [R x K/G]): a lane pair per 32-code
+// step, 16 codes per lane.
+template <int FMT>
+__global__ void pes_rows_kernel(const uint8_t* __restrict__ codes, const int8_t* __restrict__ s, int64_t R, int64_t K,
+                                int gsh, uint8_t* __restrict__ dp, int16_t* __restrict__ fst, int* __restrict__ ref) {
+  const int64_t per_row = K / 16;
+  const int64_t n = R * per_row;
+  const int64_t nb = K >> gsh;
+  const unsigned pmask = 3u << ((threadIdx.x & 31) & ~1u);
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = i / per_row, k = (i - r * per_row) * 16;
+    const uint4 q = __ldg(reinterpret_cast<const uint4*>(codes + r * K + k));
+    const int sc = (int)__ldg(s + r * nb + (k >> gsh));
+    const uint32_t wv[4] = {q.x, q.y, q.z, q.w};
+    uint32_t c[16];
+    int a[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      c[j] = (wv[j >> 2] >> (8 * (j & 3))) & 0xFFu;
+      a[j] = sc;
+    }
+    uint32_t d[4];
+    int f;
+    half_step_bytes<FMT>(c, a, pmask, d, f);
+    *reinterpret_cast<uint4*>(dp + r * K + k) = make_uint4(d[0], d[1], d[2], d[3]);
+    if ((i & 1) == 0) {
+      fst[r * (K / 32) + (k >> 5)] = (int16_t)f;
+      if (f != NO_STEP) atomicMax(ref + r, f);
+    }
+  }
+}
+
+// COLS operand: codes [K x R] -> codesT [R x K], with the exponent bytes and
+// step scales of the transposed rows.  One 64 x 64 tile per CTA (256
+// threads, 16 bytes per thread each way; lanes 2t and 2t + 1 hold the two
+// halves of a 32-code step); R % 32 == 0 and K % 32 == 0, so every step is
+// wholly inside or outside the matrix.
+template <int FMT>
+__global__ void __launch_bounds__(256) pes_cols_kernel(const uint8_t* __restrict__ codes, const int8_t* __restrict__ s,
+                                                       int64_t R, int64_t K, int gsh, uint8_t* __restrict__ codesT,
+                                                       uint8_t* __restrict__ dp, int16_t* __restrict__ fst,
+                                                       int* __restrict__ ref) {
   __shared__ uint32_t tile[TT][TT / 4 + 1];  // [k][r / 4], one padding word per row
   __shared__ int8_t ts[TT][2];               // scales of the tile's (at most two) block columns
-  __shared__ int tref[2];
   const int64_t r0 = (int64_t)blockIdx.x * TT, k0 = (int64_t)blockIdx.y * TT;
   const int nq = (int)(R >> gsh);
   const int q0 = (int)(r0 >> gsh);
@@ -89,30 +120,33 @@ __global__ void __launch_bounds__(256) pes_transpose_cols_kernel(const uint8_t* 
       const int k2 = t >> 1, qq = t & 1;
       ts[k2][qq] = (k0 + k2 < K && q0 + qq < nq) ? __ldg(s + (k0 + k2) * nq + q0 + qq) : (int8_t)-128;
     }
-    if (t < 2) tref[t] = q0 + t < nq ? __ldg(refq + q0 + t) : 0;
   }
   __syncthreads();
   const int rr = t >> 2, seg = t & 3;
   const int64_t r = r0 + rr, k = k0 + seg * 16;
-  if (r >= R || k >= K) return;
+  if (r >= R || k >= K) return;  // a lane pair leaves together
   const int qq = (int)(r >> gsh) - q0;
-  const int ref = tref[qq];
-  uint32_t c[4], d[4];
+  const unsigned pmask = 3u << ((threadIdx.x & 31) & ~1u);
+  uint32_t c[16];
+  int a[16];
 #pragma unroll
-  for (int w = 0; w < 4; ++w) {
-    uint32_t cw = 0, dw = 0;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int kk = seg * 16 + w * 4 + j;
-      const uint32_t byte = (tile[kk][rr >> 2] >> (8 * (rr & 3))) & 0xFFu;
-      cw |= byte << (8 * j);
-      dw |= rel_byte(ts[kk][qq], ref) << (8 * j);
-    }
-    c[w] = cw;
-    d[w] = dw;
+  for (int j = 0; j < 16; ++j) {
+    const int kk = seg * 16 + j;
+    c[j] = (tile[kk][rr >> 2] >> (8 * (rr & 3))) & 0xFFu;
+    a[j] = ts[kk][qq];
   }
-  *reinterpret_cast<uint4*>(codesT + r * K + k) = make_uint4(c[0], c[1], c[2], c[3]);
+  uint32_t d[4];
+  int f;
+  half_step_bytes<FMT>(c, a, pmask, d, f);
+  uint32_t cw[4];
+#pragma unroll
+  for (int w = 0; w < 4; ++w) cw[w] = c[4 * w] | c[4 * w + 1] << 8 | c[4 * w + 2] << 16 | c[4 * w + 3] << 24;
+  *reinterpret_cast<uint4*>(codesT + r * K + k) = make_uint4(cw[0], cw[1], cw[2], cw[3]);
   *reinterpret_cast<uint4*>(dp + r * K + k) = make_uint4(d[0], d[1], d[2], d[3]);
+  if ((seg & 1) == 0) {
+    fst[r * (K / 32) + (k >> 5)] = (int16_t)f;
+    if (f != NO_STEP) atomicMax(ref + r, f);
+  }
 }
 
 int log2i(int g) {
@@ -123,20 +157,22 @@ int log2i(int g) {
 
 size_t al256(size_t v) { return (v + 255) & ~(size_t)255; }
 
-// Workspace of one operand: [codesT (COLS only)] [dp] [ref].
+// Workspace of one operand: [codesT (COLS only)] [dp] [step scales] [ref].
 size_t operand_ws(int layout, int64_t R, int64_t K) {
-  return (layout == CURVEFP_LAYOUT_COLS ? al256((size_t)R * K) : 0) + al256((size_t)R * K) + al256((size_t)R * 4);
+  return (layout == CURVEFP_LAYOUT_COLS ? al256((size_t)R * K) : 0) + al256((size_t)R * K) +
+         al256((size_t)R * (K / 32) * 2) + al256((size_t)R * 4);
 }
 
 struct Prepared {
   const uint8_t* codes;
   const uint8_t* dp;
+  const int16_t* f;
   const int* ref;
-  int rsh;
 };
 
-cudaError_t prepare(int layout, const uint8_t* codes, const int8_t* s, int64_t R, int64_t K, int G, uint8_t* ws,
-                    cudaStream_t st, Prepared& out) {
+template <int FMT>
+cudaError_t prepare_t(int layout, const uint8_t* codes, const int8_t* s, int64_t R, int64_t K, int G, uint8_t* ws,
+                      cudaStream_t st, Prepared& out) {
   const int gsh = log2i(G);
   uint8_t* p = ws;
   uint8_t* codesT = nullptr;
@@ -146,25 +182,31 @@ cudaError_t prepare(int layout, const uint8_t* codes, const int8_t* s, int64_t R
   }
   uint8_t* dp = p;
   p += al256((size_t)R * K);
+  int16_t* f = reinterpret_cast<int16_t*>(p);
+  p += al256((size_t)R * (K / 32) * 2);
   int* ref = reinterpret_cast<int*>(p);
+  cudaError_t e = cudaMemsetAsync(ref, 0x80, (size_t)R * 4, st);  // 0x80808080: below every step scale
+  if (e != cudaSuccess) return e;
   if (layout == CURVEFP_LAYOUT_ROWS) {
-    pes_ref_rows_kernel<<<(unsigned)((R + 255) / 256), 256, 0, st>>>(s, R, (int)(K >> gsh), ref);
     const int64_t n16 = R * (K / 16);
     const int64_t want = (n16 + 255) / 256;
     const unsigned blocks = (unsigned)(want < 152 * 16 ? (want > 0 ? want : 1) : 152 * 16);
-    pes_dp_rows_kernel<<<blocks, 256, 0, st>>>(s, ref, R, K, gsh, dp);
-    out = Prepared{codes, dp, ref, 0};
+    pes_rows_kernel<FMT><<<blocks, 256, 0, st>>>(codes, s, R, K, gsh, dp, f, ref);
+    out = Prepared{codes, dp, f, ref};
   } else {
-    const int nq = (int)(R >> gsh);
-    cudaError_t e = cudaMemsetAsync(ref, 0x80, (size_t)nq * 4, st);
-    if (e != cudaSuccess) return e;
-    dim3 g1((unsigned)((nq + 31) / 32), (unsigned)((K + KCH - 1) / KCH));
-    pes_ref_cols_kernel<<<g1, 256, 0, st>>>(s, K, nq, ref);
     dim3 g2((unsigned)((R + TT - 1) / TT), (unsigned)((K + TT - 1) / TT));
-    pes_transpose_cols_kernel<<<g2, 256, 0, st>>>(codes, s, ref, R, K, gsh, codesT, dp);
-    out = Prepared{codesT, dp, ref, gsh};
+    pes_cols_kernel<FMT><<<g2, 256, 0, st>>>(codes, s, R, K, gsh, codesT, dp, f, ref);
+    out = Prepared{codesT, dp, f, ref};
   }
   return cudaGetLastError();
+}
+
+cudaError_t prepare(int fmt, int layout, const uint8_t* codes, const int8_t* s, int64_t R, int64_t K, int G,
+                    uint8_t* ws, cudaStream_t st, Prepared& out) {
+  if (fmt == CURVEFP_E3C3) return prepare_t<CURVEFP_E3C3>(layout, codes, s, R, K, G, ws, st, out);
+  if (fmt == CURVEFP_E4C3) return prepare_t<CURVEFP_E4C3>(layout, codes, s, R, K, G, ws, st, out);
+  if (fmt == CURVEFP_E5C2) return prepare_t<CURVEFP_E5C2>(layout, codes, s, R, K, G, ws, st, out);
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace
@@ -179,14 +221,13 @@ cudaError_t launch_gemm_tensor_reuse(int fa, int fb, int G, const uint8_t* a, co
                                      float* c, void* ws, uint32_t* status, cudaStream_t s, int sms) {
   uint8_t* w = static_cast<uint8_t*>(ws);
   Prepared pa, pb;
-  cudaError_t e = prepare(la, a, sa, M, K, G, w, s, pa);
+  cudaError_t e = prepare(fa, la, a, sa, M, K, G, w, s, pa);
   if (e != cudaSuccess) return e;
-  e = prepare(lb, b, sb, N, K, G, w + operand_ws(la, M, K), s, pb);
+  e = prepare(fb, lb, b, sb, N, K, G, w + operand_ws(la, M, K), s, pb);
   if (e != cudaSuccess) return e;
-  const PesOperands pes{pa.dp, pb.dp, pa.ref, pb.ref, pa.rsh, pb.rsh};
-  constexpr int PT = PLANE_E5M2;
+  const PesOperands pes{pa.dp, pb.dp, pa.f, pb.f, pa.ref, pb.ref};
 #define CFP_R(X, Y) \
-  if (fa == X && fb == Y) return launch_tc_t<X, Y, PT, true>(G, pa.codes, nullptr, pb.codes, nullptr, M, N, K, c, status, s, pes, sms);
+  if (fa == X && fb == Y) return launch_tc_t<X, Y, true>(G, pa.codes, nullptr, pb.codes, nullptr, M, N, K, c, status, s, pes, sms);
   CFP_R(CURVEFP_E3C3, CURVEFP_E3C3)
   CFP_R(CURVEFP_E4C3, CURVEFP_E4C3)
   CFP_R(CURVEFP_E5C2, CURVEFP_E4C3)

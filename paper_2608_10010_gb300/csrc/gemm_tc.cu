@@ -13,9 +13,8 @@ bool gemm_tensor_supported(int fa, int fb) {
 cudaError_t launch_gemm_tensor(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
                                const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, uint32_t* status,
                                cudaStream_t s, int sms) {
-  constexpr int PT = CFP_TC_PLANE;
 #define CFP_T(X, Y) \
-  if (fa == X && fb == Y) return launch_tc_t<X, Y, PT, false>(G, a, sa, b, sb, M, N, K, c, status, s, PesOperands{}, sms);
+  if (fa == X && fb == Y) return launch_tc_t<X, Y, false>(G, a, sa, b, sb, M, N, K, c, status, s, PesOperands{}, sms);
   CFP_T(CURVEFP_E3C3, CURVEFP_E3C3)
   CFP_T(CURVEFP_E4C3, CURVEFP_E4C3)
   CFP_T(CURVEFP_E5C2, CURVEFP_E4C3)

@@ -3,38 +3,42 @@
 // combine fused into the epilogue (Sec. 3.2, Eq. 2, Eq. 5).
 //
 // Decomposition.  Write every decoded operand element as
-//   x = 2^{k/K} * X_k,   X_k = +-2^{a_b - ref + e}  (an exact power of two),
+//   x = 2^{a_b} 2^{k/K} X_k,   X_k = +-2^e  (an exact power of two),
 // i.e. split each operand into K "curve planes" that hold the element in the
 // plane of its curve index k and zero elsewhere.  Plane k1 of A times plane k2
 // of B lands on the single phase h = (k1 WA + k2 WB) mod L with carry
 // c = floor((k1 WA + k2 WB) / L) (Eq. 2 on the shared lattice L), so
 //   S_h = sum_{k1,k2 : phase h} 2^c  A_{k1} B_{k2}^T,
 // a sum of dense products of power-of-two matrices, which the tensor cores
-// multiply without rounding; only the FP32 accumulation in TMEM rounds.  Block
-// scales enter the plane values as 2^{a_b - ref} (ref = largest block scale of
-// the row) and 2^{ref_i + ref_j} is applied in the epilogue.  Plane values are
-// BF16 or FP8 E5M2 (every power of two in [2^-16, 2^15] is exact in E5M2; E5C2
-// planes are stored one binade low so that the carry still fits).
+// multiply without rounding; only the FP32 accumulation in TMEM rounds.
 //
-// Shape.  A CTA owns a 128 x 96 tile of C.  A 128 x 96 x 32 FP8 MMA runs at
-// the full tensor rate (the per-instruction floor is ~45 cycles, this shape
-// takes 48); TMEM (512 columns) holds four 96-column phase accumulators plus
-// two steps of A planes, so the L phases are processed in passes of PP = 4
-// phases over the whole K; each pass adds its part of sum_h 2^{h/L} S_h to C.
+// Block scales are UE8M0 scale factors of a block-scaled MMA
+// (tcgen05.mma .kind::mxf8f6f4 .block_scale, tc_mx.cuh): 2^{a_b - ref + 32}
+// per row and 32-code step (ref = the row's largest block scale), so every
+// product is exact whatever the spread of the scales along a row, and the
+// carry 2^c is the second factor byte of the B row (2^{a_b - ref + 33}): the
+// B planes are stored once, not in plain and doubled copies.  The epilogue
+// applies 2^{ref_i + ref_j - 64}.  Plane values are FP8 E5M2 (every code of
+// the binary formats and of E4C3 with r = 2^{8/9} has an exact one).
 //
-// Roles (480 threads):
+// Shape.  A CTA owns a 128 x BN tile of C: BN = 96 (a 128 x 96 x 32 FP8 MMA
+// runs at the full tensor rate) where TMEM holds PP phase accumulators of BN
+// columns, two steps of A planes and the scale factors, else 80.  The L
+// phases are processed in passes of PP phases over the whole K; each pass
+// adds its part of sum_h 2^{h/L} S_h to an FP32 stash, the last writes C.
+//
+// Roles:
 //   warps 0-7   A producers (two threads per row, 16 codes each per step):
-//               codes -> planes in registers -> TMEM (tcgen05.st); A is the
-//               TMEM operand of the MMA and costs no shared-memory bandwidth.
-//               At the end of each pass they run the epilogue.
-//   warps 8-13  B producers (two threads per row): codes -> the planes (and
-//               x2 carry planes) that the current pass needs -> shared memory,
-//               K-major core-matrix layout.
-//   warp 14     TMEM allocation and MMA issue (one elected lane of the
-//               converged warp).
-// One mbarrier hand-off per pipeline step and operand: every wait and commit
-// sits on the path between two MMAs, so the stages are whole steps.  Every
-// wait is bounded.
+//               codes -> planes in registers -> TMEM (tcgen05.st), and the
+//               row's scale factor; at the end of each pass the epilogue.
+//   next warps  B producers (two threads per row): codes -> the planes that
+//               the current pass needs -> shared memory, K-major core-matrix
+//               layout; the row's factor bytes -> the stage's factor block.
+//   last warp   TMEM allocation, factor copies (tcgen05.cp) and MMA issue
+//               (one elected lane of the converged warp).
+// One mbarrier hand-off per pipeline step: every wait and commit sits on the
+// path between two MMAs, so the stages are whole steps.  Every wait is
+// bounded.
 #pragma once
 #include <functional>
 #include <mutex>
@@ -44,16 +48,9 @@
 
 #include "cfp_common.cuh"
 #include "kernels.cuh"
+#include "tc_mx.cuh"
 #include "tc_planes.cuh"
 #include "tc_ptx.cuh"
-
-#ifndef CFP_TC_ATPR
-#define CFP_TC_ATPR 2  // A producer threads per row (2 or 4)
-#endif
-
-#ifndef CFP_TC_PLANE
-#define CFP_TC_PLANE 1  // 0: BF16 planes (K = 16 per MMA), 1: E5M2 planes (K = 32 per MMA)
-#endif
 
 namespace cfp {
 
@@ -72,63 +69,59 @@ struct TcLattice<CURVEFP_E4C3_R8_9, CURVEFP_E4C3_R8_9> {
   static constexpr int KA = 9, KB = 9, L = 9, WA = 1, WB = 1;
 };
 
-template <int FA, int FB, int PT>
+template <int FA, int FB>
 struct TcCfg {
   using T = TcLattice<FA, FB>;
   static constexpr int KA = T::KA, KB = T::KB, L = T::L, WA = T::WA, WB = T::WB;
   static constexpr int FA_ = FA, FB_ = FB;
   static constexpr int BM = 128;
-  static constexpr int KS = PT == PLANE_BF16 ? 16 : 32;  // K per MMA = K per pipeline step (32 bytes per row)
-  // Columns per CTA (= MMA N) and phases per pass: 4 accumulators of 96
-  // columns leave 128 TMEM columns for A; N = 96 still runs the MMA at full
-  // rate (the per-instruction floor is ~45 cycles, a 128x96x32 FP8 MMA is 48).
-  static constexpr int BN = 96;
+  static constexpr int KS = 32;                           // K per MMA = K per pipeline step (one factor)
   static constexpr int PP = L == 9 ? 3 : 4;               // phases per pass
   static constexpr int NP = (L + PP - 1) / PP;            // passes
-  static constexpr int ACC_COLS = PP * BN;
   // A planes of a step occupy AU_COLS TMEM columns (8 per plane); two steps
-  // rotate (NAU units).
+  // rotate (NAU units)
   static constexpr int AU_COLS = KA * 8;
   static constexpr int NAU = 2;
-  static constexpr int ACOL0 = ACC_COLS;
-  static_assert(ACC_COLS + NAU * AU_COLS <= 512, "TMEM budget");
-  static constexpr int PLANE_BYTES = BN * 32;             // 128 rows x 32 bytes
   static constexpr int NSB = 4;                           // B stages
-  static constexpr int PBA = FA == CURVEFP_E5C2 ? 1 : 0;  // plane exponent bias
-  static constexpr int PBB = FB == CURVEFP_E5C2 ? 1 : 0;
-  static constexpr int ATPR = CFP_TC_ATPR;                // A producer threads per row
+  // TMEM: PP accumulators of BN columns, the A units, A factors (4 columns
+  // per unit: quadrant q reads column q) and B factors (4 columns per stage)
+  static constexpr int SF_COLS = NAU * 4 + NSB * 4;
+  static constexpr int BN = PP * 96 + NAU * AU_COLS + SF_COLS <= 512 ? 96 : 80;
+  static constexpr int ACC_COLS = PP * BN;
+  static constexpr int ACOL0 = ACC_COLS;
+  static constexpr int SFA0 = ACOL0 + NAU * AU_COLS;
+  static constexpr int SFB0 = SFA0 + NAU * 4;
+  static_assert(SFB0 + NSB * 4 <= 512, "TMEM budget");
+  static constexpr int PLANE_BYTES = BN * 32;             // BN rows x 32 bytes
+  static constexpr int ATPR = 2;                          // A producer threads per row
   static constexpr int NAW = 4 * ATPR;                    // A producer warps (4 TMEM lane groups)
   static constexpr int NWA = 8 / ATPR;                    // TMEM columns per A thread and plane
   static constexpr int NBT = 2 * BN;                      // B producer threads (two per row)
   static constexpr int THREADS = NAW * 32 + NBT + 32;     // A producers, B producers, MMA warp
   static constexpr int MMA_WARP = (NAW * 32 + NBT) / 32;
-  static_assert(NBT % 32 == 0 && BN % (8 * ATPR) == 0 && 8 % ATPR == 0, "producer warps");
-  // D = F32, A = B = BF16 (kind::f16) or E5M2 (kind::f8f6f4): same bit pattern
-  static constexpr uint32_t IDESC = tc::idesc_bf16_f32(BM, BN);
+  static_assert(NBT % 32 == 0 && BN % (8 * ATPR) == 0, "producer warps");
 
   __host__ __device__ static constexpr int phase(int k1, int k2) { return (k1 * WA + k2 * WB) % L; }
   __host__ __device__ static constexpr int carry(int k1, int k2) { return (k1 * WA + k2 * WB) / L; }
-  // Does pass p need B plane (k2, c)?
-  __host__ __device__ static constexpr bool needed(int p, int c, int k2) {
+  // Does pass p need B plane k2?
+  __host__ __device__ static constexpr bool needed(int p, int k2) {
     for (int k1 = 0; k1 < KA; ++k1)
-      if (carry(k1, k2) == c && phase(k1, k2) / PP == p) return true;
+      if (phase(k1, k2) / PP == p) return true;
     return false;
   }
-  // Shared-memory slot of B plane (k2, c) in pass p (-1 if unused).
-  __host__ __device__ static constexpr int slot(int p, int c, int k2) {
+  // Shared-memory slot of B plane k2 in pass p (-1 if unused).
+  __host__ __device__ static constexpr int slot(int p, int k2) {
     int s = 0;
-    for (int cc = 0; cc < 2; ++cc)
-      for (int k = 0; k < KB; ++k) {
-        const bool need = needed(p, cc, k);
-        if (cc == c && k == k2) return need ? s : -1;
-        if (need) ++s;
-      }
+    for (int k = 0; k < KB; ++k) {
+      const bool need = needed(p, k);
+      if (k == k2) return need ? s : -1;
+      if (need) ++s;
+    }
     return -1;
   }
   __host__ __device__ static constexpr int nslots(int p) {
     int s = 0;
-    for (int cc = 0; cc < 2; ++cc)
-      for (int k = 0; k < KB; ++k) s += needed(p, cc, k) ? 1 : 0;
+    for (int k = 0; k < KB; ++k) s += needed(p, k) ? 1 : 0;
     return s;
   }
   __host__ __device__ static constexpr int maxslots() {
@@ -144,39 +137,73 @@ struct TcCfg {
     return false;
   }
   static constexpr int MAXS = maxslots();
-  static constexpr int BSTAGE = MAXS * PLANE_BYTES;
+  static constexpr int SFSTAGE = 512;                       // B factor block of a stage (one copy source)
+  static constexpr int BSTAGE = MAXS * PLANE_BYTES + SFSTAGE;
   // B stages, the barrier block, and the FP32 stash of the passes' partial
   // outputs (row stride SST floats)
   static constexpr int SST = BN + 4;
   static constexpr size_t STASH = (size_t)BM * SST * 4;
   static constexpr size_t SMEM = (size_t)NSB * BSTAGE + 2048 + STASH;
+  // D = F32, A = B = E5M2, UE8M0 factors, M = 128, N = BN
+  static constexpr uint32_t IDESC = idesc_mx_e5m2(BN, false);
 };
 
-// One 16-byte core-matrix row (chunk kc of the run) of every B plane the pass needs.
-template <class Cfg, int PT, int PASS>
-__device__ __forceinline__ void write_b_planes(uint8_t* stage, int row, int kc, const uint32_t (&v)[4],
-                                               const uint32_t (&vc)[4], const uint32_t (&mk)[4][4]) {
-  const uint32_t core = (uint32_t)((row >> 3) * 256 + kc * 128 + (row & 7) * 16);
-#pragma unroll
-  for (int c = 0; c < 2; ++c) {
-    bool any = false;
-#pragma unroll
-    for (int k2 = 0; k2 < Cfg::KB; ++k2) any = any || Cfg::slot(PASS, c, k2) >= 0;
-    if (!any) continue;
-    uint32_t pw[4][Cfg::KB > 8 ? Cfg::KB : 8];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) PlaneFmt<Cfg::FB_>::planes(c ? vc[q] : v[q], mk[q], pw[q]);
-#pragma unroll
-    for (int k2 = 0; k2 < Cfg::KB; ++k2) {
-      const int sl = Cfg::slot(PASS, c, k2);
-      if (sl < 0) continue;
-      *reinterpret_cast<uint4*>(stage + (size_t)sl * Cfg::PLANE_BYTES + core) =
-          make_uint4(pw[0][k2], pw[1][k2], pw[2][k2], pw[3][k2]);
-    }
+// Plane words of 4 codes of a binary format or of E4C3 with r = 2^{8/9}:
+// values +-2^e (block-scale free) and the curve-index masks.
+template <int FMT>
+__device__ __forceinline__ void mx_decode(uint32_t w, uint32_t& v, uint32_t (&mk)[4]) {
+  if constexpr (FMT == CURVEFP_E4C3_R8_9) {
+    r89_word(w, v, mk);
+  } else {
+    uint32_t vc;
+    mx_word<FMT, 0>(w, v, vc);
+    k_masks<PLANE_E5M2, Fmt<FMT>::C>(w, mk);
   }
 }
 
-template <class Cfg, int PT, int PASS>
+// Plane words of 4 codes with per-element exponent bytes (reused operands):
+// byte i of dp is x_i + 16 for the plane value 2^{x_i} (x_i in [-16, 15]), or
+// 0x80 where the element has no plane value (zero code, or more than 31
+// binades below the largest element of its step).
+template <int FMT>
+__device__ __forceinline__ void pes_decode(uint32_t w, uint32_t dp, uint32_t& v, uint32_t (&mk)[4]) {
+  const uint32_t nz = prmt_sign((w & CodeBits<FMT>::MM) + 0x7F7F7F7Fu, 0xBA98u);
+  const uint32_t lost = prmt_sign(dp, 0xBA98u);
+  v = ((w & 0x80808080u) | e5m2_pow2(dp & 0x1F1F1F1Fu)) & nz & ~lost;
+  k_masks<PLANE_E5M2, Fmt<FMT>::C>(w, mk);
+}
+
+// Plane words and masks of a thread's 16 codes.
+template <int FMT, bool PES>
+__device__ __forceinline__ void decode_run(const uint4& cw, const uint4& dw, uint32_t (&v)[4], uint32_t (&mk)[4][4]) {
+  const uint32_t w[4] = {cw.x, cw.y, cw.z, cw.w}, d[4] = {dw.x, dw.y, dw.z, dw.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    if constexpr (PES)
+      pes_decode<FMT>(w[i], d[i], v[i], mk[i]);
+    else
+      mx_decode<FMT>(w[i], v[i], mk[i]);
+  }
+}
+
+// One 16-byte core-matrix row (chunk kc of the run) of every B plane the pass needs.
+template <class Cfg, int PASS>
+__device__ __forceinline__ void write_b_planes(uint8_t* stage, int row, int kc, const uint32_t (&v)[4],
+                                               const uint32_t (&mk)[4][4]) {
+  const uint32_t core = (uint32_t)((row >> 3) * 256 + kc * 128 + (row & 7) * 16);
+  uint32_t pw[4][Cfg::KB > 8 ? Cfg::KB : 8];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) PlaneFmt<Cfg::FB_>::planes(v[q], mk[q], pw[q]);
+#pragma unroll
+  for (int k2 = 0; k2 < Cfg::KB; ++k2) {
+    const int sl = Cfg::slot(PASS, k2);
+    if (sl < 0) continue;
+    *reinterpret_cast<uint4*>(stage + (size_t)sl * Cfg::PLANE_BYTES + core) =
+        make_uint4(pw[0][k2], pw[1][k2], pw[2][k2], pw[3][k2]);
+  }
+}
+
+template <class Cfg, int PASS>
 __device__ __forceinline__ void issue_pass(uint32_t leader, uint32_t tmem, uint64_t bdesc0, int abuf, int bstage,
                                            bool first_step) {
 #pragma unroll
@@ -185,24 +212,23 @@ __device__ __forceinline__ void issue_pass(uint32_t leader, uint32_t tmem, uint6
     for (int k2 = 0; k2 < Cfg::KB; ++k2) {
       const int h = Cfg::phase(k1, k2);
       if (h / Cfg::PP != PASS) continue;
-      const int sl = Cfg::slot(PASS, Cfg::carry(k1, k2), k2);
+      const int sl = Cfg::slot(PASS, k2);
       const uint32_t a_t = tmem + Cfg::ACOL0 + abuf * Cfg::AU_COLS + k1 * 8;
       const uint64_t bd = bdesc0 + (uint64_t)((bstage * Cfg::BSTAGE + sl * Cfg::PLANE_BYTES) >> 4);
       const uint32_t d_t = tmem + (h - PASS * Cfg::PP) * Cfg::BN;
       const uint32_t accum = (first_step && Cfg::first_of_phase(k1, k2)) ? 0u : 1u;
-      if (PT == PLANE_BF16)
-        tc::mma_f16_ts_if(leader, d_t, a_t, bd, Cfg::IDESC, accum);
-      else
-        tc::mma_f8_ts_if(leader, d_t, a_t, bd, Cfg::IDESC, accum);
+      // the carry 2^c is the B factor byte c (the row's factor times 2^c)
+      const uint32_t idesc = Cfg::IDESC | ((uint32_t)Cfg::carry(k1, k2) << 4);
+      mma_mx_if(leader, d_t, a_t, bd, idesc, tmem + Cfg::SFA0 + abuf * 4, tmem + Cfg::SFB0 + bstage * 4, accum);
     }
 }
 
-template <class Cfg, int PT>
+template <class Cfg>
 __device__ __forceinline__ void issue_step(uint32_t leader, int p, uint32_t tmem, uint64_t bdesc0, int abuf,
                                            int bstage, bool first_step) {
-  if (p == 0) issue_pass<Cfg, PT, 0>(leader, tmem, bdesc0, abuf, bstage, first_step);
-  if (Cfg::NP > 1 && p == 1) issue_pass<Cfg, PT, (Cfg::NP > 1 ? 1 : 0)>(leader, tmem, bdesc0, abuf, bstage, first_step);
-  if (Cfg::NP > 2 && p == 2) issue_pass<Cfg, PT, (Cfg::NP > 2 ? 2 : 0)>(leader, tmem, bdesc0, abuf, bstage, first_step);
+  if (p == 0) issue_pass<Cfg, 0>(leader, tmem, bdesc0, abuf, bstage, first_step);
+  if (Cfg::NP > 1 && p == 1) issue_pass<Cfg, (Cfg::NP > 1 ? 1 : 0)>(leader, tmem, bdesc0, abuf, bstage, first_step);
+  if (Cfg::NP > 2 && p == 2) issue_pass<Cfg, (Cfg::NP > 2 ? 2 : 0)>(leader, tmem, bdesc0, abuf, bstage, first_step);
 }
 
 }  // namespace
@@ -222,33 +248,35 @@ struct TailPlan {
 };
 
 // Per-element scales of both operands (PES = true; reused operands of the
-// training GEMMs): dp[r][k] = max(a(r,k) - ref, -64) + 64 beside the codes,
-// and the row reference ref = max_k a(r,k) read as refs[r >> rsh].
+// training GEMMs), written by the preparation kernels (gemm_reuse.cu):
+// dp[r][k] the element's plane exponent byte (pes_decode), f[r][s] the
+// exponent of step s's largest element minus 15 (INT16_MIN for a step
+// without nonzero codes), ref[r] = max_s f[r][s].
 struct PesOperands {
   const uint8_t* dA;
   const uint8_t* dB;
+  const int16_t* fA;
+  const int16_t* fB;
   const int* refA;
   const int* refB;
-  int rshA, rshB;
 };
 
 // Thread layout: warps 0 .. NAW-1 produce A (warp w: TMEM lane group w & 3,
 // share w >> 2 of each 32-byte run: NWA columns per plane) and run the
 // epilogue (columns [BN/ATPR share, BN/ATPR (share + 1))); the next 2 BN
 // threads produce B (thread 32 NAW + t: row t % BN, half t / BN); the last
-// warp allocates TMEM and issues the MMAs.
-template <int FA, int FB, int PT, bool PES>
-__global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(const uint8_t* __restrict__ A, const int8_t* __restrict__ sA,
-                                                         const uint8_t* __restrict__ B, const int8_t* __restrict__ sB,
-                                                         int M, int N, int K, int G, int gshift,
-                                                         float* __restrict__ C, uint32_t* status,
-                                                         const PesOperands pes, const TailPlan plan) {
-  using Cfg = TcCfg<FA, FB, PT>;
+// warp allocates TMEM and issues the factor copies and the MMAs.
+template <int FA, int FB, bool PES>
+__global__ void __launch_bounds__(TcCfg<FA, FB>::THREADS, 1)
+    gemm_tc_kernel(const uint8_t* __restrict__ A, const int8_t* __restrict__ sA, const uint8_t* __restrict__ B,
+                   const int8_t* __restrict__ sB, int M, int N, int K, int G, int gshift, float* __restrict__ C,
+                   uint32_t* status, const PesOperands pes, const TailPlan plan) {
+  using Cfg = TcCfg<FA, FB>;
   constexpr int L = Cfg::L, PP = Cfg::PP, NP = Cfg::NP, BN = Cfg::BN, NSB = Cfg::NSB;
   constexpr int NAW = Cfg::NAW, NWA = Cfg::NWA, ATPR = Cfg::ATPR;
-  constexpr int CB = PT == PLANE_E5M2 ? 4 : 2;  // code bytes per TMEM column / value word
   static_assert(NP <= 3, "pass dispatch");
   static_assert(NSB == TC_MAX_RING && Cfg::NAU == 2, "barrier rings");
+  static_assert(NWA == 4, "16-byte runs per producer thread");
   extern __shared__ __align__(1024) uint8_t smem[];
   uint8_t* bstage = smem;
   TcShared& sh = *reinterpret_cast<TcShared*>(smem + (size_t)NSB * Cfg::BSTAGE);
@@ -294,7 +322,7 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
   const bool rowok = is_prod && r < (is_a ? M : N);
   int ref = -128;
   if (PES) {
-    if (rowok) ref = __ldg(is_a ? pes.refA + (r >> pes.rshA) : pes.refB + (r >> pes.rshB));
+    if (rowok) ref = __ldg(is_a ? pes.refA + r : pes.refB + r);
   } else if (rowok) {
     const int8_t* s = (is_a ? sA : sB) + (int64_t)r * nb;
     if ((nb & 15) == 0 && (reinterpret_cast<uintptr_t>(s) & 15) == 0) {
@@ -320,32 +348,26 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
 
   if (is_prod) {
     // ------------------------------ producers ------------------------------
-    const uint8_t* src = (is_a ? A : B) + (int64_t)r * K + part * (is_a ? NWA : 4) * CB;
-    const uint8_t* dsrc = PES ? (is_a ? pes.dA : pes.dB) + (int64_t)r * K + part * (is_a ? NWA : 4) * CB : nullptr;
-    const int8_t* srow = (is_a ? sA : sB) + (int64_t)r * nb;
-    const int bias = is_a ? Cfg::PBA : Cfg::PBB;
+    const uint8_t* src = (is_a ? A : B) + (int64_t)r * K + part * 16;
+    const uint8_t* dsrc = PES ? (is_a ? pes.dA : pes.dB) + (int64_t)r * K + part * 16 : nullptr;
+    const int8_t* srow = PES ? nullptr : (is_a ? sA : sB) + (int64_t)r * nb;
+    const int16_t* frow = PES ? (is_a ? pes.fA : pes.fB) + (int64_t)r * (K / Cfg::KS) : nullptr;
     auto pass_of = [&](int g) { return (NP > 1 && g >= nsub ? 1 : 0) + (NP > 2 && g >= 2 * nsub ? 1 : 0); };
-    auto load = [&](int g, uint4& cw, int& off, uint4& dw) {
+    // codes (16 bytes), per-element exponent bytes (PES) and the step's raw
+    // scale (block scale, or the PES step exponent)
+    auto load = [&](int g, uint4& cw, int& raw, uint4& dw) {
       cw = make_uint4(0, 0, 0, 0);
       dw = make_uint4(0, 0, 0, 0);
-      off = 0;
+      raw = -32768;
       if (rowok && g < total) {
         const int s = s0 + g - pass_of(g) * nsub;  // step of the whole K
-        const uint8_t* p = src + (int64_t)s * Cfg::KS;
-        const int nbytes = (is_a ? NWA : 4) * CB;  // 16, 8 or 4
-        if (nbytes == 16) {
-          cw = __ldg(reinterpret_cast<const uint4*>(p));
-        } else if (nbytes == 8) {
-          const uint2 t = __ldg(reinterpret_cast<const uint2*>(p));
-          cw.x = t.x;
-          cw.y = t.y;
+        cw = __ldg(reinterpret_cast<const uint4*>(src + (int64_t)s * Cfg::KS));
+        if (PES) {
+          dw = __ldg(reinterpret_cast<const uint4*>(dsrc + (int64_t)s * Cfg::KS));
+          raw = (int)__ldg(frow + s);
         } else {
-          cw.x = __ldg(reinterpret_cast<const uint32_t*>(p));
+          raw = (int)__ldg(srow + (s >> gshift));
         }
-        if (PES)
-          dw = __ldg(reinterpret_cast<const uint4*>(dsrc + (int64_t)s * Cfg::KS));  // 16 relative scales
-        else
-          off = (int)__ldg(srow + (s >> gshift));  // raw scale: consumed two steps later
       }
     };
     const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
@@ -379,7 +401,7 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
 #pragma unroll
             for (int q = 0; q < PP; ++q)
               if (pe * PP + q < L) t = fmaf(phase_const(L, pe * PP + q), __uint_as_float(acc[q][c]), t);
-            y[c] = scalbnf(t, ref + Cfg::PBA + sh.refB[c0 + c] + Cfg::PBB);
+            y[c] = scalbnf(t, ref + sh.refB[c0 + c] - 2 * MX_OFF);
           }
           float4* s4 = reinterpret_cast<float4*>(strow + c0);
           if (pe > 0) {
@@ -416,18 +438,23 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
       return ok;
     };
     // One pipeline step of this producer thread; false ends the loop (abort).
-    auto step = [&](const int g, const uint4 cw, const int raw_scale, const uint4 dw) -> bool {
-      const int off = raw_scale - ref - bias;
+    auto step = [&](const int g, uint4 cw, const int raw, const uint4 dw) -> bool {
+      // the step's scale factor relative to the row reference; a block too
+      // far below it to have a factor byte is dropped
+      bool keep = raw != -32768;
+      uint32_t sf = 0;
+      if (keep) sf = mx_sf(raw - ref, 0, keep);
+      if (!keep) cw = make_uint4(0, 0, 0, 0);
       const int p = pass_of(g), s = g - p * nsub;
+      uint32_t v[4], mk[4][4];
+      if (is_a)
+        decode_run<FA, PES>(cw, dw, v, mk);
+      else
+        decode_run<FB, PES>(cw, dw, v, mk);
       if (is_a) {
-        uint32_t v[NWA], vc[NWA], mk[NWA][4];
-        if constexpr (PES)
-          decode_words_pes<FA, NWA>(cw, dw, bias, v, vc, mk, false);
-        else
-          PlaneFmt<FA>::template decode<PT, NWA>(cw, off, v, vc, mk, false);
-        uint32_t pl[NWA][Cfg::KA > 8 ? Cfg::KA : 8];
+        uint32_t pl[4][Cfg::KA > 8 ? Cfg::KA : 8];
 #pragma unroll
-        for (int c = 0; c < NWA; ++c) PlaneFmt<FA>::planes(v[c], mk[c], pl[c]);
+        for (int c = 0; c < 4; ++c) PlaneFmt<FA>::planes(v[c], mk[c], pl[c]);
         const int buf = g & 1;
         if (g >= 2) {
           // warp-uniform outcome: the TMEM stores below are warp-collective
@@ -441,16 +468,14 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
           }
         }
         // plane k1 occupies 8 columns of the unit; this thread's share of
-        // the 32-byte run is columns NWA part .. NWA part + NWA - 1
+        // the 32-byte run is columns 4 part .. 4 part + 3
 #pragma unroll
         for (int j = 0; j < Cfg::KA; ++j) {
-          uint32_t reg[NWA];
-#pragma unroll
-          for (int c = 0; c < NWA; ++c) reg[c] = pl[c][j];
-          const uint32_t ta = lane_base + Cfg::ACOL0 + buf * Cfg::AU_COLS + j * 8 + part * NWA;
-          if constexpr (NWA == 2) tc::tmem_st2(ta, reg);
-          else tc::tmem_st4(ta, reg);
+          const uint32_t reg[4] = {pl[0][j], pl[1][j], pl[2][j], pl[3][j]};
+          tc::tmem_st4(lane_base + Cfg::ACOL0 + buf * Cfg::AU_COLS + j * 8 + part * NWA, reg);
         }
+        // the row's factor (quadrant q reads column q of the unit's four)
+        if (part == 0) tc::tmem_st1(lane_base + Cfg::SFA0 + buf * 4 + (warp & 3), sf * 0x01010101u);
         tc::tmem_wait_st();
         tc::fence_before_sync();
         __syncwarp();
@@ -471,15 +496,14 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
           sh.abort_flag = 1;
           return false;
         }
-        uint32_t v[4], vc[4], mk[4][4];
-        if constexpr (PES)
-          decode_words_pes<FB, 4>(cw, dw, bias, v, vc, mk, true);
-        else
-          PlaneFmt<FB>::template decode<PT, 4>(cw, off, v, vc, mk, true);
         uint8_t* stg = bstage + (size_t)st * Cfg::BSTAGE;
-        if (p == 0) write_b_planes<Cfg, PT, 0>(stg, rloc, part, v, vc, mk);
-        if (NP > 1 && p == 1) write_b_planes<Cfg, PT, (NP > 1 ? 1 : 0)>(stg, rloc, part, v, vc, mk);
-        if (NP > 2 && p == 2) write_b_planes<Cfg, PT, (NP > 2 ? 2 : 0)>(stg, rloc, part, v, vc, mk);
+        if (p == 0) write_b_planes<Cfg, 0>(stg, rloc, part, v, mk);
+        if (NP > 1 && p == 1) write_b_planes<Cfg, (NP > 1 ? 1 : 0)>(stg, rloc, part, v, mk);
+        if (NP > 2 && p == 2) write_b_planes<Cfg, (NP > 2 ? 2 : 0)>(stg, rloc, part, v, mk);
+        // factor bytes of the row: byte 0 plain, byte 1 the carry's 2x
+        if (part == 0)
+          *reinterpret_cast<uint32_t*>(stg + Cfg::MAXS * Cfg::PLANE_BYTES + sfb_off(rloc)) =
+              keep ? (sf | (sf + 1) << 8) : 0u;
         tc::fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(&sh.full[st]);
@@ -524,7 +548,8 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
     }
   } else {
     // ------------------------------ MMA issuer -------------------------------
-    // The whole warp runs the loop; the elected lane issues MMAs and commits.
+    // The whole warp runs the loop; the elected lane copies the stage's B
+    // factors into TMEM, issues the MMAs and commits.
     const uint32_t leader = tc::elect_one();
     const uint64_t bdesc0 = tc::smem_desc(tc::smem_u32(bstage), 128, 256);
     bool ok = true;
@@ -538,7 +563,9 @@ __global__ void __launch_bounds__(TcCfg<FA, FB, PT>::THREADS, 1) gemm_tc_kernel(
       if ((g & 7) == 0) ok = ok && !read_abort(&sh.abort_flag);
       if (!ok) break;
       tc::fence_after_sync();
-      issue_step<Cfg, PT>(leader, p, tmem, bdesc0, g & 1, st, s == 0);
+      tmem_cp_sf_if(leader, tmem + Cfg::SFB0 + st * 4,
+                    bstage + (size_t)st * Cfg::BSTAGE + Cfg::MAXS * Cfg::PLANE_BYTES);
+      issue_step<Cfg>(leader, p, tmem, bdesc0, g & 1, st, s == 0);
       tc::mma_commit_if(leader, &sh.empty[st]);
       if (s == nsub - 1) tc::mma_commit_if(leader, &sh.acc_full);
     }
@@ -625,15 +652,14 @@ inline TailPlan tail_plan(int64_t tiles, int sms, int nsub) {
   return t;
 }
 
-template <int FA, int FB, int PT, bool PES>
+template <int FA, int FB, bool PES>
 static cudaError_t launch_tc_t(int G, const uint8_t* a, const int8_t* sa, const uint8_t* b, const int8_t* sb,
                                int64_t M, int64_t N, int64_t K, float* c, uint32_t* st, cudaStream_t s,
                                const PesOperands& pes, int sms) {
-  using Cfg = TcCfg<FA, FB, PT>;
+  using Cfg = TcCfg<FA, FB>;
   static_assert(sizeof(TcShared) <= 2048, "shared tail");
   static_assert(Cfg::SMEM <= 227 * 1024, "shared memory");
-  static_assert(!PES || (PT == PLANE_E5M2 && Cfg::NWA == 4), "per-element scales: E5M2 planes, 16-byte runs");
-  auto kern = gemm_tc_kernel<FA, FB, PT, PES>;
+  auto kern = gemm_tc_kernel<FA, FB, PES>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg::SMEM);
   if (e != cudaSuccess) return e;
   const int64_t ntn = (N + Cfg::BN - 1) / Cfg::BN, ntm = (M + Cfg::BM - 1) / Cfg::BM;

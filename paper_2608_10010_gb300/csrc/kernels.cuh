@@ -21,9 +21,6 @@ cudaError_t launch_selftest_wait(int arrive, long long limit, uint32_t* status, 
 cudaError_t launch_gemm_tensor(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
                                const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, uint32_t* status,
                                cudaStream_t st, int sms);
-cudaError_t launch_gemm_tensor_sparse(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
-                                      const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, uint32_t* status,
-                                      cudaStream_t st);
 bool gemm_tensor_supported(int fa, int fb);
 bool gemm_narrow_supported(int fa, int fb);
 cudaError_t launch_gemm_tensor_narrow(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,

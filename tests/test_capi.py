@@ -105,8 +105,10 @@ def test_oriented_gemm_validation(lib):
     wsb = lib.curvefp_gemm_oriented_workspace_bytes
     al = lambda v: (v + 255) // 256 * 256  # noqa: E731
     assert wsb(1, 0, 0, 256, 96, 64) == 0 and wsb(0, 1, 1, 256, 96, 64) == 0
-    assert wsb(1, 0, 1, 256, 96, 64) == al(256 * 64) + al(4 * 256) + 2 * al(96 * 64) + al(4 * 96)
-    assert wsb(1, 1, 1, 256, 96, 64) == 2 * al(256 * 64) + al(4 * 256) + 2 * al(96 * 64) + al(4 * 96)
+    # per operand: [R K codes (COLS)] + R K exponent bytes + R K / 16 step-scale bytes + 4 R
+    op = lambda R, K, cols: (al(R * K) if cols else 0) + al(R * K) + al(R * K // 16) + al(4 * R)  # noqa: E731
+    assert wsb(1, 0, 1, 256, 96, 64) == op(256, 64, False) + op(96, 64, True)
+    assert wsb(1, 1, 1, 256, 96, 64) == op(256, 64, True) + op(96, 64, True)
     go = lib.curvefp_gemm_oriented
     go.argtypes = [C.c_int] * 4 + [P, P, C.c_int, P, P, C.c_int, C.c_int64, C.c_int64, C.c_int64, P, P, P, P,
                                    C.c_size_t, P, P]
@@ -122,7 +124,7 @@ def test_oriented_gemm_validation(lib):
     assert call(ws=P(4096 + 16), wsn=1 << 30) == INVALID  # workspace not 256-byte aligned
     assert call(ws=d, wsn=16) == INVALID               # workspace too small
     assert call(ps=d, pl=d, ws=d, wsn=1 << 30) == INVALID  # phase sums only from EXACT
-    assert call(algo=2, ws=d, wsn=1 << 30) == UNSUPPORTED  # sparse: ROWS x ROWS only
+    assert call(algo=2, ws=d, wsn=1 << 30) == INVALID      # 2 is not an algorithm
     assert call(la=1, lb=1, K=48, ws=d, wsn=1 << 30) == INVALID  # tensor steps need K % 32
     assert call(algo=0, c=None) == INVALID             # exact: nothing to write
     assert call(algo=0, ps=d, pl=None) == INVALID      # exact: both phase arrays or neither

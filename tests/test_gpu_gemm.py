@@ -149,7 +149,7 @@ def test_exact_zero_and_extreme_operands(torch):
 
 # ---- tensor kernel ------------------------------------------------------------------
 
-@pytest.mark.parametrize("algo", ["tensor", "tensor_sparse"])
+@pytest.mark.parametrize("algo", ["tensor", "tensor_narrow"])
 @pytest.mark.parametrize("fa,fb", TC_PAIRS)
 def test_tensor_pairs_ragged(torch, fa, fb, algo):
     rng = np.random.default_rng(99 + hash((fa, fb)) % 1000)
@@ -161,7 +161,7 @@ def test_tensor_pairs_ragged(torch, fa, fb, algo):
         check_tensor(torch, a, sa, b, sb, fa, fb, block, algo=algo)
 
 
-@pytest.mark.parametrize("algo", ["tensor", "tensor_sparse"])
+@pytest.mark.parametrize("algo", ["tensor", "tensor_narrow"])
 @pytest.mark.parametrize("fa,fb", TC_PAIRS)
 def test_tensor_full_code_space(torch, fa, fb, algo):
     """Uniformly random codes (every level, both signs, zeros) and scale spread."""
@@ -172,13 +172,14 @@ def test_tensor_full_code_space(torch, fa, fb, algo):
 
 
 @pytest.mark.parametrize("fa,fb", TC_PAIRS)
-def test_tensor_sparse_matches_dense(torch, fa, fb):
-    """Two plane pairs per 2:4-sparse MMA against one per dense MMA: the same
-    exact products, summed in a different order in FP32."""
+def test_narrow_matches_tile(torch, fa, fb):
+    """The two tensor-core kernels (2:4-sparse pair planes along N against
+    dense plane pairs of a tile): the same exact products, summed in a
+    different order in FP32."""
     rng = np.random.default_rng(11)
     a, sa = rand_operand(rng, fa, 300, 1024, 32, spread=4)
     b, sb = rand_operand(rng, fb, 200, 1024, 32, spread=4)
-    cs, st = gpu_gemm(torch, a, sa, b, sb, fa, fb, 32, "tensor_sparse")
+    cs, st = gpu_gemm(torch, a, sa, b, sb, fa, fb, 32, "tensor_narrow")
     cd, st2 = gpu_gemm(torch, a, sa, b, sb, fa, fb, 32, "tensor")
     assert st == 0 and st2 == 0
     na = oracle.row_norms(a, sa, fa)
@@ -254,7 +255,6 @@ def test_llama7b_linear_full_size(torch):
     rows = _sample(2048)
     check_exact(torch, ra, rsa, rb, rsb, "E3C3", "E3C3", 32, rows=rows)
     check_tensor(torch, ra, rsa, rb, rsb, "E3C3", "E3C3", 32, rows=rows)
-    check_tensor(torch, ra, rsa, rb, rsb, "E3C3", "E3C3", 32, rows=rows, algo="tensor_sparse")
     # the benchmark's GEMM: phases along N, 2:4-sparse pair planes (64 token groups x 32 weight tiles)
     check_tensor(torch, ra, rsa, rb, rsb, "E3C3", "E3C3", 32, rows=rows, algo="tensor_narrow")
 

@@ -88,7 +88,7 @@ def test_static_quantize_stays_inside(torch, group, rule):
 
 @pytest.mark.parametrize("algo,fa,fb", [("exact", "E3C3", "E5C2"), ("tensor", "E3C3", "E3C3"),
                                         ("tensor", "E5C2", "E4C3"), ("tensor", "E4C3_R8_9", "E4C3_R8_9"),
-                                        ("tensor_sparse", "E4C3", "E4C3"), ("skinny", "E4C3", "E5C2"),
+                                        ("tensor_narrow", "E5C2", "E4C3"), ("skinny", "E4C3", "E5C2"),
                                         ("auto", "E4C3", "E4C3"), ("exact", "E4C3_R3_4", "E4C3_R3_4"),
                                         ("tensor_narrow", "E3C3", "E3C3"), ("tensor_narrow", "E5C2", "E5C2"),
                                         ("tensor_narrow", "E4C3", "E5C2")])

@@ -98,9 +98,9 @@ def test_quantized_activations_and_weights(torch, fa, fb):
     check(torch, a, sa, b, sb, fa, fb, G)
 
 
-def test_wide_scale_spread_flushes_like_tensor(torch):
-    """Block scales 40 binades apart: planes below 2^-14 of a row's largest
-    block scale flush on both tensor paths, still within tolerance."""
+def test_wide_scale_spread_in_the_factors(torch):
+    """Block scales 40 binades apart: both tensor paths carry them in the
+    MMAs' scale factors, within tolerance of the oracle and of each other."""
     rng = np.random.default_rng(7)
     a, sa = rand_operand(rng, "E4C3", 8, 512, 32, spread=20)
     b, sb = rand_operand(rng, "E4C3", 256, 512, 32, spread=20)
