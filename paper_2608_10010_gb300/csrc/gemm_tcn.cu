@@ -45,10 +45,10 @@
 //               one thread per weight row (all 32 codes of its steps): codes
 //               -> pair planes, metadata and the row's scale factor -> TMEM;
 //               after the last step they run the epilogue.
-//   next warps  X producers: groups taking every NGX-th step, one 4-code word
-//               of one token per work item -> the step's R blocks; the
-//               token's scale factors -> the stage's factor block (copied to
-//               TMEM by the MMA warp).
+//   next warps  X producers: groups taking every NGX-th step, 8 codes of one
+//               token per work item -> one 16-byte chunk of each of the
+//               step's R blocks; the token's scale factors -> the stage's
+//               factor block (copied to TMEM by the MMA warp).
 //   last warp   TMEM allocation, factor copies and MMA issue (one elected
 //               lane).
 // With fewer weight tiles than fill the SMs' last wave, tiles are split in K
@@ -98,7 +98,7 @@ struct TcnCfg {
   static constexpr int SFSTAGE = 1024;               // factor block of a step (two copy sources)
   static constexpr int PFW = 4;  // own steps of weight codes in flight per W thread
   static constexpr int PFX = 2;  // own steps of activation codes in flight per X thread
-  static constexpr int XI = MTMAX * 8 / (XPG * 32);  // X work items (4-code words) per thread and step
+  static constexpr int XI = MTMAX * 4 / (XPG * 32);  // X work items (8-code chunks) per thread and step
   // more than half of the SM's shared memory: one CTA per SM (the split plan
   // assumes it, and the CTA allocates all of TMEM)
   static constexpr size_t SMEM_USED = (size_t)NSB * (BSTAGE + SFSTAGE) + 2048;
@@ -161,7 +161,9 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16
 
 // X: [Mx x K] token codes, W: [Nw x K] weight codes (K contiguous), scales
 // [rows x K/G].  C: [Mx x Nw] (TR = false) or [Nw x Mx] (TR = true), row-major.
-template <int FX, int FW, bool TR>
+// FULL: every tile has MTMAX tokens (Mt == MTMAX), so the stage offsets of
+// the X producers are constants.
+template <int FX, int FW, bool TR, bool FULL>
 __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
     gemm_tcn_kernel(const uint8_t* __restrict__ X, const int8_t* __restrict__ sX, const uint8_t* __restrict__ W,
                     const int8_t* __restrict__ sW, int M, int N, int K, int G, int gshift, int Mt,
@@ -412,49 +414,47 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
     }
   } else if (is_x) {
     // ---------------------------- X producers -----------------------------
-    // Work item wi of a group covers one 4-code word: lane bits of wi give 8
-    // tokens x 4 words of a 16-code chunk kc, so a warp's 8-byte stores fill
-    // 256 consecutive bytes of an R block.  Items of padding tokens (and
-    // lattice positions that hold no plane) write nothing: the stages were
-    // zeroed at the start.  The item of a token's first word also writes the
-    // token's scale factor into the factor block: one word per column n =
-    // h Mt + m of the MMA (the factor ids read bytes 0 and 1).
+    // Work item wi of a group covers 8 codes (16-byte chunk c of a 64-byte R
+    // row) of one token: lane bits of wi give 8 tokens x the 4 chunks, so a
+    // warp's 16-byte stores fill 512 consecutive bytes of an R block.  Items
+    // of padding tokens (and lattice positions that hold no plane) write
+    // nothing: the stages were zeroed at the start.  The item of a token's
+    // first chunk also writes the token's scale factor into the factor
+    // block: one word per column n = h Mt + m of the MMA (the factor ids read
+    // bytes 0 and 1).
     constexpr int PF = Cfg::PFX, XI = Cfg::XI, NGX = Cfg::NGX;
     const int tg = t_x % (Cfg::XPG * 32);  // thread of the group
     // per item: activation row (-1: padding), its row reference, its token
-    // and the byte offset of its word in a stage (block b adds b Mt 64 bytes)
-    int xrow[XI], xref[XI], xtok[XI];
+    // and the byte offset of its chunk in a stage (block b adds b Mt 64 bytes)
+    int xrow[XI], xref[XI], xtok[XI], xcol[XI];
     uint32_t xbase[XI];
-    auto word_of = [&](int wi) { return ((wi >> 5) & 1) * 4 + ((wi & 31) >> 3); };  // 4-code word of the step
 #pragma unroll
     for (int i = 0; i < XI; ++i) {
       const int wi = tg + i * Cfg::XPG * 32, xl = wi & 31;
-      const int tok = (wi >> 6) * 8 + (xl & 7);  // token of the tile
+      const int tok = (wi >> 5) * 8 + (xl & 7), c = xl >> 3;  // token of the tile, chunk of the row
       const bool act = tok < Mt && x0 + tok < M;
       xrow[i] = act ? x0 + tok : -1;
       xref[i] = act ? sh.refB[tok] : 0;
-      xtok[i] = word_of(wi) == 0 ? tok : -1;  // writes the token's factors
-      // the word's 8 interleaved bytes in 16-byte chunk j >> 1 of a 64-byte row
-      const int j = word_of(wi);
-      xbase[i] = (uint32_t)((tok >> 3) * 512 + (j >> 1) * 128 + (tok & 7) * 16 + (j & 1) * 8);
+      xtok[i] = c == 0 ? tok : -1;  // writes the token's factors
+      xcol[i] = c * 8;
+      xbase[i] = (uint32_t)((tok >> 3) * 512 + c * 128 + (tok & 7) * 16);
     }
-    auto load = [&](int i, uint32_t (&cw)[XI], int (&raw)[XI]) {
+    auto load = [&](int i, uint2 (&cw)[XI], int (&raw)[XI]) {
       const int g = gx + i * NGX;
 #pragma unroll
       for (int e = 0; e < XI; ++e) {
-        cw[e] = 0u;
+        cw[e] = make_uint2(0u, 0u);
         raw[e] = 0;
         if (xrow[e] >= 0 && g < total) {
           const int s = s0 + g;
-          const int wi = tg + e * Cfg::XPG * 32;
-          cw[e] = __ldg(reinterpret_cast<const uint32_t*>(X + (int64_t)xrow[e] * K + (int64_t)s * Cfg::KS +
-                                                          word_of(wi) * 4));
+          cw[e] = __ldg(reinterpret_cast<const uint2*>(X + (int64_t)xrow[e] * K + (int64_t)s * Cfg::KS + xcol[e]));
           raw[e] = (int)__ldg(sX + (int64_t)xrow[e] * nb + (s >> gshift));
         }
       }
     };
-    const uint32_t bstride = (uint32_t)Mt * Cfg::ROWB;  // bytes per column block
-    auto step = [&](const int g, const uint32_t (&cw)[XI], const int (&raw)[XI]) -> bool {
+    // bytes per column block (a constant for whole tiles)
+    const uint32_t bstride = FULL ? (uint32_t)(Cfg::MTMAX * Cfg::ROWB) : (uint32_t)Mt * Cfg::ROWB;
+    auto step = [&](const int g, const uint2 (&cw)[XI], const int (&raw)[XI]) -> bool {
       const int st = g % NSB;
       if (g >= NSB) {
         const bool ok = wait_all(&sh.empty[st], ((g / NSB) - 1) & 1);
@@ -471,24 +471,44 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
         if (xrow[e] < 0) continue;
         bool keep;
         const uint32_t sf = mx_sf(raw[e] - xref[e], Cfg::PBX, keep);
-        uint32_t v, vc, mk[4];
-        mx_word<FX, Cfg::PBX>(keep ? cw[e] : 0u, v, vc);
-        k_masks<PLANE_E5M2, Fmt<FX>::C>(cw[e], mk);
-        uint32_t pv[8], pc[8];
-        planes_of<Fmt<FX>::C>(v, mk, pv);
-        planes_of<Fmt<FX>::C>(vc, mk, pc);
+        uint32_t pv[2][8], pc[2][8];
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+          const uint32_t w = q ? cw[e].y : cw[e].x;
+          uint32_t v, vc, mk[4];
+          mx_word<FX, Cfg::PBX>(keep ? w : 0u, v, vc);
+          k_masks<PLANE_E5M2, Fmt<FX>::C>(w, mk);
+          planes_of<Fmt<FX>::C>(v, mk, pv[q]);
+          planes_of<Fmt<FX>::C>(vc, mk, pc[q]);
+        }
         // R block b interleaves Q block b with Q block b - PO; Q block u < L
         // is the carry copy of plane u, u >= L plane u - L
 #pragma unroll
         for (int b = Cfg::RB0; b < 2 * L; ++b) {
-          const uint32_t x = b < L ? pc[b] : pv[b - L];
-          const uint32_t y = b - Cfg::PO < L ? pc[b - Cfg::PO] : pv[b - Cfg::PO - L];
-          *reinterpret_cast<uint2*>(stg + xbase[e] + (b - Cfg::RB0) * bstride) = interleave2(x, y);
+          uint2 lo, hi;
+          {
+            const uint32_t x = b < L ? pc[0][b] : pv[0][b - L];
+            const uint32_t y = b - Cfg::PO < L ? pc[0][b - Cfg::PO] : pv[0][b - Cfg::PO - L];
+            lo = interleave2(x, y);
+          }
+          {
+            const uint32_t x = b < L ? pc[1][b] : pv[1][b - L];
+            const uint32_t y = b - Cfg::PO < L ? pc[1][b - Cfg::PO] : pv[1][b - Cfg::PO - L];
+            hi = interleave2(x, y);
+          }
+          *reinterpret_cast<uint4*>(stg + xbase[e] + (b - Cfg::RB0) * bstride) = make_uint4(lo.x, lo.y, hi.x, hi.y);
         }
         if (xtok[e] >= 0) {
           const uint32_t sw = sf * 0x01010101u;
+          if constexpr (FULL && Cfg::MTMAX == 32) {
+            // n = 32 h + m: row m of both copy sources, all four words
 #pragma unroll
-          for (int h = 0; h < L; ++h) *reinterpret_cast<uint32_t*>(sfs + sfb_off(h * Mt + xtok[e])) = sw;
+            for (int c = 0; c < L / 4; ++c)
+              *reinterpret_cast<uint4*>(sfs + c * 512 + xtok[e] * 16) = make_uint4(sw, sw, sw, sw);
+          } else {
+#pragma unroll
+            for (int h = 0; h < L; ++h) *reinterpret_cast<uint32_t*>(sfs + sfb_off(h * Mt + xtok[e])) = sw;
+          }
         }
       }
       tc::fence_proxy_async_smem();
@@ -497,7 +517,7 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
       return true;
     };
     const int nown = (total - gx + NGX - 1) / NGX;
-    uint32_t q[PF][XI];
+    uint2 q[PF][XI];
     int rq[PF][XI];
 #pragma unroll
     for (int u = 0; u < PF; ++u) load(u, q[u], rq[u]);
@@ -607,13 +627,13 @@ cudaError_t launch_tcn_t(int G, const uint8_t* x, const int8_t* sx, const uint8_
   using Cfg = TcnCfg<FX, FW>;
   static_assert(sizeof(TcShared) <= 2048, "shared tail");
   static_assert(Cfg::SMEM <= 227 * 1024, "shared memory");
-  auto kern = gemm_tcn_kernel<FX, FW, TR>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg::SMEM);
-  if (e != cudaSuccess) return e;
   // token groups of equal size Mt (a multiple of 8) of at most MTMAX tokens
   int64_t ng = (Mx + Cfg::MTMAX - 1) / Cfg::MTMAX;
   const int Mt = (int)(((Mx + ng - 1) / ng + 7) / 8 * 8);
   ng = (Mx + Mt - 1) / Mt;
+  auto kern = Mt == Cfg::MTMAX ? gemm_tcn_kernel<FX, FW, TR, true> : gemm_tcn_kernel<FX, FW, TR, false>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg::SMEM);
+  if (e != cudaSuccess) return e;
   const int64_t ntw = (Nw + Cfg::BM - 1) / Cfg::BM, tiles = ntw * ng;
   const TailPlan plan = tcn_plan(tiles, sms, (int)(K / Cfg::KS));
   if (plan.nsplit > 0) {
