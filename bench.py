@@ -39,14 +39,14 @@ sys.path.insert(0, ROOT)
 
 M, N, K, G = 2048, 4096, 4096, 32
 # The step's GEMM: the tensor-core kernel with the phases along the MMA's N
-# dimension and 2:4-sparse pair planes (TENSOR_NARROW; 0.845 ms against the
-# 128 x 96 tile kernel's 1.08 ms at this size).
+# dimension, 2:4-sparse pair planes and block-scaled MMAs (TENSOR_NARROW;
+# 0.81 ms against the tile kernel's 1.05 ms at this size).
 GEMM_ALGO = "tensor_narrow"
 # DRAM bytes (read + written) of one launch of that GEMM at this size, from an
 # ncu capture (dram__bytes_read.sum + dram__bytes_write.sum) of the kernel as
 # it stands; set to None whenever the kernel changes until it is captured
 # again.
-GEMM_DRAM_TRAFFIC = 33_445_632 + 833_536
+GEMM_DRAM_TRAFFIC = 27_204_352 + 1_268_736
 FMT = "E3C3"
 WORKLOAD = "E3C3 Llama-7B-like linear: X[2048x4096] (1% outlier channels x20) . W[4096x4096]^T, block 32"
 METRIC = "CurveFP GEMM TOPS & quantize GB/s at 1 GB300, as % of roofline"
@@ -183,8 +183,8 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
         r = {"case": name, "algo": algo, "M": Mx, "N": Nx, "K": Kx, "formats": f"{fa}x{fb}", "ms": round(ms, 4),
              "tops": round(tops, 3)}
         if algo in ("tensor", "tensor_narrow"):
-            # the narrow kernel's same-format pairs use 2:4-sparse pair planes: half the MMA work
-            issued = planes // 2 if algo == "tensor_narrow" and fa == fb else planes
+            # the narrow kernel uses 2:4-sparse pair planes: half the MMA work
+            issued = planes // 2 if algo == "tensor_narrow" else planes
             r["tensor_work_frac"] = round(tops * issued / fp8_peak, 4)
         if hbm_bound:
             wbytes = Nx * Kx + Nx * Kx // G
@@ -260,7 +260,9 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
     gemm_case("fwd X.W", q(X, "E4C3", 0), "E4C3", q(Wt, "E4C3", 1), "E4C3", 64)
     gemm_case("fwd X.W narrow", q(X, "E4C3", 0), "E4C3", q(Wt, "E4C3", 1), "E4C3", 64, algo="tensor_narrow")
     gemm_case("dgrad dY.W^T", q(dY, "E5C2", 0), "E5C2", q(Wt, "E4C3", 0), "E4C3", 32)
+    gemm_case("dgrad dY.W^T narrow", q(dY, "E5C2", 0), "E5C2", q(Wt, "E4C3", 0), "E4C3", 32, algo="tensor_narrow")
     gemm_case("wgrad dY^T.X", q(dY, "E5C2", 1), "E5C2", q(X, "E4C3", 1), "E4C3", 32)
+    gemm_case("wgrad dY^T.X narrow", q(dY, "E5C2", 1), "E5C2", q(X, "E4C3", 1), "E4C3", 32, algo="tensor_narrow")
     # the same triplet on operands quantized once and reused (the backward
     # GEMMs read W, X and dY in the forward pass's block orientation; the
     # timed region includes the operand preparation kernels)
@@ -444,20 +446,50 @@ def run_ours(args):
     cq = torch.empty(xq.shape, dtype=torch.uint8, device=dev)
     sq = torch.empty((xq.shape[0], xq.shape[1] // G), dtype=torch.int8, device=dev)
     qt = []
-    for i in range(8):
-        flush_l2()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        cfp.quantize(xq, "E4C3", G, 0, codes=cq, scales=sq, stream=stream)
-        e1.record(stream)
-        e1.synchronize()
-        if i >= 3:
-            qt.append(e0.elapsed_time(e1))
+    with ClockSampler(local) as qclk:
+        for i in range(24):
+            flush_l2()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            cfp.quantize(xq, "E4C3", G, 0, codes=cq, scales=sq, stream=stream)
+            e1.record(stream)
+            e1.synchronize()
+            if i >= 4:
+                qt.append(e0.elapsed_time(e1))
     q_ms = statistics.median(qt)
     q_bytes = qn * (2 + 1) + qn // G
     q_gbs = q_bytes / (q_ms / 1e3) / 1e9
     del xq, cq, sq
     torch.cuda.empty_cache()
+
+    # the small E4C3 workload (A[128x256] and B[256x128] ~ N(0,1) FP32, block
+    # 32 along K): the latency of the whole path, both quantizers and the
+    # GEMM, on one stream (median of 200 runs, operands in L2)
+    A1, B1 = inputs.small_e4c3()
+    A1d, B1d = torch.from_numpy(A1).to(dev), torch.from_numpy(B1).to(dev)
+    a1 = torch.empty((128, 256), dtype=torch.uint8, device=dev)
+    sa1 = torch.empty((128, 256 // G), dtype=torch.int8, device=dev)
+    b1 = torch.empty((128, 256), dtype=torch.uint8, device=dev)
+    sb1 = torch.empty((128, 256 // G), dtype=torch.int8, device=dev)
+    C1 = torch.empty((128, 128), dtype=torch.float32, device=dev)
+    c1_ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    c1_q, c1_g, c1_t = [], [], []
+    for i in range(220):
+        c1_ev[0].record(stream)
+        cfp.quantize(A1d, "E4C3", G, 0, codes=a1, scales=sa1, stream=stream)
+        cfp.quantize(B1d, "E4C3", G, 1, codes=b1, scales=sb1, stream=stream)
+        c1_ev[1].record(stream)
+        cfp.gemm(a1, sa1, b1, sb1, "E4C3", "E4C3", G, "auto", out=C1, stream=stream)
+        c1_ev[2].record(stream)
+        c1_ev[2].synchronize()
+        if i >= 20:
+            c1_q.append(c1_ev[0].elapsed_time(c1_ev[1]) * 1e3)
+            c1_g.append(c1_ev[1].elapsed_time(c1_ev[2]) * 1e3)
+            c1_t.append(c1_ev[0].elapsed_time(c1_ev[2]) * 1e3)
+    config1 = {"workload": "E4C3 A[128x256] . B[256x128] ~ N(0,1) fp32, block 32 along K: quantize both + GEMM (AUTO)",
+               "quantize_us": round(statistics.median(c1_q), 2), "gemm_us": round(statistics.median(c1_g), 2),
+               "total_us": round(statistics.median(c1_t), 2), "launches": 3,
+               "note": "latency-bound (4.2M MACs); operands in L2"}
 
     # end-to-end through the C ABI with host buffers (pinned), per step:
     # H2D of X and W, the four calls, D2H of C.
@@ -576,12 +608,20 @@ def run_ours(args):
                      "unit": "TFLOP/s", "frac": round(gemm_tops / fp8_peak, 6), "traffic": GEMM_DRAM_TRAFFIC,
                      "bytes_algorithmic": M * K + N * K + (M + N) * K // G + 4 * M * N,
                      "peak_source": f"FP8 dense = 2 x bf16 burst ({bf16} TFLOP/s, {peak_src})",
-                     "kernel": "gemm_tcn_kernel (tcgen05.mma.sp kind::f8f6f4, E5M2 pair planes, phases along N)",
+                     "kernel": "gemm_tcn_kernel (tcgen05.mma.sp kind::mxf8f6f4.block_scale, E5M2 pair planes, "
+                               "UE8M0 block-scale factors, phases along N)",
                      "tensor_work_frac": round(gemm_tops * planes / fp8_peak, 4),
                      "note": f"achieved counts algorithmic closed-product ops (2 per MAC); the kernel issues "
                              f"{planes} dense-equivalent FP8 MACs per useful MAC (4 sparse pair-plane MMAs of "
                              f"logical K 64 per 32 codes, 8 phase columns per token), so the tensor-pipe work "
-                             f"is tensor_work_frac of peak"},
+                             f"is tensor_work_frac of peak",
+                     "quantizer": {"bound": "hbm", "workload": "2^30 BF16 elements, N(0,1) with 0.1% x100 outliers, "
+                                                               "E4C3, block 32 (input 2 GiB > L2, L2 flushed)",
+                                   "ms": round(q_ms, 4), "achieved": round(q_gbs, 1), "unit": "GB/s",
+                                   "bytes_per_elem": 3 + 1 / G, "frac_of_8TBps": round(q_gbs / 8000.0, 4),
+                                   "peak": hbm, "frac": round(q_gbs / hbm, 4),
+                                   "peak_source": f"copy bandwidth ({peak_src})", "clocks": qclk.summary()},
+                     "config1": config1},
         "kernels_ms": {k: round(v, 4) for k, v in mean.items()},
         "quantize": {"gbs_w": round(q_gbs_w, 1), "gbs_x": round(q_gbs_x, 1), "frac_w": round(q_gbs_w / hbm, 4),
                      "frac_x": round(q_gbs_x / hbm, 4), "peak_gbs": hbm, "bytes_per_elem": 4 + 1 + 1 / G,

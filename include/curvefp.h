@@ -49,7 +49,7 @@ extern "C" {
  * (CurveFP8, 8 bits, 127 positive levels, H = 8 and 4): Table 1, binary radix.
  * E4C3_R8_9, E4C3_R3_4: E4C3 codes with the rational radices r = 2^{8/9}
  * (9 phases) and r = 2^{3/4} (32 phases) of the radix frontier (Sec. 3.1
- * Eq. 1 with r = 2^{p/q}, Eq. 4, Table 7): level x = (-1)^s 2^{a_b}
+ * Eq. 1 with r = 2^{p/q}, Eq. 4, Table 2): level x = (-1)^s 2^{a_b}
  * 2^{p n/(8q)}; block scale = the smallest a_b with max|x| <= 2^{a_b}
  * 2^{63 p/(8q)}; an exact tie in the nearest-level search (only between zero
  * and L_nmin = 2^{-7} for r = 2^{8/9}) goes to zero; dequantization is
@@ -131,10 +131,11 @@ curvefp_status_t curvefp_quantize(curvefp_format_t fmt, int block, const void* x
                                   int64_t rows, int64_t cols, int64_t ld, int block_axis, uint8_t* codes,
                                   int8_t* scales, uint32_t* device_status, void* stream);
 
-/* Static operands (Sec. 3.1: "static operands choose a representable
- * power-of-two scale by reconstruction-MSE search"; Sec. 4.2 evaluates
- * tensorwise, rowwise and block scaling).  A scale group is a block of
- * `block` elements of a row, a whole row, or the whole tensor. */
+/* Static operands (Sec. 3.1: the scale of a weight, fixed ahead of time, is
+ * picked among representable powers of two by the reconstruction error it
+ * gives; Sec. 4.2 compares scales per tensor, per row and per block).  A
+ * scale group is a block of `block` elements of a row, a whole row, or the
+ * whole tensor. */
 typedef enum { CURVEFP_SCALE_BLOCK = 0, CURVEFP_SCALE_ROW = 1, CURVEFP_SCALE_TENSOR = 2 } curvefp_scale_group_t;
 /* CEIL_ABSMAX: the group's ceil-absmax scale a_c (as curvefp_quantize).
  * MSE: the candidate a in [a_c - 3, a_c + 1] (clamped to int8) with the
@@ -179,10 +180,11 @@ curvefp_status_t curvefp_quantize_static(curvefp_format_t fmt, int block, curvef
  *   The array is shared by every call on a device and keeps the last call's
  *   contents; each call clears the part it uses before its kernels.  Calls
  *   that overlap on the GPU (different streams without ordering) race on it.
- *   The first call on a device looks the array's device address up
- *   (cudaGetSymbolAddress, with that device current); make that first call
- *   before any stream capture.  Other arguments, results and errors as
- *   curvefp_quantize_static. */
+ *   Every call looks the array's device address up on the current device
+ *   (cudaGetSymbolAddress; nothing is cached, so a device reset between
+ *   calls is harmless); the first call on a device also loads the library's
+ *   module there, so make that first call before any stream capture.  Other
+ *   arguments, results and errors as curvefp_quantize_static. */
 #define CURVEFP_NOALLOC_SCRATCH_BYTES (8u << 20)
 curvefp_status_t curvefp_quantize_static_noalloc(curvefp_format_t fmt, int block, curvefp_scale_group_t group,
                                                  curvefp_scale_rule_t rule, const void* x, curvefp_dtype_t dtype,
@@ -237,7 +239,8 @@ curvefp_status_t curvefp_gemm(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, 
                               int64_t N, int64_t K, float* c, uint32_t* device_status, void* stream);
 
 /* Validation form of the EXACT GEMM that also exports the per-phase integer
- * accumulators (Eq. 5 "signed integer counts" summed per phase; App. A.1).
+ * accumulators (Eq. 5: the signed integer counts of each phase, summed with
+ * their bin weights; App. A.1).
  *   phase_sums : M*N*H two's-complement int128 values stored as (lo, hi) int64
  *                pairs, [M][N][H]; S_h at LSB 2^{lsb}.
  *   phase_lsb  : [M x N] int32, lsb = min_b(sa[i,b] + sb[j,b]) + t_min with
@@ -297,7 +300,7 @@ curvefp_status_t curvefp_gemm_oriented(curvefp_gemm_algo_t algo, curvefp_format_
                                        void* stream);
 
 /* curvefp_gemm_phases computed with the histogram layout (Eq. 5, App. A.1:
- * "equal addresses can be merged with signed popcounts"): every product's
+ * products with equal addresses merge into one signed count): every product's
  * address (phase h, bin t) is counted in a per-output histogram n_{h,t}
  * (lanes of a warp with equal addresses merge by signed popcount), and
  * S_h = sum_t n_{h,t} 2^t.  Same outputs, requirements and format pairs as

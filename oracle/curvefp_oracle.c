@@ -36,7 +36,7 @@
  *   R6 exported per-phase sums are integers S_h at the per-output LSB
  *      lambda = min_b(sa_b + sb_b) + t_min.
  *   R11, R12 static-operand scale groups and MSE-search scales (below).
- *   R14 rational radix r = 2^{p/q} (Sec. 3.1, Eq. 4, Table 7's E4C3 points
+ *   R14 rational radix r = 2^{p/q} (Sec. 3.1, Eq. 4, Table 2's E4C3 points
  *      r = 2^{8/9} and r = 2^{3/4}): the level of index n is 2^{p n/(qK)};
  *      the closed product of two codes of the same format has
  *      u = p (n_a + n_b), phase h = (u mod qK)/g and bin t = floor(u/qK)
@@ -221,9 +221,9 @@ int oracle_quantize(int id, int G, const float* x, int64_t rows, int64_t cols, i
   return flags;
 }
 
-/* Element encode with given block scales (Sec. 3.1: "given a_b,
- * quantization preserves the source sign and selects the magnitude whose
- * reconstructed value is nearest").  x is [R x Cc] row-major, blocks of G
+/* Element encode with given block scales (Sec. 3.1: with the block scale
+ * fixed, an element keeps its sign and takes the magnitude level whose
+ * reconstruction lies closest to it).  x is [R x Cc] row-major, blocks of G
  * along columns, scales [R x Cc/G].  Returns the NaN flag. */
 int oracle_encode(int id, int G, const float* x, int64_t R, int64_t Cc, const int8_t* scales,
                   uint8_t* codes) {
@@ -248,9 +248,10 @@ int oracle_encode(int id, int G, const float* x, int64_t R, int64_t Cc, const in
 }
 
 /* ---- Static operands: scale granularity and MSE-search scales ----------
- * Sec. 3.1: "static operands choose a representable power-of-two scale by
- * reconstruction-MSE search; dynamic training operands use ceil-absmax";
- * Sec. 4.2 evaluates tensorwise, rowwise and fixed-size block scaling.
+ * Sec. 3.1: a static operand's power-of-two scale is picked by the
+ * reconstruction error it gives, a dynamic (training) operand's by the
+ * ceil-absmax rule; Sec. 4.2 compares per-tensor, per-row and fixed-size
+ * block scales.
  * Readings (listed with the others):
  *   R11 a scale group is a block of G elements of a row, a whole row, or the
  *       whole tensor; scales are stored per block of G ([rows x cols/G]),
@@ -582,8 +583,8 @@ int64_t oracle_gemm_elem(int ida, int idb, const uint8_t* A, const int8_t* eA, c
   return bad;
 }
 
-/* Histogram layout (Eq. 5, App. A.1: "equal addresses can be merged with
- * signed popcounts"): signed counts n_{h,t} for ONE output, t in
+/* Histogram layout (Eq. 5, App. A.1: products with the same address may be
+ * merged into one signed count): signed counts n_{h,t} for ONE output, t in
  * [tlo, tlo + nt).  Used by the tests to check that both accumulation
  * layouts give the same phase sums.  Returns -1 if a t falls outside. */
 int oracle_histogram(int ida, int idb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,

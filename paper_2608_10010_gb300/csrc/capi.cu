@@ -104,14 +104,10 @@ curvefp_status_t curvefp_quantize_static_noalloc(curvefp_format_t fmt, int block
   const size_t need = cfp::quantize_static_workspace(rows, cols, block, group);
   if (need > CURVEFP_NOALLOC_SCRATCH_BYTES) return CURVEFP_ERR_UNSUPPORTED;
   void* scratch = nullptr;
-  if (need) {
-    // this device's copy of the array, looked up once per device
-    static void* addr[64] = {nullptr};
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return CURVEFP_ERR_CUDA;
-    if (!addr[dev] && cudaGetSymbolAddress(&addr[dev], g_static_scratch) != cudaSuccess) return CURVEFP_ERR_CUDA;
-    scratch = addr[dev];
-  }
+  // the current device's copy of the array, looked up on every call (nothing
+  // cached: an address kept from before a device reset would be stale, and
+  // concurrent callers share no host state)
+  if (need && cudaGetSymbolAddress(&scratch, g_static_scratch) != cudaSuccess) return CURVEFP_ERR_CUDA;
   return curvefp_quantize_static(fmt, block, group, rule, x, dtype, rows, cols, codes, scales, scratch, need,
                                  device_status, stream);
 }

@@ -712,9 +712,9 @@ __global__ void __launch_bounds__(256) dequantize_kernel(const uint8_t* __restri
 }
 
 // ---------------------------------------------------------------------------
-// Static operands (Sec. 3.1: "static operands choose a representable
-// power-of-two scale by reconstruction-MSE search"; Sec. 4.2: tensorwise,
-// rowwise and block scaling).  A scale group is a block of G elements, a row
+// Static operands (Sec. 3.1: a fixed operand's power-of-two scale is picked
+// by the reconstruction error it gives; Sec. 4.2 compares per-tensor,
+// per-row and per-block scales).  A scale group is a block of G elements, a row
 // or the whole tensor; its scale is the ceil-absmax scale a_c, or, for the MSE
 // rule, the candidate a in [a_c - 3, a_c + 1] with the smallest
 //   D(a) = sum_i floor((x_i - xhat_i)^2 2^{60 - 2 a_c}),

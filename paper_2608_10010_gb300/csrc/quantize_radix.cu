@@ -1,5 +1,5 @@
 // Launchers for the rational-radix E4C3 formats (Sec. 3.1 Eq. 1 with
-// r = 2^{p/q}; Table 7's points r = 2^{8/9} and r = 2^{3/4}): the shared
+// r = 2^{p/q}; Table 2's points r = 2^{8/9} and r = 2^{3/4}): the shared
 // quantizer kernels of quantize_kernels.cuh with these formats' rank tables
 // and the exact encode of radix.cuh, and their dequantizer.
 #include "quantize_kernels.cuh"

@@ -131,7 +131,7 @@ def test_oriented_gemm_validation(lib):
 
 
 def test_rational_radix_host_rules(lib):
-    """The rational-radix formats: phase counts (Table 7: 9 and 32), pairing
+    """The rational-radix formats: phase counts (Table 2: 9 and 32), pairing
     only with themselves, and the entry points that do not take them."""
     P = ctypes.c_void_p
     d = P(4096)

@@ -1,5 +1,5 @@
 """GPU parity of the rational-radix E4C3 formats (r = 2^{8/9}, 9 phases;
-r = 2^{3/4}, 32 phases; Sec. 3.1 Eq. 1, Eq. 4, Table 7): codes, scales,
+r = 2^{3/4}, 32 phases; Sec. 3.1 Eq. 1, Eq. 4, Table 2): codes, scales,
 dequantized values and exact per-phase int128 sums bit-identical to the
 oracle, through the C ABI."""
 import numpy as np

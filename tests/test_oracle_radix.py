@@ -1,5 +1,5 @@
 """Pins for the oracle's rational-radix formats (Sec. 3.1 Eq. 1 with
-r = 2^{p/q}, Eq. 4, App. A.1; Table 7's E4C3 points r = 2^{8/9} and
+r = 2^{p/q}, Eq. 4, App. A.1; Table 2's E4C3 points r = 2^{8/9} and
 r = 2^{3/4}).  Every check is against 80-digit arithmetic, the exponent
 identity of Eq. 1, or a value the paper prints.
 """
@@ -51,7 +51,7 @@ def quant_one_block(oracle, fmt, vals):
 
 
 def test_table7_phase_counts(oracle):
-    """Table 7 (radix frontier): E4C3 with r = 2^{8/9} needs 9 phases and
+    """Table 2 (radix frontier): E4C3 with r = 2^{8/9} needs 9 phases and
     r = 2^{3/4} needs 32; the oracle's lattice for each format has exactly
     that many phases, and every phase class is reached by some product (the
     subgroup argument of App. A.1)."""
