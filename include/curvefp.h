@@ -173,7 +173,7 @@ curvefp_status_t curvefp_quantize_static(curvefp_format_t fmt, int block, curvef
  *   The scratch lives in a fixed file-scope device array of the library,
  *   CURVEFP_NOALLOC_SCRATCH_BYTES (8 MiB) on every GPU that loads the library,
  *   held until the process exits.  That is enough for row groups of up to
- *   ~100,000 rows; tensor and block groups need almost none.  The call makes
+ *   about 98,000 rows; tensor and block groups need almost none.  The call makes
  *   no cudaMalloc, cudaFree or other allocating call.
  *   Returns CURVEFP_ERR_UNSUPPORTED, before any device work, when the groups
  *   need more scratch than the array holds.

@@ -245,10 +245,13 @@ __device__ __forceinline__ uint32_t ranks4_f32(const uint32_t* tab, const uint32
 // Fast path (finite block, scale >= -100): one shared-memory rank lookup per
 // element (BF16: the byte itself; FP32: plus one 16-bit compare), signs merged
 // four at a time.  Other blocks take the exact per-element slow path.
+// With gscale (static operands with row or tensor scale groups) the scale of
+// block b is gscale[b / bpg] instead of the block's own ceil-absmax scale.
 template <int FMT, typename T, int G>
 __global__ void __launch_bounds__(256) quantize_rows_kernel(const T* __restrict__ x, int64_t rows, int64_t cols,
                                                             int64_t ld, uint8_t* __restrict__ codes,
-                                                            int8_t* __restrict__ scales, uint32_t* status) {
+                                                            int8_t* __restrict__ scales, uint32_t* status,
+                                                            const int8_t* __restrict__ gscale, int64_t bpg) {
   using F = Fmt<FMT>;
   constexpr int VEC = Elem<T>::VEC;
   constexpr bool BF16 = sizeof(T) == 2;
@@ -320,9 +323,10 @@ __global__ void __launch_bounds__(256) quantize_rows_kernel(const T* __restrict_
 #pragma unroll
       for (int o = TPB / 2; o > 0; o >>= 1) mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
       const bool ok = blk[u] < nblk;
-      int a = block_scale<FMT>(mx);
+      const bool grouped = gscale != nullptr;
+      int a = grouped ? (ok ? (int)gscale[blk[u] / bpg] : 0) : block_scale<FMT>(mx);
       const bool fast = mx < 0x7F800000u && a >= -100;
-      if (__any_sync(0xffffffffu, !fast)) {  // rare: NaN / Inf / subnormal-scale blocks
+      if (!grouped && __any_sync(0xffffffffu, !fast)) {  // rare: NaN / Inf / subnormal-scale blocks
         uint32_t mx2 = 0u;
 #pragma unroll
         for (int q = 0; q < VPT; ++q)
@@ -732,7 +736,10 @@ __device__ __forceinline__ uint32_t load_bits(const T* x, int64_t i) {
 }
 
 // Eq. 1 reconstruction in FP32 of a code at scale a: one rounding of the
-// exact product RN32(2^{k/K}) 2^{a+e}.
+// exact product RN32(2^{k/K}) 2^{a+e}.  Where 2^{a+e} keeps the product in
+// FP32's normal range the product is exact and is formed on the exponent
+// field (integer arithmetic only: FP64 is a slow pipe on this GPU); the
+// other cases round once through FP64.
 template <int FMT>
 __device__ __forceinline__ float recon_f32(uint32_t code, int a) {
   using F = Fmt<FMT>;
@@ -742,14 +749,20 @@ __device__ __forceinline__ float recon_f32(uint32_t code, int a) {
   const int n = (int)m - F::B;
   const int e = n >= 0 ? n / F::K : -((-n + F::K - 1) / F::K);
   const int k = n - e * F::K;
-  const float ck = __uint_as_float(F::K == 8 ? CFP_CK_F32_K8_DEV[k] : CFP_CK_F32_K4_DEV[k]);
-  const float v = __double2float_rn(ldexp((double)ck, a + e));
-  return (code & 0x80u) ? -v : v;
+  const uint32_t ckb = F::K == 8 ? CFP_CK_F32_K8_DEV[k] : CFP_CK_F32_K4_DEV[k];  // in [1, 2): exponent field 127
+  const int E = a + e;
+  uint32_t vb;
+  if (E >= -126 && E <= 127) {
+    vb = ckb + ((uint32_t)E << 23);
+  } else {
+    vb = __float_as_uint(__double2float_rn(ldexp((double)__uint_as_float(ckb), E)));
+  }
+  return __uint_as_float(vb | ((code & 0x80u) << 24));
 }
 
-// floor((x - xhat)^2 2^{60 - 2 ac}) exactly: x - xhat is exact in FP64 (both
-// FP32, within a factor 16 unless xhat = 0), e = M 2^{E-53}, e^2 = M^2 2^{2E-106}.
-__device__ __forceinline__ unsigned __int128 sq_term(float x, float xhat, int ac) {
+// The same term through FP64 (x - xhat is exact in FP64 while the two
+// exponents differ by less than 29).
+__device__ __forceinline__ unsigned __int128 sq_term_f64(float x, float xhat, int ac) {
   const double e = fabs((double)x - (double)xhat);
   if (e == 0.0) return 0;
   int E;
@@ -757,6 +770,49 @@ __device__ __forceinline__ unsigned __int128 sq_term(float x, float xhat, int ac
   const unsigned long long M = (unsigned long long)ldexp(fr, 53);
   const unsigned __int128 sq = (unsigned __int128)M * M;
   const int sh = 2 * E - 106 + 60 - 2 * ac;
+  if (sh >= 0) return sh >= 128 ? (unsigned __int128)0 : sq << sh;
+  return sh <= -128 ? (unsigned __int128)0 : sq >> (-sh);
+}
+
+// A finite FP32 value as M 2^E with a signed integer M (|M| < 2^24).
+__device__ __forceinline__ void f32_int(float v, int& M, int& E) {
+  const uint32_t b = __float_as_uint(v);
+  const int ef = (int)((b >> 23) & 0xFFu);
+  const int mm = (int)(b & 0x7FFFFFu);
+  M = ef ? (mm | 0x800000) : mm;
+  E = ef ? ef - 150 : -149;
+  if (b >> 31) M = -M;
+}
+
+// floor((x - xhat)^2 2^{60 - 2 ac}) exactly, in integer arithmetic: with
+// x = Mx 2^Ex, xhat = Mh 2^Eh and Emin = min(Ex, Eh), x - xhat =
+// (Mx 2^{Ex - Emin} - Mh 2^{Eh - Emin}) 2^Emin.  xhat is the nearest level to
+// x or the saturation level of a scale at most 3 binades below the group's
+// ceil-absmax scale, so the exponents differ by at most a few binades (more
+// only when xhat = 0, where the difference is x itself); the integer
+// difference then needs at most 32 bits and its square 64.
+__device__ __forceinline__ unsigned __int128 sq_term(float x, float xhat, int ac) {
+  int Mx, Ex, Mh, Eh;
+  f32_int(x, Mx, Ex);
+  f32_int(xhat, Mh, Eh);
+  long long d;
+  int E;
+  if (Mh == 0) {
+    d = Mx;
+    E = Ex;
+  } else if (Mx == 0) {
+    d = Mh;
+    E = Eh;
+  } else {
+    E = min(Ex, Eh);
+    const int sx = Ex - E, sh2 = Eh - E;
+    if (sx > 30 || sh2 > 30) return sq_term_f64(x, xhat, ac);  // not reached by the callers (see above)
+    d = ((long long)Mx << sx) - ((long long)Mh << sh2);
+  }
+  if (d == 0) return 0;
+  const unsigned long long ad = (unsigned long long)(d < 0 ? -d : d);
+  const unsigned __int128 sq = (unsigned __int128)ad * ad;
+  const int sh = 2 * E + 60 - 2 * ac;
   if (sh >= 0) return sh >= 128 ? (unsigned __int128)0 : sq << sh;
   return sh <= -128 ? (unsigned __int128)0 : sq >> (-sh);
 }
@@ -769,74 +825,102 @@ __device__ __forceinline__ void atomic_add_u128(unsigned long long* p, unsigned 
   if (hi + carry) atomicAdd(p + 1, hi + carry);
 }
 
-// Group statistics: max |x| as an FP32 bit pattern (NaN left out; Inf =
-// 0x7F800000), one atomic max per group and thread run.
+// Row and tensor groups are cut into spans of at most QS_SPAN elements; one
+// CTA per span (span c of group g = blockIdx.x: g = bid / cpg, c = bid % cpg)
+// reads it with coalesced loads and raises its group's result once.
+constexpr int64_t QS_SPAN = 16384;
+
+// Group maxima: max |x| as an FP32 bit pattern (NaN left out; Inf =
+// 0x7F800000), one atomic max per CTA.
 template <typename T>
-__global__ void __launch_bounds__(256) qs_stats_kernel(const T* __restrict__ x, int64_t n, int64_t glen,
-                                                       uint32_t* amax, uint32_t* status) {
+__global__ void __launch_bounds__(256) qs_gmax_kernel(const T* __restrict__ x, int64_t glen, int64_t cpg,
+                                                      uint32_t* amax, uint32_t* status) {
+  __shared__ uint32_t red[8];
+  const int64_t g = blockIdx.x / cpg, c = blockIdx.x - g * cpg;
+  const int64_t i0 = g * glen + c * QS_SPAN, i1 = g * glen + min(glen, (c + 1) * QS_SPAN);
   bool nan = false;
-  uint32_t run = 0u;
-  int64_t run_g = -1;
-  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t g = i / glen;
-    if (g != run_g) {
-      if (run_g >= 0 && run) atomicMax(&amax[run_g], run);
-      run_g = g;
-      run = 0u;
+  uint32_t m = 0u;
+  constexpr int VEC = 16 / (int)sizeof(T);
+  const bool vec = ((i0 | i1) % VEC) == 0 && (reinterpret_cast<uintptr_t>(x) & 15) == 0;
+  if (vec) {
+    const uint4* p = reinterpret_cast<const uint4*>(x + i0);
+    const int64_t nv = (i1 - i0) / VEC;
+    for (int64_t v = threadIdx.x; v < nv; v += blockDim.x) {
+      const uint4 q = __ldcs(p + v);
+      const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        if constexpr (sizeof(T) == 2) {
+          const uint32_t lo = (w[k] << 16) & 0x7FFFFFFFu, hi = w[k] & 0x7FFF0000u;
+          nan |= lo > 0x7F800000u || hi > 0x7F800000u;
+          m = max(m, max(lo > 0x7F800000u ? 0u : lo, hi > 0x7F800000u ? 0u : hi));
+        } else {
+          const uint32_t b = w[k] & 0x7FFFFFFFu;
+          nan |= b > 0x7F800000u;
+          m = max(m, b > 0x7F800000u ? 0u : b);
+        }
+      }
     }
-    const uint32_t b = load_bits(x, i) & 0x7FFFFFFFu;
-    if (b > 0x7F800000u) nan = true;
-    else run = max(run, b);
+  } else {
+    for (int64_t i = i0 + threadIdx.x; i < i1; i += blockDim.x) {
+      const uint32_t b = load_bits(x, i) & 0x7FFFFFFFu;
+      nan |= b > 0x7F800000u;
+      m = max(m, b > 0x7F800000u ? 0u : b);
+    }
   }
-  if (run_g >= 0 && run) atomicMax(&amax[run_g], run);
-  if (nan && status) atomicOr(status, CURVEFP_DEV_NAN);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) m = max(m, __shfl_xor_sync(0xffffffffu, m, o));
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = m;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int w = 1; w < (int)(blockDim.x >> 5); ++w) m = max(m, red[w]);
+    if (m) atomicMax(&amax[g], m);
+  }
+  if (__any_sync(0xffffffffu, nan) && (threadIdx.x & 31) == 0 && status) atomicOr(status, CURVEFP_DEV_NAN);
 }
 
-// Per group and candidate: D(a) over this thread's elements, flushed with one
-// exact 128-bit atomic add per candidate and group run.
+// 128-bit sum of a warp's lanes (exact; carries from the low words).
+__device__ __forceinline__ unsigned __int128 warp_sum_u128(unsigned __int128 v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const unsigned long long lo = __shfl_xor_sync(0xffffffffu, (unsigned long long)v, o);
+    const unsigned long long hi = __shfl_xor_sync(0xffffffffu, (unsigned long long)(v >> 64), o);
+    v += ((unsigned __int128)hi << 64) | lo;
+  }
+  return v;
+}
+
+// Per group and candidate: D(a) over the CTA's span, one exact 128-bit
+// atomic add per warp and candidate.
 template <int FMT, typename T>
-__global__ void __launch_bounds__(256) qs_mse_kernel(const T* __restrict__ x, int64_t n, int64_t glen,
+__global__ void __launch_bounds__(256) qs_mse_kernel(const T* __restrict__ x, int64_t glen, int64_t cpg,
                                                      const uint32_t* __restrict__ amax, unsigned long long* D) {
   __shared__ uint32_t lut[256];
   for (int i = threadIdx.x; i < 256; i += blockDim.x) lut[i] = __ldg(lut_src<Fmt<FMT>::K>() + i);
   __syncthreads();
-  // each thread takes a contiguous run of elements (fewer group changes)
-  const int64_t nthreads = (int64_t)gridDim.x * blockDim.x;
-  const int64_t tid = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  const int64_t per = (n + nthreads - 1) / nthreads;
-  const int64_t i0 = tid * per, i1 = min(n, i0 + per);
-  unsigned __int128 acc[5];
-  int64_t run_g = -1;
-  int ac = 0;
-  bool search = false;
-  auto flush = [&]() {
-    if (run_g >= 0 && search)
-      for (int c = 0; c < 5; ++c)
-        if (acc[c]) atomic_add_u128(D + (run_g * 5 + c) * 2, acc[c]);
-  };
+  const int64_t g = blockIdx.x / cpg, c = blockIdx.x - g * cpg;
+  const uint32_t am = amax[g];
+  if (am == 0u || am >= 0x7F800000u) return;  // the group keeps a_c
+  const int ac = block_scale<FMT>(am);
+  const int64_t i0 = g * glen + c * QS_SPAN, i1 = g * glen + min(glen, (c + 1) * QS_SPAN);
+  unsigned __int128 acc[5] = {0, 0, 0, 0, 0};
   bool dummy = false;
-  for (int64_t i = i0; i < i1; ++i) {
-    const int64_t g = i / glen;
-    if (g != run_g) {
-      flush();
-      run_g = g;
-      const uint32_t am = amax[g];
-      ac = block_scale<FMT>(am);
-      search = am != 0u && am < 0x7F800000u;
-      for (int c = 0; c < 5; ++c) acc[c] = 0;
-    }
-    if (!search) continue;
+  for (int64_t i = i0 + threadIdx.x; i < i1; i += blockDim.x) {
     const uint32_t b = load_bits(x, i);
     if ((b & 0x7FFFFFFFu) > 0x7F800000u) continue;  // NaN: left out
     const float xv = __uint_as_float(b);
-    for (int c = 0; c < 5; ++c) {
-      const int a = ac - 3 + c;
+#pragma unroll
+    for (int k = 0; k < 5; ++k) {
+      const int a = ac - 3 + k;
       if (a < -128 || a > 127) continue;
-      const uint32_t code = encode_slow<FMT>(lut, b, a, dummy);
-      acc[c] += sq_term(xv, recon_f32<FMT>(code, a), ac);
+      acc[k] += sq_term(xv, recon_f32<FMT>(encode_slow<FMT>(lut, b, a, dummy), a), ac);
     }
   }
-  flush();
+#pragma unroll
+  for (int k = 0; k < 5; ++k) {
+    const unsigned __int128 s = warp_sum_u128(acc[k]);
+    if ((threadIdx.x & 31) == 0 && s) atomic_add_u128(D + (g * 5 + k) * 2, s);
+  }
 }
 
 // The group's scale: a_c, or the MSE candidate with the smallest D (ties: the
@@ -861,29 +945,32 @@ __device__ __forceinline__ int choose_scale(uint32_t am, const unsigned long lon
   return best;
 }
 
-// Encode every element under its group's scale; scales stored per block of G.
+// Encode with one scale per group, element by element: the fallback for
+// inputs that are not 16-byte aligned (the block quantizer loads 16-byte
+// vectors).
 template <int FMT, typename T>
-__global__ void __launch_bounds__(256) qs_encode_kernel(const T* __restrict__ x, int64_t n, int64_t glen, int G,
-                                                        int rule, const uint32_t* __restrict__ amax,
-                                                        const unsigned long long* __restrict__ D, uint8_t* codes,
-                                                        int8_t* scales, uint32_t* status) {
+__global__ void __launch_bounds__(256) qs_encode_scalar_kernel(const T* __restrict__ x, int64_t n, int64_t glen, int G,
+                                                               const int8_t* __restrict__ gscale, uint8_t* codes,
+                                                               int8_t* scales, uint32_t* status) {
   __shared__ uint32_t lut[256];
   for (int i = threadIdx.x; i < 256; i += blockDim.x) lut[i] = __ldg(lut_src<Fmt<FMT>::K>() + i);
   __syncthreads();
   const int gs = __ffs(G) - 1;
   bool nan = false;
-  int64_t run_g = -1;
-  int a = 0;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t g = i / glen;
-    if (g != run_g) {
-      run_g = g;
-      a = choose_scale<FMT>(amax[g], D ? D + g * 10 : nullptr, D ? rule : 0);
-    }
+    const int a = gscale[i / glen];
     codes[i] = (uint8_t)encode_slow<FMT>(lut, load_bits(x, i), a, nan);
     if ((i & (G - 1)) == 0) scales[i >> gs] = (int8_t)a;  // G is a power of two
   }
   if (nan && status) atomicOr(status, CURVEFP_DEV_NAN);
+}
+
+// One scale per group (the encode pass then takes it per block).
+template <int FMT>
+__global__ void qs_choose_kernel(const uint32_t* __restrict__ amax, const unsigned long long* __restrict__ D,
+                                 int rule, int64_t ngroups, int8_t* __restrict__ gscale) {
+  for (int64_t g = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; g < ngroups; g += (int64_t)gridDim.x * blockDim.x)
+    gscale[g] = (int8_t)choose_scale<FMT>(amax[g], D ? D + g * 10 : nullptr, D ? rule : 0);
 }
 
 // Block groups: one thread per block of G elements does everything in
@@ -908,17 +995,21 @@ __global__ void __launch_bounds__(256) qs_block_kernel(const T* __restrict__ x, 
     const bool search = rule == 1 && am != 0u && am < 0x7F800000u;
     if (search) {
       const int ac = block_scale<FMT>(am);
+      unsigned __int128 acc[5] = {0, 0, 0, 0, 0};
+      for (int i = 0; i < G; ++i) {
+        const uint32_t b = load_bits(x, i0 + i);
+        if ((b & 0x7FFFFFFFu) > 0x7F800000u) continue;
+        const float xv = __uint_as_float(b);
+#pragma unroll
+        for (int k = 0; k < 5; ++k) {
+          const int a = ac - 3 + k;
+          if (a < -128 || a > 127) continue;
+          acc[k] += sq_term(xv, recon_f32<FMT>(encode_slow<FMT>(lut, b, a, dummy), a), ac);
+        }
+      }
       for (int c = 0; c < 5; ++c) {
-        const int a = ac - 3 + c;
-        unsigned __int128 d = 0;
-        if (a >= -128 && a <= 127)
-          for (int i = 0; i < G; ++i) {
-            const uint32_t b = load_bits(x, i0 + i);
-            if ((b & 0x7FFFFFFFu) > 0x7F800000u) continue;
-            d += sq_term(__uint_as_float(b), recon_f32<FMT>(encode_slow<FMT>(lut, b, a, dummy), a), ac);
-          }
-        Dg[2 * c] = (unsigned long long)d;
-        Dg[2 * c + 1] = (unsigned long long)(d >> 64);
+        Dg[2 * c] = (unsigned long long)acc[c];
+        Dg[2 * c + 1] = (unsigned long long)(acc[c] >> 64);
       }
     }
     const int a = choose_scale<FMT>(am, Dg, search ? 1 : 0);
@@ -974,7 +1065,7 @@ static cudaError_t launch_q(const void* x, int64_t rows, int64_t cols, int64_t l
     if (grid > cap) grid = cap;
     if (grid < 1) grid = 1;
     quantize_rows_kernel<FMT, T, G><<<(unsigned)grid, 256, 0, st>>>(static_cast<const T*>(x), rows, cols, ld,
-                                                                      codes, scales, status);
+                                                                      codes, scales, status, nullptr, 1);
   } else {
     dim3 grid((unsigned)((cols + 255) / 256), (unsigned)(rows / G));
     quantize_cols_kernel<FMT, T, G><<<grid, 256, 0, st>>>(static_cast<const T*>(x), rows, cols, ld, codes, scales,
@@ -996,10 +1087,44 @@ static cudaError_t launch_q_g(int G, const void* x, int64_t rows, int64_t cols, 
   return cudaErrorInvalidValue;
 }
 
+// The register-fed block quantizer with a scale per group of bpg blocks.
+template <int FMT, typename T, int G>
+static cudaError_t launch_q_grp(const T* x, int64_t rows, int64_t cols, uint8_t* codes, int8_t* scales,
+                                uint32_t* status, cudaStream_t st, int sms, const int8_t* gscale, int64_t bpg) {
+  constexpr int VEC = Elem<T>::VEC;
+  constexpr int TPB = (sizeof(T) == 2 && G == 32) ? 2 : ((G / VEC) < 8 ? (G / VEC) : 8);
+  const int64_t nblk = rows * (cols / G);
+  constexpr int VPT = (G / VEC) / TPB;
+  constexpr int PER_WARP = (32 / TPB) * (VPT >= 4 ? 1 : 4 / VPT);
+  const int64_t warps_needed = (nblk + PER_WARP - 1) / PER_WARP;
+  int64_t grid = (warps_needed + 7) / 8;
+  const int64_t cap = (int64_t)sms * 8;
+  if (grid > cap) grid = cap;
+  if (grid < 1) grid = 1;
+  quantize_rows_kernel<FMT, T, G><<<(unsigned)grid, 256, 0, st>>>(x, rows, cols, cols, codes, scales, status, gscale,
+                                                                    bpg);
+  return cudaGetLastError();
+}
+
+template <int FMT, typename T>
+static cudaError_t launch_q_grouped(int G, const T* x, int64_t rows, int64_t cols, uint8_t* codes, int8_t* scales,
+                                    uint32_t* status, cudaStream_t st, int sms, const int8_t* gscale, int64_t bpg) {
+  switch (G) {
+    case 32: return launch_q_grp<FMT, T, 32>(x, rows, cols, codes, scales, status, st, sms, gscale, bpg);
+    case 64: return launch_q_grp<FMT, T, 64>(x, rows, cols, codes, scales, status, st, sms, gscale, bpg);
+    case 128: return launch_q_grp<FMT, T, 128>(x, rows, cols, codes, scales, status, st, sms, gscale, bpg);
+    case 256: return launch_q_grp<FMT, T, 256>(x, rows, cols, codes, scales, status, st, sms, gscale, bpg);
+    case 512: return launch_q_grp<FMT, T, 512>(x, rows, cols, codes, scales, status, st, sms, gscale, bpg);
+  }
+  return cudaErrorInvalidValue;
+}
+
+// Workspace of row / tensor groups: group maxima (4 bytes), group scales
+// (1 byte) and the MSE sums (5 candidates x 16 bytes) per group.
 inline size_t qs_workspace_bytes(int64_t rows, int64_t cols, int G, int group) {
   if (group == 0) return 0;
   const int64_t ngroups = group == 1 ? rows : 1;
-  return (size_t)((ngroups * 4 + 15) / 16 * 16) + (size_t)ngroups * 80;
+  return (size_t)((ngroups * 4 + 15) / 16 * 16) + (size_t)((ngroups + 15) / 16 * 16) + (size_t)ngroups * 80;
 }
 
 template <int FMT, typename T>
@@ -1016,17 +1141,30 @@ static cudaError_t launch_qs_t(int G, int group, int rule, const void* xv, int64
   }
   const int64_t glen = group == 1 ? cols : n;
   const int64_t ngroups = n / glen;
-  uint32_t* amax = static_cast<uint32_t*>(ws);
-  unsigned long long* D = reinterpret_cast<unsigned long long*>(static_cast<uint8_t*>(ws) + (ngroups * 4 + 15) / 16 * 16);
+  uint8_t* w8 = static_cast<uint8_t*>(ws);
+  uint32_t* amax = reinterpret_cast<uint32_t*>(w8);
+  int8_t* gscale = reinterpret_cast<int8_t*>(w8 + (ngroups * 4 + 15) / 16 * 16);
+  unsigned long long* D =
+      reinterpret_cast<unsigned long long*>(w8 + (ngroups * 4 + 15) / 16 * 16 + (ngroups + 15) / 16 * 16);
   cudaError_t e = cudaMemsetAsync(ws, 0, qs_workspace_bytes(rows, cols, G, group), st);
   if (e != cudaSuccess) return e;
+  const int64_t cpg = (glen + QS_SPAN - 1) / QS_SPAN;  // spans per group
+  const unsigned nspan = (unsigned)(ngroups * cpg);
+  qs_gmax_kernel<T><<<nspan, 256, 0, st>>>(x, glen, cpg, amax, status);
+  if (rule == 1) qs_mse_kernel<FMT, T><<<nspan, 256, 0, st>>>(x, glen, cpg, amax, D);
+  int64_t cg = (ngroups + 255) / 256;
+  qs_choose_kernel<FMT><<<(unsigned)(cg < 1024 ? cg : 1024), 256, 0, st>>>(amax, rule == 1 ? D : nullptr, rule,
+                                                                        ngroups, gscale);
+  // encode: the register-fed block quantizer with the group's scale per block
+  // (16-byte aligned input), else element by element
+  if ((reinterpret_cast<uintptr_t>(x) & 15) == 0) {
+    const int64_t bpg = glen / G;
+    return launch_q_grouped<FMT, T>(G, x, rows, cols, codes, scales, status, st, sms, gscale, bpg);
+  }
   int64_t grid = (n + 255) / 256;
   if (grid > (int64_t)sms * 8) grid = (int64_t)sms * 8;
-  const unsigned g = (unsigned)(grid < 1 ? 1 : grid);
-  qs_stats_kernel<T><<<g, 256, 0, st>>>(x, n, glen, amax, status);
-  if (rule == 1) qs_mse_kernel<FMT, T><<<g, 256, 0, st>>>(x, n, glen, amax, D);
-  qs_encode_kernel<FMT, T><<<g, 256, 0, st>>>(x, n, glen, G, rule, amax, rule == 1 ? D : nullptr, codes, scales,
-                                               status);
+  qs_encode_scalar_kernel<FMT, T><<<(unsigned)(grid < 1 ? 1 : grid), 256, 0, st>>>(x, n, glen, G, gscale, codes,
+                                                                                   scales, status);
   return cudaGetLastError();
 }
 
