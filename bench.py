@@ -712,6 +712,7 @@ def run_reference(args):
 def run_only(args):
     """One kernel of the path, a few launches, no timing: the target of the
     ncu captures (--only gemm: the step's GEMM (GEMM_ALGO) of the workload above;
+    --only tile: the tile kernel (TENSOR) on the same problem;
     --only quantize: 2^28 BF16 elements, E4C3, block 32; skinny, narrow,
     reuse, r89: the decode GEMM, the few-row tensor-core GEMM, the
     reused-operand dgrad and the r = 2^{8/9} GEMM)."""
@@ -722,14 +723,15 @@ def run_only(args):
 
     dev = torch.device("cuda", 0)
     cfp.load()
-    if args.only == "gemm":
+    if args.only in ("gemm", "tile"):  # the step's GEMM, or the tile kernel (TENSOR) on the same problem
         X, W = inputs.llama7b_linear(M, K, N)
         a, sa = cfp.quantize(torch.from_numpy(X).to(dev), FMT, G, 0)
         b, sb = cfp.quantize(torch.from_numpy(W).to(dev), FMT, G, 0)
+        algo = GEMM_ALGO if args.only == "gemm" else "tensor"
         for _ in range(args.steps):
-            c = cfp.gemm(a, sa, b, sb, FMT, FMT, G, GEMM_ALGO)
+            c = cfp.gemm(a, sa, b, sb, FMT, FMT, G, algo)
         torch.cuda.synchronize()
-        print(json.dumps({"only": "gemm", "launches": args.steps, "c00": float(c[0, 0])}))
+        print(json.dumps({"only": args.only, "algo": algo, "launches": args.steps, "c00": float(c[0, 0])}))
     elif args.only == "quantize":
         x = inputs.bandwidth_tensor_cuda(1 << 28, 4096, 3)
         for _ in range(args.steps):
@@ -778,7 +780,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--only", choices=["gemm", "quantize", "skinny", "narrow", "reuse", "r89"], default=None)
+    ap.add_argument("--only", choices=["gemm", "tile", "quantize", "skinny", "narrow", "reuse", "r89"], default=None)
     ap.add_argument("--narrow-m", type=int, default=16, help="activation rows of --only narrow")
     ap.add_argument("--no-sweep", action="store_true", help="skip the other workloads (quantize sweep, GEMM shapes)")
     ap.add_argument("--out", default=None, help="also write the JSON line to this file (atomically: temp + rename)")
