@@ -210,6 +210,10 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
     sh.abort_flag = 0;
   }
   if (warp == Cfg::MMA_WARP) {
+    // TMEM allocation and release are warp-collective (.sync.aligned): the
+    // MMA warp reaches them, and every wait of its loop (whole-warp waits),
+    // with all 32 lanes together
+    __syncwarp();
     tc::tmem_alloc(&sh.tmem_base, 512);
     tc::tmem_relinquish();
   }
@@ -575,6 +579,7 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
   tc::fence_before_sync();
   __syncthreads();
   if (warp == Cfg::MMA_WARP) {
+    __syncwarp();
     tc::fence_after_sync();
     tc::tmem_dealloc(tmem, 512);
   }
