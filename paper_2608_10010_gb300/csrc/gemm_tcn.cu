@@ -75,6 +75,7 @@ struct TcnCfg {
   static constexpr int NJ = HB;           // sparse MMAs per step
   static constexpr int PO = HB * WW;      // lattice distance of the partner plane
   static constexpr int RB0 = L - (NJ - 1) * WW, NRB = 2 * L - RB0;
+  static_assert(2 * PO == L && Fmt<FX>::K == L && RB0 > PO, "partner planes half the lattice apart");
   static constexpr int ROWB = 64;         // bytes of one operand row (logical K 64)
   static constexpr int PBX = FX == CURVEFP_E5C2 ? 1 : 0;  // X planes one binade low
   // TMEM columns: accumulators, W units, metadata (8 per unit, 2 used), A
@@ -127,22 +128,32 @@ __device__ __forceinline__ int row_ref(const int8_t* s, int nb) {
 // Metadata word of 16 codes (four code words) of a 2:4 operand with 8-bit
 // elements: per chunk of two elements, position bit(2c) and 2 + bit(2c + 1),
 // where bit is the curve-index bit MBIT that selects the partner plane.
-template <int MBIT>
-__device__ __forceinline__ uint32_t pair_meta(uint32_t w0, uint32_t w1, uint32_t w2, uint32_t w3) {
-  const uint32_t w[4] = {w0, w1, w2, w3};
-  uint32_t m = 0;
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const uint32_t t = (w[q] >> MBIT) & 0x01010101u;  // bit of element i at 8 i
-    m |= (((t * 0x01041040u) >> 24) | 0x88u) << (8 * q);  // ... at 2 i, plus bit 3 of each nibble
-  }
-  return m;
-}
-
+// Element c = 4q + i (byte i of word q) puts its bit at bit 2c = 8q + 2i:
+// gathering the four words' bits side by side puts it at 8i + 2q, a 4 x 4
+// matrix of 2-bit cells stored transposed, which two delta swaps (the
+// off-diagonal 2 x 2 blocks, then the off-diagonal cells of each block)
+// transpose.
 // Interleave two words (elements 4q..4q+3 each) into X0 Y0 X1 Y1 | X2 Y2 X3 Y3.
 __device__ __forceinline__ uint2 interleave2(uint32_t x, uint32_t y) {
   return make_uint2(__byte_perm(x, y, 0x5140), __byte_perm(x, y, 0x7362));
 }
+
+template <int MBIT>
+__device__ __forceinline__ uint32_t pair_meta(uint32_t w0, uint32_t w1, uint32_t w2, uint32_t w3) {
+  const uint32_t w[4] = {w0, w1, w2, w3};
+  uint32_t a = 0;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int sh = MBIT - 2 * q;  // bit MBIT of byte i -> bit 8 i + 2 q
+    a |= (sh >= 0 ? w[q] >> sh : w[q] << -sh) & (0x01010101u << (2 * q));
+  }
+  uint32_t t = (a ^ (a >> 12)) & 0x0000F0F0u;
+  a ^= t ^ (t << 12);
+  t = (a ^ (a >> 6)) & 0x00CC00CCu;
+  a ^= t ^ (t << 6);
+  return a | 0x88888888u;  // bit 3 of each nibble: the second element's position is 2 + bit
+}
+
 
 __device__ __forceinline__ bool wait_all(uint64_t* bar, uint32_t parity) {
   return __all_sync(0xffffffffu, tc::mbar_wait(bar, parity));
@@ -475,32 +486,71 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
         if (xrow[e] < 0) continue;
         bool keep;
         const uint32_t sf = mx_sf(raw[e] - xref[e], Cfg::PBX, keep);
-        uint32_t pv[2][8], pc[2][8];
+        constexpr int C = Fmt<FX>::C;
+        if constexpr (C == 3) {
+          // Three curve-index bits.  R block b holds Q_b[k] in byte 2k and Q_{b-PO}[k] in byte 2k + 1 (Q
+          // block u < L: the carry copy of plane u, u >= L: plane u - L).  With
+          // PO = L/2 the two planes share their two low curve-index bits (class
+          // b mod PO) and differ in the top bit T, so a code of that class sits
+          // in the even byte where its T equals the top bit of b mod L, else in
+          // the odd byte.  Per 16-bit lane (one code) three words place the
+          // code's value by its T: qcc for b < L (carry copies on both sides;
+          // b mod L has T = 1), qpc for L <= b < L + PO (plain even, carry odd;
+          // T = 0) and qpp for b >= L + PO (plain, T = 1); block b is its word
+          // masked to the codes of class b mod PO.
+          uint32_t qcc[4], qpc[4], qpp[4], dm0[4], dm1[4];
 #pragma unroll
-        for (int q = 0; q < 2; ++q) {
-          const uint32_t w = q ? cw[e].y : cw[e].x;
-          uint32_t v, vc, mk[4];
-          mx_word<FX, Cfg::PBX>(keep ? w : 0u, v, vc);
-          k_masks<PLANE_E5M2, Fmt<FX>::C>(w, mk);
-          planes_of<Fmt<FX>::C>(v, mk, pv[q]);
-          planes_of<Fmt<FX>::C>(vc, mk, pc[q]);
-        }
-        // R block b interleaves Q block b with Q block b - PO; Q block u < L
-        // is the carry copy of plane u, u >= L plane u - L
+          for (int q = 0; q < 2; ++q) {
+            const uint32_t w = q ? cw[e].y : cw[e].x;
+            uint32_t v, vc;
+            mx_word<FX, Cfg::PBX>(keep ? w : 0u, v, vc);
+            const uint32_t wt = w << (8 - C), w0 = w << 7, w1 = w << 6;  // bits C - 1, 0, 1 -> bit 7
 #pragma unroll
-        for (int b = Cfg::RB0; b < 2 * L; ++b) {
-          uint2 lo, hi;
-          {
-            const uint32_t x = b < L ? pc[0][b] : pv[0][b - L];
-            const uint32_t y = b - Cfg::PO < L ? pc[0][b - Cfg::PO] : pv[0][b - Cfg::PO - L];
-            lo = interleave2(x, y);
+            for (int hh = 0; hh < 2; ++hh) {
+              // lanes of codes 4q + 2hh and 4q + 2hh + 1: duplicated sign
+              // masks, duplicated values, (plain, carry) interleaved
+              const uint32_t sdup = hh ? 0xBBAAu : 0x9988u, dup = hh ? 0x3322u : 0x1100u, ilv = hh ? 0x7362u : 0x5140u;
+              const int i = 2 * q + hh;
+              const uint32_t dt = prmt_sign(wt, sdup);
+              dm0[i] = prmt_sign(w0, sdup);
+              dm1[i] = prmt_sign(w1, sdup);
+              qcc[i] = __byte_perm(vc, vc, dup) & (dt ^ 0xFF00FF00u);
+              qpp[i] = __byte_perm(v, v, dup) & (dt ^ 0xFF00FF00u);
+              qpc[i] = __byte_perm(v, vc, ilv) & (dt ^ 0x00FF00FFu);
+            }
           }
-          {
-            const uint32_t x = b < L ? pc[1][b] : pv[1][b - L];
-            const uint32_t y = b - Cfg::PO < L ? pc[1][b - Cfg::PO] : pv[1][b - Cfg::PO - L];
-            hi = interleave2(x, y);
+#pragma unroll
+          for (int b = Cfg::RB0; b < 2 * L; ++b) {
+            const int j = b % Cfg::PO;
+            uint32_t r[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const uint32_t src = b < L ? qcc[i] : (b < L + Cfg::PO ? qpc[i] : qpp[i]);
+              r[i] = src & ((j & 1) ? dm0[i] : ~dm0[i]) & ((j & 2) ? dm1[i] : ~dm1[i]);
+            }
+            *reinterpret_cast<uint4*>(stg + xbase[e] + (b - Cfg::RB0) * bstride) = make_uint4(r[0], r[1], r[2], r[3]);
           }
-          *reinterpret_cast<uint4*>(stg + xbase[e] + (b - Cfg::RB0) * bstride) = make_uint4(lo.x, lo.y, hi.x, hi.y);
+        } else {
+          // Two curve-index bits: the tokens' planes of each word and their
+          // carry copies, then per R block Q_b and Q_{b-PO} interleaved
+          uint32_t pv[2][8], pc[2][8];
+#pragma unroll
+          for (int q = 0; q < 2; ++q) {
+            const uint32_t w = q ? cw[e].y : cw[e].x;
+            uint32_t v, vc, mk[4];
+            mx_word<FX, Cfg::PBX>(keep ? w : 0u, v, vc);
+            k_masks<PLANE_E5M2, C>(w, mk);
+            planes_of<C>(v, mk, pv[q]);
+            planes_of<C>(vc, mk, pc[q]);
+          }
+#pragma unroll
+          for (int b = Cfg::RB0; b < 2 * L; ++b) {
+            const uint2 lo = interleave2(b < L ? pc[0][b] : pv[0][b - L],
+                                         b - Cfg::PO < L ? pc[0][b - Cfg::PO] : pv[0][b - Cfg::PO - L]);
+            const uint2 hi = interleave2(b < L ? pc[1][b] : pv[1][b - L],
+                                         b - Cfg::PO < L ? pc[1][b - Cfg::PO] : pv[1][b - Cfg::PO - L]);
+            *reinterpret_cast<uint4*>(stg + xbase[e] + (b - Cfg::RB0) * bstride) = make_uint4(lo.x, lo.y, hi.x, hi.y);
+          }
         }
         if (xtok[e] >= 0) {
           const uint32_t sw = sf * 0x01010101u;

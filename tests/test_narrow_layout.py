@@ -232,3 +232,116 @@ def test_plane_bytes_of_every_code_in_every_lane(fmt, bias):
             assert e5m2_value((v >> (8 * lane)) & 0xFF) == want_v, (c, lane)
             if fmt != "E5C2" or bias == 1:
                 assert e5m2_value((vc >> (8 * lane)) & 0xFF) == want_c, (c, lane)
+
+
+# ---- byte-level emulation of the activation R blocks and the weight metadata
+
+def byte_perm(x, y, s):
+    """__byte_perm(x, y, s): result byte i = byte (nibble i of s) of y:x."""
+    src = (x & M32) | (y & M32) << 32
+    return sum(((src >> (8 * ((s >> (4 * i)) & 7))) & 0xFF) << (8 * i) for i in range(4))
+
+
+def r_blocks_emulated(w2, fx, bias, L, PO, RB0):
+    """The X producer's R blocks for one work item (8 codes in two words),
+    as gemm_tcn.cu forms them: three byte-duplicated words placed by the top
+    curve-index bit, masked per block to the codes of class b mod PO."""
+    C = FMTS[fx][1]
+    qcc, qpc, qpp, dm0, dm1 = [0] * 4, [0] * 4, [0] * 4, [0] * 4, [0] * 4
+    for q in range(2):
+        w = w2[q]
+        v, vc = mx_word(w, fx, bias)
+        wt, w0, w1 = (w << (8 - C)) & M32, (w << 7) & M32, (w << 6) & M32
+        for hh in range(2):
+            sdup, dup, ilv = (0xBBAA, 0x3322, 0x7362) if hh else (0x9988, 0x1100, 0x5140)
+            i = 2 * q + hh
+            dt = prmt_sign(wt, sdup)
+            dm0[i] = prmt_sign(w0, sdup)
+            dm1[i] = prmt_sign(w1, sdup)
+            qcc[i] = byte_perm(vc, vc, dup) & (dt ^ 0xFF00FF00)
+            qpp[i] = byte_perm(v, v, dup) & (dt ^ 0xFF00FF00)
+            qpc[i] = byte_perm(v, vc, ilv) & (dt ^ 0x00FF00FF)
+    out = {}
+    for b in range(RB0, 2 * L):
+        j = b % PO
+        words = []
+        for i in range(4):
+            src = qcc[i] if b < L else (qpc[i] if b < L + PO else qpp[i])
+            words.append(src & (dm0[i] if j & 1 else ~dm0[i] & M32) & (dm1[i] if j & 2 else ~dm1[i] & M32))
+        out[b] = b"".join(x.to_bytes(4, "little") for x in words)
+    return out
+
+
+def r_blocks_defined(w2, fx, bias, L, PO, RB0):
+    """R_b[2k] = Q_b[k], R_b[2k + 1] = Q_{b - PO}[k]; Q_u = the carry bytes
+    of the codes of plane u (u < L), the plain bytes of plane u - L (u >= L);
+    a code's plane is its curve index (low C bits)."""
+    C = FMTS[fx][1]
+    codes, vb, cb = [], [], []
+    for w in w2:
+        v, vc = mx_word(w, fx, bias)
+        for lane in range(4):
+            codes.append((w >> (8 * lane)) & 0xFF)
+            vb.append((v >> (8 * lane)) & 0xFF)
+            cb.append((vc >> (8 * lane)) & 0xFF)
+
+    def Q(u, k):
+        plane = codes[k] & ((1 << C) - 1)
+        if u < L:
+            return cb[k] if plane == u else 0
+        return vb[k] if plane == u - L else 0
+
+    return {b: bytes(x for k in range(8) for x in (Q(b, k), Q(b - PO, k))) for b in range(RB0, 2 * L)}
+
+
+@pytest.mark.parametrize("fx,fw", [("E3C3", "E3C3"), ("E4C3", "E4C3"), ("E4C3", "E5C2")])
+def test_r_blocks_are_the_interleaved_q_blocks(fx, fw):
+    """The R blocks the activation producers store for three curve-index bits
+    (16 bytes per block and work item) equal their definition byte for byte,
+    for every such kernel orientation's lattice (L, PO, first block) and
+    random codes (zeros, both signs, every curve index).  (E5C2 tokens keep
+    the per-plane masks and byte interleave, which the algebra tests above
+    model.)"""
+    KX, KW = 1 << FMTS[fx][1], 1 << FMTS[fw][1]
+    L = max(KX, KW)
+    WW, HB = L // KW, KW // 2
+    PO, RB0 = HB * WW, L - (HB - 1) * WW
+    bias = 1 if fx == "E5C2" else 0
+    rng = np.random.default_rng(29)
+    valid = np.array([c for c in range(256) if not (fx == "E3C3" and c & 0x40)], np.int64)
+    for _ in range(3000):
+        c = rng.choice(valid, size=8)
+        if rng.random() < 0.2:
+            c[rng.integers(0, 8)] = 0  # zero codes
+        w2 = [int(c[0] | c[1] << 8 | c[2] << 16 | c[3] << 24), int(c[4] | c[5] << 8 | c[6] << 16 | c[7] << 24)]
+        assert r_blocks_emulated(w2, fx, bias, L, PO, RB0) == r_blocks_defined(w2, fx, bias, L, PO, RB0), c
+
+
+def pair_meta_emulated(w, mbit):
+    """gemm_tcn.cu pair_meta: gather the selector bits of four code words,
+    transpose the 4 x 4 matrix of 2-bit cells with two delta swaps."""
+    a = 0
+    for q in range(4):
+        sh = mbit - 2 * q
+        a |= ((w[q] >> sh) if sh >= 0 else (w[q] << -sh)) & (0x01010101 << (2 * q)) & M32
+    t = (a ^ (a >> 12)) & 0x0000F0F0
+    a ^= t ^ (t << 12)
+    t = (a ^ (a >> 6)) & 0x00CC00CC
+    a ^= t ^ (t << 6)
+    return (a | 0x88888888) & M32
+
+
+@pytest.mark.parametrize("mbit", [1, 2])
+def test_pair_metadata_selects_the_partner_plane(mbit):
+    """Metadata of 16 codes of a 2:4 operand with 8-bit elements: per chunk of
+    two elements (codes 2c, 2c + 1) the positions bit(2c) and 2 + bit(2c + 1)
+    of the curve-index bit that selects the partner plane (nibble c)."""
+    rng = np.random.default_rng(31)
+    for _ in range(20000):
+        w = [int(x) for x in rng.integers(0, 1 << 32, size=4, dtype=np.uint64)]
+        codes = [(w[k // 4] >> (8 * (k % 4))) & 0xFF for k in range(16)]
+        want = 0
+        for c in range(8):
+            b0, b1 = (codes[2 * c] >> mbit) & 1, (codes[2 * c + 1] >> mbit) & 1
+            want |= (b0 | (2 + b1) << 2) << (4 * c)
+        assert pair_meta_emulated(w, mbit) == want, w
