@@ -92,11 +92,11 @@ typedef enum {
  * fastest tensor-core kernel at every M.  In both tensor-core kernels the
  * block scales enter the MMAs as UE8M0 scale factors (block-scaled MMAs), so
  * the plane values are the codes' own powers of two.
- * AUTO (measured on the FFN shapes, N = 14336, K = 4096, and the
- * 2048 x 4096 x 4096 linear): SKINNY for M <= CURVEFP_AUTO_SKINNY_M;
- * TENSOR_NARROW for same-format pairs, and for the mixed pairs up to
- * CURVEFP_AUTO_NARROW_M; TENSOR above; SKINNY up to CURVEFP_SKINNY_MAX_M for
- * pairs without a tensor-core kernel.  (Value 2 is not an algorithm.) */
+ * AUTO (measured on the FFN shapes, N = 14336, K = 4096, the
+ * 2048 x 4096 x 4096 linear and the training triplet's three GEMMs): SKINNY
+ * for M <= CURVEFP_AUTO_SKINNY_M; TENSOR_NARROW for every pair it supports;
+ * TENSOR for r = 2^{8/9}; SKINNY up to CURVEFP_SKINNY_MAX_M for pairs without
+ * a tensor-core kernel.  (Value 2 is not an algorithm.) */
 typedef enum {
   CURVEFP_GEMM_EXACT = 0,
   CURVEFP_GEMM_TENSOR = 1,
@@ -106,7 +106,6 @@ typedef enum {
 } curvefp_gemm_algo_t;
 #define CURVEFP_SKINNY_MAX_M 8
 #define CURVEFP_AUTO_SKINNY_M 1
-#define CURVEFP_AUTO_NARROW_M 96
 
 /* Bits of the device status word. */
 #define CURVEFP_DEV_NAN 1u     /* quantize: a NaN input was encoded as 0x00        */

@@ -148,13 +148,13 @@ curvefp_status_t curvefp_gemm(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, 
   // rational radix: EXACT, and TENSOR for r = 2^{8/9}
   if (fmt_radix(fmt_a) && algo != CURVEFP_GEMM_TENSOR) return CURVEFP_ERR_UNSUPPORTED;
   // AUTO: the fastest kernel by M (measured on the FFN and Llama-like
-  // shapes): CUDA cores for one row; phases along N for every larger M with
-  // a same-format pair (2:4-sparse pair planes) and up to 96 rows for the
-  // mixed pairs (dense planes); tiles above
+  // shapes and the training triplet): CUDA cores for one row; phases along N
+  // (2:4-sparse pair planes) for every larger M of the pairs that kernel
+  // takes; tiles for the rest
   if (algo == CURVEFP_GEMM_AUTO) {
     if (M <= CURVEFP_AUTO_SKINNY_M)
       algo = CURVEFP_GEMM_SKINNY;
-    else if (cfp::gemm_narrow_supported(fmt_a, fmt_b) && (fmt_a == fmt_b || M <= CURVEFP_AUTO_NARROW_M))
+    else if (cfp::gemm_narrow_supported(fmt_a, fmt_b))
       algo = CURVEFP_GEMM_TENSOR_NARROW;
     else if (M <= CURVEFP_SKINNY_MAX_M && !cfp::gemm_tensor_supported(fmt_a, fmt_b))
       algo = CURVEFP_GEMM_SKINNY;
