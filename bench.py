@@ -715,7 +715,8 @@ def run_only(args):
     --only tile: the tile kernel (TENSOR) on the same problem;
     --only quantize: 2^28 BF16 elements, E4C3, block 32; skinny, narrow,
     reuse, r89: the decode GEMM, the few-row tensor-core GEMM, the
-    reused-operand dgrad and the r = 2^{8/9} GEMM)."""
+    reused-operand dgrad and the r = 2^{8/9} GEMM; static: the static
+    quantizer with row groups and the MSE search, E3C3, W[4096 x 4096])."""
     import torch
 
     import paper_2608_10010_gb300 as cfp
@@ -754,6 +755,12 @@ def run_only(args):
             c = cfp.gemm(a, sa, b, sb, "E3C3", "E3C3", G, "tensor_narrow")
         torch.cuda.synchronize()
         print(json.dumps({"only": "narrow", "M": args.narrow_m, "launches": args.steps, "c00": float(c[0, 0])}))
+    elif args.only == "static":  # static scales: row groups, MSE search, E3C3 W[4096 x 4096] ~ N(0, 0.02^2)
+        Wt = torch.randn((4096, 4096), device=dev, generator=torch.Generator(device=dev).manual_seed(4)) * 0.02
+        for _ in range(args.steps):
+            codes, scales = cfp.quantize_static(Wt, "E3C3", G, "row", "mse")
+        torch.cuda.synchronize()
+        print(json.dumps({"only": "static", "launches": args.steps, "scale0": int(scales[0, 0])}))
     elif args.only == "reuse":  # dgrad on the reused weight, triplet shape (T 4096, 4096 -> 11008)
         X, Wt, dY = inputs.training_triplet_cuda()
         qw, sw = cfp.quantize(Wt, "E4C3", G, 1)
@@ -780,7 +787,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--only", choices=["gemm", "tile", "quantize", "skinny", "narrow", "reuse", "r89"], default=None)
+    ap.add_argument("--only", choices=["gemm", "tile", "quantize", "skinny", "narrow", "reuse", "r89", "static"],
+                    default=None)
     ap.add_argument("--narrow-m", type=int, default=16, help="activation rows of --only narrow")
     ap.add_argument("--no-sweep", action="store_true", help="skip the other workloads (quantize sweep, GEMM shapes)")
     ap.add_argument("--out", default=None, help="also write the JSON line to this file (atomically: temp + rename)")

@@ -817,6 +817,123 @@ __device__ __forceinline__ unsigned __int128 sq_term(float x, float xhat, int ac
   return sh <= -128 ? (unsigned __int128)0 : sq >> (-sh);
 }
 
+// ---- the five MSE candidates of one element, sharing the scale-free work --
+// The code of x at scale a (encode_slow) depends on a only through the binade
+// test of Fv = Fx - a: the saturation code, zero, the smallest level (m
+// clamped to 1) or the interior code K Fv + j + B, whose reconstruction
+// (recon_f32) RN32(2^{k/K}) 2^{a + e} has a + e = Fx + [j = K] and
+// k = j mod K whatever a is.  So an element needs one midpoint count and one
+// interior value, and per candidate a class and one exact term.
+
+// |v| of a finite FP32 bit pattern as M 2^E (M >= 0; f32_int's split).
+__device__ __forceinline__ void f32_mag(uint32_t absb, int& M, int& E) {
+  const int ef = (int)(absb >> 23);
+  const int mm = (int)(absb & 0x7FFFFFu);
+  M = ef ? (mm | 0x800000) : mm;
+  E = ef ? ef - 150 : -149;
+}
+
+// The candidates of one group (scale ac): their scales and, as M 2^E, their
+// saturation level (code 2B - 1) and smallest level (code 1).
+struct MseCands {
+  int ac, a[5], Ms[5], Es[5], Ml[5], El[5];
+  bool valid[5];
+};
+template <int FMT>
+__device__ __forceinline__ MseCands mse_cands(int ac) {
+  MseCands c;
+  c.ac = ac;
+#pragma unroll
+  for (int k = 0; k < 5; ++k) {
+    const int a = ac - 3 + k;
+    c.a[k] = a;
+    c.valid[k] = a >= -128 && a <= 127;
+    f32_mag(__float_as_uint(recon_f32<FMT>((uint32_t)(2 * Fmt<FMT>::B - 1), a)) & 0x7FFFFFFFu, c.Ms[k], c.Es[k]);
+    f32_mag(__float_as_uint(recon_f32<FMT>(1u, a)) & 0x7FFFFFFFu, c.Ml[k], c.El[k]);
+  }
+  return c;
+}
+
+// floor(q 2^sh) for q = ad^2 as a 128-bit integer (sq_term's shift; sh >= 128
+// reads 0 as there).
+__device__ __forceinline__ unsigned __int128 sq_shift(uint32_t ad, int sh) {
+  const unsigned long long q = (unsigned long long)ad * ad;
+  unsigned long long lo = 0ull, hi = 0ull;
+  if (sh >= 0) {
+    if (sh < 64) {
+      lo = q << sh;
+      hi = sh ? q >> (64 - sh) : 0ull;
+    } else if (sh < 128) {
+      hi = q << (sh - 64);
+    }
+  } else if (sh > -64) {
+    lo = q >> -sh;
+  }
+  return ((unsigned __int128)hi << 64) | lo;
+}
+
+// Adds the five terms floor((x - xhat_a)^2 2^{60 - 2 ac}) of a finite, non-NaN
+// element (bits b) to acc, exactly as sq_term(x, recon_f32(encode_slow(x, a),
+// a), ac) per candidate.  Returns false, adding nothing, where the element
+// takes the general path: an interior value outside FP32's normal range, or
+// a reconstruction more than 8 binades from x (the integer difference then
+// needs more than 32 bits).  ck: the K values RN32(2^{k/K}) as FP32 bits.
+template <int FMT>
+__device__ __forceinline__ bool mse_add5(const uint32_t* lut, const uint32_t* ck, uint32_t b, const MseCands& c,
+                                         unsigned __int128 (&acc)[5]) {
+  using F = Fmt<FMT>;
+  const uint32_t absb = b & 0x7FFFFFFFu;
+  if (absb == 0u) return true;  // x = 0 reconstructs as 0 at every scale
+  int Fx;
+  uint32_t mant;
+  split_f32(absb, Fx, mant);
+  const int j = mid_count(lut, mant);
+  const int Ei = Fx + (j == F::K ? 1 : 0);
+  if (Ei < -126 || Ei > 127) return false;
+  // x = Mx 2^Ex; the interior value RN32(2^{k/K}) 2^Ei (normal) = Mi 2^{Ei - 23}
+  int Mx, Ex;
+  f32_mag(absb, Mx, Ex);
+  const int Mi = (int)((ck[j & (F::K - 1)] & 0x7FFFFFu) | 0x800000u), Eiv = Ei - 23;
+  // Classes by threshold on a (encode_slow's tests with Fv = Fx - a):
+  // saturated for a < as, zero for a > az, clamped to the smallest level for
+  // a > acl (and not zero), interior otherwise.
+  const int as = Fx - F::EMAX + (j == F::K ? 1 : 0);
+  const int az = Fx - ZeroBoundary<FMT>::FZ - (mant < RadixConst<F::K>::MU_Z ? 1 : 0);
+  const int acl = Fx + (j + F::B - 1) / F::K;  // K (Fx - a) + j + B < 1; j + B - 1 >= 0
+  // the interior term (x and its interior value are within one binade)
+  unsigned __int128 tint;
+  {
+    const int E = min(Ex, Eiv), sx = Ex - E, s2 = Eiv - E;
+    const long long d = (long long)((uint32_t)Mx << sx) - (long long)((uint32_t)Mi << s2);
+    tint = sq_shift((uint32_t)(d < 0 ? -d : d), 2 * E + 60 - 2 * c.ac);
+  }
+  unsigned __int128 t[5];
+  bool ok = true;
+#pragma unroll
+  for (int k = 0; k < 5; ++k) {
+    const int a = c.a[k];
+    const bool sat = a < as, zero = !sat && a > az, clamp = !sat && !zero && a > acl;
+    const bool own = sat || zero || clamp;
+    t[k] = tint;
+    // a candidate's own term only where the element is not interior there
+    // (mostly the saturating scales below a_c); a warp skips the branch when
+    // none of its lanes takes it
+    if (own) {
+      int Mh = sat ? c.Ms[k] : (clamp ? c.Ml[k] : 0);
+      int Eh = sat ? c.Es[k] : (clamp ? c.El[k] : Ex);
+      const int E = min(Ex, Eh), sx = Ex - E, s2 = Eh - E;
+      ok = ok && sx <= 8 && s2 <= 8;
+      const long long d = (long long)((uint32_t)Mx << (sx & 15)) - (long long)((uint32_t)Mh << (s2 & 15));
+      t[k] = sq_shift((uint32_t)(d < 0 ? -d : d), 2 * E + 60 - 2 * c.ac);
+    }
+  }
+  if (!ok) return false;
+#pragma unroll
+  for (int k = 0; k < 5; ++k)
+    if (c.valid[k]) acc[k] += t[k];
+  return true;
+}
+
 // Exact 128-bit accumulation into global memory ([lo, hi] words).
 __device__ __forceinline__ void atomic_add_u128(unsigned long long* p, unsigned __int128 v) {
   const unsigned long long lo = (unsigned long long)v, hi = (unsigned long long)(v >> 64);
@@ -893,10 +1010,11 @@ __device__ __forceinline__ unsigned __int128 warp_sum_u128(unsigned __int128 v) 
 // Per group and candidate: D(a) over the CTA's span, one exact 128-bit
 // atomic add per warp and candidate.
 template <int FMT, typename T>
-__global__ void __launch_bounds__(256) qs_mse_kernel(const T* __restrict__ x, int64_t glen, int64_t cpg,
+__global__ void __launch_bounds__(256, 3) qs_mse_kernel(const T* __restrict__ x, int64_t glen, int64_t cpg,
                                                      const uint32_t* __restrict__ amax, unsigned long long* D) {
-  __shared__ uint32_t lut[256];
+  __shared__ uint32_t lut[256], ck[8];
   for (int i = threadIdx.x; i < 256; i += blockDim.x) lut[i] = __ldg(lut_src<Fmt<FMT>::K>() + i);
+  if (threadIdx.x < 8) ck[threadIdx.x] = Fmt<FMT>::K == 8 ? CFP_CK_F32_K8_DEV[threadIdx.x] : CFP_CK_F32_K4_DEV[threadIdx.x & 3];
   __syncthreads();
   const int64_t g = blockIdx.x / cpg, c = blockIdx.x - g * cpg;
   const uint32_t am = amax[g];
@@ -905,9 +1023,11 @@ __global__ void __launch_bounds__(256) qs_mse_kernel(const T* __restrict__ x, in
   const int64_t i0 = g * glen + c * QS_SPAN, i1 = g * glen + min(glen, (c + 1) * QS_SPAN);
   unsigned __int128 acc[5] = {0, 0, 0, 0, 0};
   bool dummy = false;
-  for (int64_t i = i0 + threadIdx.x; i < i1; i += blockDim.x) {
-    const uint32_t b = load_bits(x, i);
-    if ((b & 0x7FFFFFFFu) > 0x7F800000u) continue;  // NaN: left out
+  [[maybe_unused]] const MseCands cand = mse_cands<FMT>(ac);
+  auto element = [&](uint32_t b) {
+    if ((b & 0x7FFFFFFFu) > 0x7F800000u) return;  // NaN: left out
+    if constexpr (!IsRadix<FMT>::value)
+      if (mse_add5<FMT>(lut, ck, b, cand, acc)) return;
     const float xv = __uint_as_float(b);
 #pragma unroll
     for (int k = 0; k < 5; ++k) {
@@ -915,6 +1035,19 @@ __global__ void __launch_bounds__(256) qs_mse_kernel(const T* __restrict__ x, in
       if (a < -128 || a > 127) continue;
       acc[k] += sq_term(xv, recon_f32<FMT>(encode_slow<FMT>(lut, b, a, dummy), a), ac);
     }
+  };
+  constexpr int VEC = Elem<T>::VEC;
+  if (((i0 | i1) % VEC) == 0 && (reinterpret_cast<uintptr_t>(x) & 15) == 0) {
+    // 16-byte loads: VEC independent elements per thread and iteration
+    const uint4* p = reinterpret_cast<const uint4*>(x + i0);
+    const int64_t nv = (i1 - i0) / VEC;
+    for (int64_t v = threadIdx.x; v < nv; v += blockDim.x) {
+      const uint4 q = __ldcs(p + v);
+#pragma unroll
+      for (int e = 0; e < VEC; ++e) element(Elem<T>::bits(q, e));
+    }
+  } else {
+    for (int64_t i = i0 + threadIdx.x; i < i1; i += blockDim.x) element(load_bits(x, i));
   }
 #pragma unroll
   for (int k = 0; k < 5; ++k) {
@@ -976,29 +1109,48 @@ __global__ void qs_choose_kernel(const uint32_t* __restrict__ amax, const unsign
 // Block groups: one thread per block of G elements does everything in
 // registers (no workspace).
 template <int FMT, typename T>
-__global__ void __launch_bounds__(256) qs_block_kernel(const T* __restrict__ x, int64_t nblk, int G, int rule,
+__global__ void __launch_bounds__(256, 3) qs_block_kernel(const T* __restrict__ x, int64_t nblk, int G, int rule,
                                                        uint8_t* codes, int8_t* scales, uint32_t* status) {
-  __shared__ uint32_t lut[256];
+  __shared__ uint32_t lut[256], ck[8];
   for (int i = threadIdx.x; i < 256; i += blockDim.x) lut[i] = __ldg(lut_src<Fmt<FMT>::K>() + i);
+  if (threadIdx.x < 8) ck[threadIdx.x] = Fmt<FMT>::K == 8 ? CFP_CK_F32_K8_DEV[threadIdx.x] : CFP_CK_F32_K4_DEV[threadIdx.x & 3];
   __syncthreads();
   bool nan = false, dummy = false;
+  // a thread's block with 16-byte loads where the input allows (G is a power
+  // of two >= 32), element by element otherwise
+  constexpr int VEC = Elem<T>::VEC;
+  const bool vec = (reinterpret_cast<uintptr_t>(x) & 15) == 0 && (reinterpret_cast<uintptr_t>(codes) & 7) == 0;
+  auto for_block = [&](int64_t i0, auto&& f) {  // f(element index in the block, bits)
+    if (vec) {
+      const uint4* p = reinterpret_cast<const uint4*>(x + i0);
+      for (int v = 0; v < G / VEC; ++v) {
+        const uint4 q = __ldg(p + v);
+#pragma unroll
+        for (int e = 0; e < VEC; ++e) f(v * VEC + e, Elem<T>::bits(q, e));
+      }
+    } else {
+      for (int i = 0; i < G; ++i) f(i, load_bits(x, i0 + i));
+    }
+  };
   for (int64_t blk = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; blk < nblk;
        blk += (int64_t)gridDim.x * blockDim.x) {
     const int64_t i0 = blk * G;
     uint32_t am = 0u;
-    for (int i = 0; i < G; ++i) {
-      const uint32_t b = load_bits(x, i0 + i) & 0x7FFFFFFFu;
+    for_block(i0, [&](int, uint32_t bits) {
+      const uint32_t b = bits & 0x7FFFFFFFu;
       if (b > 0x7F800000u) nan = true;
       else am = max(am, b);
-    }
+    });
     unsigned long long Dg[10];
     const bool search = rule == 1 && am != 0u && am < 0x7F800000u;
     if (search) {
       const int ac = block_scale<FMT>(am);
       unsigned __int128 acc[5] = {0, 0, 0, 0, 0};
-      for (int i = 0; i < G; ++i) {
-        const uint32_t b = load_bits(x, i0 + i);
-        if ((b & 0x7FFFFFFFu) > 0x7F800000u) continue;
+      [[maybe_unused]] const MseCands cand = mse_cands<FMT>(ac);
+      for_block(i0, [&](int, uint32_t b) {
+        if ((b & 0x7FFFFFFFu) > 0x7F800000u) return;
+        if constexpr (!IsRadix<FMT>::value)
+          if (mse_add5<FMT>(lut, ck, b, cand, acc)) return;
         const float xv = __uint_as_float(b);
 #pragma unroll
         for (int k = 0; k < 5; ++k) {
@@ -1006,7 +1158,7 @@ __global__ void __launch_bounds__(256) qs_block_kernel(const T* __restrict__ x, 
           if (a < -128 || a > 127) continue;
           acc[k] += sq_term(xv, recon_f32<FMT>(encode_slow<FMT>(lut, b, a, dummy), a), ac);
         }
-      }
+      });
       for (int c = 0; c < 5; ++c) {
         Dg[2 * c] = (unsigned long long)acc[c];
         Dg[2 * c + 1] = (unsigned long long)(acc[c] >> 64);
@@ -1014,7 +1166,21 @@ __global__ void __launch_bounds__(256) qs_block_kernel(const T* __restrict__ x, 
     }
     const int a = choose_scale<FMT>(am, Dg, search ? 1 : 0);
     scales[blk] = (int8_t)a;
-    for (int i = 0; i < G; ++i) codes[i0 + i] = (uint8_t)encode_slow<FMT>(lut, load_bits(x, i0 + i), a, dummy);
+    if (vec) {
+      const uint4* p = reinterpret_cast<const uint4*>(x + i0);
+      for (int v = 0; v < G / VEC; ++v) {
+        const uint4 q = __ldg(p + v);
+        uint32_t w[2] = {0u, 0u};
+#pragma unroll
+        for (int e = 0; e < VEC; ++e) w[e >> 2] |= encode_slow<FMT>(lut, Elem<T>::bits(q, e), a, dummy) << (8 * (e & 3));
+        if constexpr (VEC == 4)
+          *reinterpret_cast<uint32_t*>(codes + i0 + v * VEC) = w[0];
+        else
+          *reinterpret_cast<uint2*>(codes + i0 + v * VEC) = make_uint2(w[0], w[1]);
+      }
+    } else {
+      for (int i = 0; i < G; ++i) codes[i0 + i] = (uint8_t)encode_slow<FMT>(lut, load_bits(x, i0 + i), a, dummy);
+    }
   }
   if (nan && status) atomicOr(status, CURVEFP_DEV_NAN);
 }
