@@ -239,16 +239,17 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
         (ar, sar), (br, sbr) = cfp.quantize(Ar, fmt, 512, 0, stream=stream), cfp.quantize(Br, fmt, 512, 0, stream=stream)
         ms_g = _time_ms(torch, stream, lambda: cfp.gemm(ar, sar, br, sbr, fmt, fmt, 512, "exact", stream=stream),
                         flush_l2, reps=3, warm=1)
-        tc_ms = None
-        if fmt in ("E4C3", "E4C3_R8_9"):  # the tensor-core kernel on the Llama-7B-like linear, G512
-            (al, sal), (bl, sbl) = cfp.quantize(Xl, fmt, 512, 0, stream=stream), cfp.quantize(Wl, fmt, 512, 0,
-                                                                                               stream=stream)
-            tc_ms = _time_ms(torch, stream, lambda: cfp.gemm(al, sal, bl, sbl, fmt, fmt, 512, "tensor",
-                                                             out=Cl, stream=stream), flush_l2)
-            del al, sal, bl, sbl
-        res["radix"].append({"format": fmt, "phases": cfp.phase_count(fmt, fmt),
-                             "tensor_gemm_2048x4096x4096_G512_ms": None if tc_ms is None else round(tc_ms, 4),
-                             "tensor_gemm_tops": None if tc_ms is None else round(2 * 2048 * 4096 * 4096 / (tc_ms / 1e3) / 1e12, 3),
+        # the format's tensor-core kernel on the Llama-7B-like linear, G512
+        # (r = 2^{3/4}: 32 phases along N, TENSOR_NARROW)
+        tc_algo = "tensor_narrow" if fmt == "E4C3_R3_4" else "tensor"
+        (al, sal), (bl, sbl) = cfp.quantize(Xl, fmt, 512, 0, stream=stream), cfp.quantize(Wl, fmt, 512, 0,
+                                                                                           stream=stream)
+        tc_ms = _time_ms(torch, stream, lambda: cfp.gemm(al, sal, bl, sbl, fmt, fmt, 512, tc_algo,
+                                                         out=Cl, stream=stream), flush_l2)
+        del al, sal, bl, sbl
+        res["radix"].append({"format": fmt, "phases": cfp.phase_count(fmt, fmt), "tensor_algo": tc_algo,
+                             "tensor_gemm_2048x4096x4096_G512_ms": round(tc_ms, 4),
+                             "tensor_gemm_tops": round(2 * 2048 * 4096 * 4096 / (tc_ms / 1e3) / 1e12, 3),
                              "quantize_fp32_8192x8192_G512_ms": round(ms_q, 4),
                              "quantize_gbs": round(Xr.numel() * (4 + 1 + 1 / 512) / (ms_q / 1e3) / 1e9, 1),
                              "exact_gemm_1024x1024x4096_ms": round(ms_g, 4),

@@ -57,8 +57,10 @@ extern "C" {
  * accepted by curvefp_quantize, curvefp_quantize_static (and its variants),
  * curvefp_dequantize, curvefp_gemm_requant's destination, the EXACT GEMMs
  * (curvefp_gemm, curvefp_gemm_phases, curvefp_gemm_phases_histogram; both
- * operands of the same format) and, for r = 2^{8/9}, curvefp_gemm TENSOR
- * (nine planes per operand, 81 plane pairs, three passes of three phases);
+ * operands of the same format), for r = 2^{8/9} curvefp_gemm TENSOR (nine
+ * planes per operand, 81 plane pairs, three passes of three phases) and for
+ * r = 2^{3/4} curvefp_gemm TENSOR_NARROW (32 planes per operand, 16 pair
+ * planes, the 32 phases along the MMA's N dimension), AUTO picking those;
  * the other algorithms, curvefp_gemm_q32 and curvefp_gemm_oriented return
  * CURVEFP_ERR_UNSUPPORTED for them. */
 typedef enum {
@@ -89,14 +91,18 @@ typedef enum {
  * Eq. 5): a step of 32 codes takes K_w/2 2:4-sparse MMAs of 128 x (L Mt)
  * (weight curve planes j and j + K_w/2 share one compressed operand; Mt <=
  * 256/L tokens per CTA), against K_a K_b dense MMAs of a 128-row tile; the
- * fastest tensor-core kernel at every M.  In both tensor-core kernels the
+ * fastest tensor-core kernel at every M.  For r = 2^{3/4} (32 phases) the
+ * same layout with Mt = 8 tokens: 16 sparse MMAs of 128 x 256 x 64 per step,
+ * one weight stage in TMEM (the 256-column accumulator leaves room for no
+ * second).  In both tensor-core kernels the
  * block scales enter the MMAs as UE8M0 scale factors (block-scaled MMAs), so
  * the plane values are the codes' own powers of two.
  * AUTO (measured on the FFN shapes, N = 14336, K = 4096, the
  * 2048 x 4096 x 4096 linear and the training triplet's three GEMMs): SKINNY
  * for M <= CURVEFP_AUTO_SKINNY_M; TENSOR_NARROW for every pair it supports;
- * TENSOR for r = 2^{8/9}; SKINNY up to CURVEFP_SKINNY_MAX_M for pairs without
- * a tensor-core kernel.  (Value 2 is not an algorithm.) */
+ * TENSOR for r = 2^{8/9} and TENSOR_NARROW for r = 2^{3/4} at every M;
+ * SKINNY up to CURVEFP_SKINNY_MAX_M for pairs without a tensor-core kernel.
+ * (Value 2 is not an algorithm.) */
 typedef enum {
   CURVEFP_GEMM_EXACT = 0,
   CURVEFP_GEMM_TENSOR = 1,
@@ -224,8 +230,9 @@ curvefp_status_t curvefp_dequantize(curvefp_format_t fmt, int block, const uint8
  *   75 binades of the row's largest block scale on both operands (the
  *   quantizer writes 0 as the scale of an all-zero block, so this holds
  *   unless both operands' data lie below about 2^-75).  Format pairs: E3C3 x
- *   E3C3, E4C3 x E4C3, E5C2 x E4C3, E4C3 x E5C2, E5C2 x E5C2, and (TENSOR)
- *   E4C3_R8_9 x E4C3_R8_9 (others return CURVEFP_ERR_UNSUPPORTED).  TENSOR and
+ *   E3C3, E4C3 x E4C3, E5C2 x E4C3, E4C3 x E5C2, E5C2 x E5C2, (TENSOR)
+ *   E4C3_R8_9 x E4C3_R8_9 and (TENSOR_NARROW) E4C3_R3_4 x E4C3_R3_4 (others
+ *   return CURVEFP_ERR_UNSUPPORTED).  TENSOR and
  *   TENSOR_NARROW zero parts of C with cudaMemsetAsync before adding split-K
  *   pieces to them (two additions per output, so results do not depend on
  *   their order).

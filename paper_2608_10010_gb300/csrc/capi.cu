@@ -145,8 +145,12 @@ curvefp_status_t curvefp_gemm(curvefp_gemm_algo_t algo, curvefp_format_t fmt_a, 
   if (algo == CURVEFP_GEMM_EXACT)
     return from_cuda(cfp::launch_gemm_exact(fmt_a, fmt_b, block, a, sa, b, sb, M, N, K, c, nullptr, nullptr,
                                             device_status, st));
-  // rational radix: EXACT, and TENSOR for r = 2^{8/9}
-  if (fmt_radix(fmt_a) && algo != CURVEFP_GEMM_TENSOR) return CURVEFP_ERR_UNSUPPORTED;
+  // rational radix: EXACT, TENSOR for r = 2^{8/9}, TENSOR_NARROW for
+  // r = 2^{3/4}; AUTO picks the tensor-core kernel of the format
+  if (fmt_radix(fmt_a) && algo == CURVEFP_GEMM_AUTO)
+    algo = fmt_a == CURVEFP_E4C3_R3_4 ? CURVEFP_GEMM_TENSOR_NARROW : CURVEFP_GEMM_TENSOR;
+  if (fmt_radix(fmt_a) && algo != CURVEFP_GEMM_TENSOR && algo != CURVEFP_GEMM_TENSOR_NARROW)
+    return CURVEFP_ERR_UNSUPPORTED;
   // AUTO: the fastest kernel by M (measured on the FFN and Llama-like
   // shapes and the training triplet): CUDA cores for one row; phases along N
   // (2:4-sparse pair planes) for every larger M of the pairs that kernel

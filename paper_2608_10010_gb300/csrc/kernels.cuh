@@ -26,6 +26,9 @@ bool gemm_narrow_supported(int fa, int fb);
 cudaError_t launch_gemm_tensor_narrow(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
                                       const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, uint32_t* status,
                                       cudaStream_t st, int sms);
+cudaError_t launch_gemm_tensor_narrow_r34(int G, const uint8_t* x, const int8_t* sx, const uint8_t* w,
+                                          const int8_t* sw, int64_t M, int64_t N, int64_t K, float* c,
+                                          uint32_t* st, cudaStream_t s, int sms);
 bool is_radix_format(int fmt);
 cudaError_t launch_gemm_skinny(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
                                const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, cudaStream_t st, int sms);

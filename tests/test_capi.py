@@ -145,6 +145,7 @@ def test_rational_radix_host_rules(lib):
     # GEMM: mixed radix, and the tensor-core algorithms
     assert lib.curvefp_gemm(0, 3, 1, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED
     assert lib.curvefp_gemm(1, 4, 4, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED  # r = 2^{3/4}
+    assert lib.curvefp_gemm(5, 3, 3, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED  # narrow, r = 2^{8/9}
     assert lib.curvefp_gemm(3, 3, 3, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED  # skinny
     assert lib.curvefp_gemm(2, 4, 4, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED
     assert lib.curvefp_gemm_q32(3, 3, 32, d, d, d, d, 4, 4, 64, d, None, None) == UNSUPPORTED

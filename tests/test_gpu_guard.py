@@ -91,7 +91,8 @@ def test_static_quantize_stays_inside(torch, group, rule):
                                         ("tensor_narrow", "E5C2", "E4C3"), ("skinny", "E4C3", "E5C2"),
                                         ("auto", "E4C3", "E4C3"), ("exact", "E4C3_R3_4", "E4C3_R3_4"),
                                         ("tensor_narrow", "E3C3", "E3C3"), ("tensor_narrow", "E5C2", "E5C2"),
-                                        ("tensor_narrow", "E4C3", "E5C2")])
+                                        ("tensor_narrow", "E4C3", "E5C2"),
+                                        ("tensor_narrow", "E4C3_R3_4", "E4C3_R3_4")])
 def test_gemm_stays_inside(torch, algo, fa, fb):
     import paper_2608_10010_gb300 as cfp
 

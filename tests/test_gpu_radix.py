@@ -243,3 +243,81 @@ def test_tensor_gemm_r89_llama_g512_sampled(torch):
     err = normalised_error(c.cpu().numpy()[np.ix_(ii, jj)], ref["C"], oracle.row_norms(ah, sah, fmt, G),
                            oracle.row_norms(bh, sbh, fmt, G))
     assert err <= 1e-5, err
+
+
+@pytest.mark.parametrize("block", [32, 512])
+@pytest.mark.parametrize("algo", ["tensor_narrow", "auto"])
+def test_narrow_gemm_r34_within_tolerance(torch, block, algo):
+    """Tensor-core GEMM for r = 2^{3/4} (32 planes per operand, pair planes j
+    and j + 16 in 2:4-sparse MMAs, the 32 phases along N): within 1e-5 of the
+    oracle's fp64 combine, normalised by the row norms; M ragged against the
+    8-token tiles, N against the 128-row tiles; AUTO takes the same kernel."""
+    import paper_2608_10010_gb300 as cfp
+    from tests.gpu_util import normalised_error
+
+    fmt = "E4C3_R3_4"
+    M, N, K = 37, 320, 1024
+    a, sa, _ = oracle.quantize(inputs.outlier_channels((M, K), 21), fmt, block, 0)
+    b, sb, _ = oracle.quantize(inputs.normal((N, K), 22, 0.02), fmt, block, 0)
+    st = new_status(torch)
+    c = cfp.gemm(to_dev(torch, a), to_dev(torch, sa), to_dev(torch, b), to_dev(torch, sb), fmt, fmt, block, algo,
+                 status=st)
+    torch.cuda.synchronize()
+    ref = oracle.gemm(a, sa, b, sb, fmt, fmt, block, phases=False)
+    assert status_bits(st) == 0
+    err = normalised_error(c.cpu().numpy(), ref["C"], oracle.row_norms(a, sa, fmt, block),
+                           oracle.row_norms(b, sb, fmt, block))
+    assert err <= 1e-5, err
+
+
+def test_narrow_gemm_r34_every_code(torch):
+    """Every code byte (both signs, the zero code, all 32 curve planes and
+    both halves of each pair) on both operands with block scales spread over
+    24 binades: within 1e-5 of the oracle."""
+    import paper_2608_10010_gb300 as cfp
+    from tests.gpu_util import normalised_error
+
+    fmt, G = "E4C3_R3_4", 32
+    rng = np.random.default_rng(23)
+    M, N, K = 24, 256, 512
+    a = rng.integers(0, 256, size=(M, K)).astype(np.uint8)
+    b = rng.integers(0, 256, size=(N, K)).astype(np.uint8)
+    a[0, :256] = np.arange(256, dtype=np.uint8)
+    b[:, :256] = np.arange(256, dtype=np.uint8)[None, :]
+    sa = rng.integers(-12, 12, size=(M, K // G)).astype(np.int8)
+    sb = rng.integers(-12, 12, size=(N, K // G)).astype(np.int8)
+    st = new_status(torch)
+    c = cfp.gemm(to_dev(torch, a), to_dev(torch, sa), to_dev(torch, b), to_dev(torch, sb), fmt, fmt, G,
+                 "tensor_narrow", status=st)
+    torch.cuda.synchronize()
+    ref = oracle.gemm(a, sa, b, sb, fmt, fmt, G, phases=False)
+    assert status_bits(st) == 0
+    err = normalised_error(c.cpu().numpy(), ref["C"], oracle.row_norms(a, sa, fmt, G),
+                           oracle.row_norms(b, sb, fmt, G))
+    assert err <= 1e-5, err
+
+
+def test_narrow_gemm_r34_llama_g512_sampled(torch):
+    """r = 2^{3/4} at full size (Llama-7B-like linear, G512) on the tensor
+    cores, with the split tail of the last wave: 64 x 64 sampled outputs
+    against the oracle."""
+    import paper_2608_10010_gb300 as cfp
+    from tests.gpu_util import normalised_error
+
+    fmt, G = "E4C3_R3_4", 512
+    X, W = inputs.llama7b_linear(2048, 4096, 4096)
+    qx, sx = cfp.quantize(to_dev(torch, X), fmt, G, 0)
+    qw, sw = cfp.quantize(to_dev(torch, W), fmt, G, 0)
+    st = new_status(torch)
+    c = cfp.gemm(qx, sx, qw, sw, fmt, fmt, G, "tensor_narrow", status=st)
+    torch.cuda.synchronize()
+    assert status_bits(st) == 0
+    rng = np.random.default_rng(29)
+    ii = np.sort(rng.choice(2048, 64, replace=False))
+    jj = np.sort(rng.choice(4096, 64, replace=False))
+    ah, sah = qx.cpu().numpy()[ii], sx.cpu().numpy()[ii]
+    bh, sbh = qw.cpu().numpy()[jj], sw.cpu().numpy()[jj]
+    ref = oracle.gemm(ah, sah, bh, sbh, fmt, fmt, G, phases=False)
+    err = normalised_error(c.cpu().numpy()[np.ix_(ii, jj)], ref["C"], oracle.row_norms(ah, sah, fmt, G),
+                           oracle.row_norms(bh, sbh, fmt, G))
+    assert err <= 1e-5, err

@@ -345,3 +345,42 @@ def test_pair_metadata_selects_the_partner_plane(mbit):
             b0, b1 = (codes[2 * c] >> mbit) & 1, (codes[2 * c + 1] >> mbit) & 1
             want |= (b0 | (2 + b1) << 2) << (4 * c)
         assert pair_meta_emulated(w, mbit) == want, w
+
+
+# ---- the plane bytes of r = 2^{3/4} (gemm_tcn_r34.cu) -----------------------
+
+def r34_word_emulated(w):
+    """gemm_tcn_r34.cu r34_word: the E5M2 byte of +-2^q, the nonzero mask and
+    the curve plane j of four codes, from 3m in 16-bit lanes."""
+    m4 = w & 0x7F7F7F7F
+    nz = prmt_sign((m4 + 0x7F7F7F7F) & M32, 0xBA98)
+    lo = ((m4 & 0x00FF00FF) * 3) & M32
+    hi = (((m4 >> 8) & 0x00FF00FF) * 3) & M32
+    j4 = (lo & 0x001F001F) | ((hi & 0x001F001F) << 8)
+    q4 = ((lo >> 5) & 0x000F000F) | (((hi >> 5) & 0x000F000F) << 8)
+    v = ((w & 0x80808080) | (((q4 + 0x09090909) << 2) & M32)) & nz
+    return v, nz, j4
+
+
+def test_r34_plane_bytes_of_every_code_in_every_lane():
+    """Every code byte in every lane: the element 2^{3n/32} (n = m - 64) is
+    2^q 2^{j/32} with the plane byte +-2^q and the curve plane j (3n = 32 q +
+    j, 0 <= j < 32); the zero code gives 0; no lane disturbs another."""
+    rng = np.random.default_rng(37)
+    for c in range(256):
+        m = c & 0x7F
+        n = m - 64
+        q, j = (3 * n) // 32, (3 * n) % 32
+        s = -1.0 if c & 0x80 else 1.0
+        for lane in range(4):
+            nb = rng.integers(0, 256, size=4)
+            nb[lane] = c
+            w = int(nb[0]) | int(nb[1]) << 8 | int(nb[2]) << 16 | int(nb[3]) << 24
+            v, nz, j4 = r34_word_emulated(w)
+            vb = (v >> (8 * lane)) & 0xFF
+            if m == 0:
+                assert vb == 0 and (nz >> (8 * lane)) & 0xFF == 0, c
+                continue
+            assert e5m2_value(vb) == s * 2.0 ** q, (c, lane)
+            assert (j4 >> (8 * lane)) & 0xFF == j, (c, lane)
+            assert np.isclose(s * 2.0 ** q * 2.0 ** (j / 32), s * 2.0 ** (3 * n / 32), rtol=1e-15)
