@@ -744,7 +744,8 @@ def run_only(args):
     --only quantize: 2^28 BF16 elements, E4C3, block 32; skinny, narrow,
     reuse, r89: the decode GEMM, the few-row tensor-core GEMM, the
     reused-operand dgrad and the r = 2^{8/9} GEMM; static: the static
-    quantizer with row groups and the MSE search, E3C3, W[4096 x 4096])."""
+    quantizer with row groups and the MSE search, E3C3, W[4096 x 4096];
+    dgrad: the training triplet's dgrad on the narrow kernel, E5C2 x E4C3)."""
     import torch
 
     import paper_2608_10010_gb300 as cfp
@@ -783,6 +784,15 @@ def run_only(args):
             c = cfp.gemm(a, sa, b, sb, "E3C3", "E3C3", G, "tensor_narrow")
         torch.cuda.synchronize()
         print(json.dumps({"only": "narrow", "M": args.narrow_m, "launches": args.steps, "c00": float(c[0, 0])}))
+    elif args.only == "dgrad":  # dY[4096 x 11008] E5C2 . W^T (W [11008 x 4096] E4C3, block axis 0 of W^T)
+        X, Wt, dY = inputs.training_triplet_cuda()
+        qg, sg = cfp.quantize(dY, "E5C2", G, 0)
+        qw, sw = cfp.quantize(Wt, "E4C3", G, 0)
+        del X, Wt, dY
+        for _ in range(args.steps):
+            c = cfp.gemm(qg, sg, qw, sw, "E5C2", "E4C3", G, "tensor_narrow")
+        torch.cuda.synchronize()
+        print(json.dumps({"only": "dgrad", "launches": args.steps, "c00": float(c[0, 0])}))
     elif args.only == "static":  # static scales: row groups, MSE search, E3C3 W[4096 x 4096] ~ N(0, 0.02^2)
         Wt = torch.randn((4096, 4096), device=dev, generator=torch.Generator(device=dev).manual_seed(4)) * 0.02
         for _ in range(args.steps):
@@ -815,7 +825,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--only", choices=["gemm", "tile", "quantize", "skinny", "narrow", "reuse", "r89", "static"],
+    ap.add_argument("--only", choices=["gemm", "tile", "quantize", "skinny", "narrow", "reuse", "r89", "static", "dgrad"],
                     default=None)
     ap.add_argument("--narrow-m", type=int, default=16, help="activation rows of --only narrow")
     ap.add_argument("--no-sweep", action="store_true", help="skip the other workloads (quantize sweep, GEMM shapes)")

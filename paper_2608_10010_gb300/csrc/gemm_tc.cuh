@@ -328,21 +328,7 @@ __global__ void __launch_bounds__(TcCfg<FA, FB>::THREADS, 1)
   if (PES) {
     if (rowok) ref = __ldg(is_a ? pes.refA + r : pes.refB + r);
   } else if (rowok) {
-    const int8_t* s = (is_a ? sA : sB) + (int64_t)r * nb;
-    if ((nb & 15) == 0 && (reinterpret_cast<uintptr_t>(s) & 15) == 0) {
-      // 16 scales per load, all loads in flight at once, byte-wise signed max
-      uint32_t m4 = 0x80808080u;
-#pragma unroll 8
-      for (int b = 0; b < nb; b += 16) {
-        const uint4 q = __ldg(reinterpret_cast<const uint4*>(s + b));
-        m4 = __vmaxs4(m4, __vmaxs4(__vmaxs4(q.x, q.y), __vmaxs4(q.z, q.w)));
-      }
-      ref = max(max((int)(int8_t)(m4 & 0xFF), (int)(int8_t)((m4 >> 8) & 0xFF)),
-                max((int)(int8_t)((m4 >> 16) & 0xFF), (int)(int8_t)(m4 >> 24)));
-    } else {
-#pragma unroll 8
-      for (int b = 0; b < nb; ++b) ref = max(ref, (int)__ldg(s + b));
-    }
+    ref = row_ref((is_a ? sA : sB) + (int64_t)r * nb, nb);
   }
   if (!is_a && is_prod && part == 0) sh.refB[rloc] = ref;
   tc::fence_before_sync();

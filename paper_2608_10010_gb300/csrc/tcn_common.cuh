@@ -1,7 +1,7 @@
 // Helpers shared by the phases-along-N tensor-core kernels (gemm_tcn.cu:
-// binary formats; gemm_tcn_r34.cu: r = 2^{3/4}): row references of the scale
-// factors, the 2:4 metadata of pair planes, whole-warp bounded waits, TMEM
-// stores and the K-split plan of the last wave.
+// binary formats; gemm_tcn_r34.cu: r = 2^{3/4}): the 2:4 metadata of pair
+// planes, whole-warp bounded waits, TMEM stores and the K-split plan of the
+// last wave.
 #pragma once
 #include <mutex>
 #include <unordered_map>
@@ -11,25 +11,6 @@
 namespace cfp {
 
 namespace {
-
-// Largest block scale of a row (the row reference of the scale factors).
-__device__ __forceinline__ int row_ref(const int8_t* s, int nb) {
-  int ref = -128;
-  if ((nb & 15) == 0 && (reinterpret_cast<uintptr_t>(s) & 15) == 0) {
-    uint32_t m4 = 0x80808080u;
-#pragma unroll 8
-    for (int b = 0; b < nb; b += 16) {
-      const uint4 q = __ldg(reinterpret_cast<const uint4*>(s + b));
-      m4 = __vmaxs4(m4, __vmaxs4(__vmaxs4(q.x, q.y), __vmaxs4(q.z, q.w)));
-    }
-    ref = max(max((int)(int8_t)(m4 & 0xFF), (int)(int8_t)((m4 >> 8) & 0xFF)),
-              max((int)(int8_t)((m4 >> 16) & 0xFF), (int)(int8_t)(m4 >> 24)));
-  } else {
-#pragma unroll 8
-    for (int b = 0; b < nb; ++b) ref = max(ref, (int)__ldg(s + b));
-  }
-  return ref;
-}
 
 // Interleave two words (elements 4q..4q+3 each) into X0 Y0 X1 Y1 | X2 Y2 X3 Y3.
 __device__ __forceinline__ uint2 interleave2(uint32_t x, uint32_t y) {
