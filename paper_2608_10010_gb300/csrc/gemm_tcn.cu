@@ -33,12 +33,15 @@
 // lattice distance of the partner plane) and the operand of pair j is the
 // window from R block L - j WW: K_W/2 sparse MMAs of logical K 64 per step.
 //
-// Orientation.  X takes the carry copies, so its planes need one binade more
-// than W's; an E5C2 operand goes on the weight side (its 32 binades fill
-// E5M2): E5C2 x E4C3 runs transposed (X = the E4C3 operand, C stored as
-// C[w][m]).  E5C2 x E5C2 stores the X planes one binade low (its lowest
-// binade's plain copy, 2^-17, has no E5M2 value and is dropped: an element
-// at least 2^30 below the top binade of its block).
+// Orientation.  The tokens are A's rows and the weights B's for every pair.
+// X takes the carry copies, so its planes need one binade more than W's: E5C2
+// tokens store their planes one binade low (the lowest binade's plain copy,
+// 2^-17, has no E5M2 value and is dropped: an element at least 2^30 below the
+// top binade of its block).  E5C2 tokens against E4C3 weights put their four
+// planes on every other position of the 8-phase lattice (WX = 2): half of the
+// R blocks stay empty, and the W side carries the E4C3 operand's four pair
+// planes, so the producers' work per MMA is lower than with the operands
+// swapped (two pair planes of E5C2 weights against 8-plane tokens).
 //
 // Roles (15 warps for 8-phase pairs, 17 for E5C2 x E5C2):
 //   warps 0-7   W producers: two groups of 4 warps taking alternate steps,
@@ -67,7 +70,7 @@ template <int FX, int FW>
 struct TcnCfg {
   using P = Pair<FX, FW>;
   static constexpr int KW = Fmt<FW>::K, L = P::L, WX = P::WA, WW = P::WB;
-  static_assert(WX == 1, "X planes sit on every lattice position");
+  static_assert(WX == 1 || (WX == 2 && Fmt<FX>::C == 2), "X planes on every (or every other) lattice position");
   static constexpr int BM = 128;          // weight rows per CTA (TMEM lanes)
   static constexpr int KS = 32;           // codes per pipeline step (one scale factor)
   static constexpr int MTMAX = 256 / L;   // tokens per CTA: L Mt <= 256 (MMA N)
@@ -76,7 +79,7 @@ struct TcnCfg {
   static constexpr int NJ = HB;           // sparse MMAs per step
   static constexpr int PO = HB * WW;      // lattice distance of the partner plane
   static constexpr int RB0 = L - (NJ - 1) * WW, NRB = 2 * L - RB0;
-  static_assert(2 * PO == L && Fmt<FX>::K == L && RB0 > PO, "partner planes half the lattice apart");
+  static_assert(2 * PO == L && RB0 > PO && PO % WX == 0, "partner planes half the lattice apart");
   static constexpr int ROWB = 64;         // bytes of one operand row (logical K 64)
   static constexpr int PBX = FX == CURVEFP_E5C2 ? 1 : 0;  // X planes one binade low
   // TMEM columns: accumulators, W units, metadata (8 per unit, 2 used), A
@@ -110,10 +113,10 @@ struct TcnCfg {
 }  // namespace
 
 // X: [Mx x K] token codes, W: [Nw x K] weight codes (K contiguous), scales
-// [rows x K/G].  C: [Mx x Nw] (TR = false) or [Nw x Mx] (TR = true), row-major.
+// [rows x K/G].  C: [Mx x Nw], row-major.
 // FULL: every tile has MTMAX tokens (Mt == MTMAX), so the stage offsets of
 // the X producers are constants.
-template <int FX, int FW, bool TR, bool FULL>
+template <int FX, int FW, bool FULL>
 __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
     gemm_tcn_kernel(const uint8_t* __restrict__ X, const int8_t* __restrict__ sX, const uint8_t* __restrict__ W,
                     const int8_t* __restrict__ sW, int M, int N, int K, int G, int gshift, int Mt,
@@ -336,32 +339,15 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
 #pragma unroll
         for (int j = 0; j < 8; ++j) y[j] = scalbnf(t[j], ref + sh.refB[lt + j] - 2 * MX_OFF);
         const int m0 = x0 + lt;
-        if constexpr (TR) {
-          // C[w][m]: the thread's 8 consecutive tokens
-          float* dst = C + (int64_t)wrow * M + m0;
-          if (split) {
 #pragma unroll
-            for (int j = 0; j < 8; ++j)
-              if (m0 + j < M) atomicAdd(dst + j, y[j]);
-          } else if (m0 + 8 <= M && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
-            reinterpret_cast<float4*>(dst)[0] = make_float4(y[0], y[1], y[2], y[3]);
-            reinterpret_cast<float4*>(dst)[1] = make_float4(y[4], y[5], y[6], y[7]);
-          } else {
-#pragma unroll
-            for (int j = 0; j < 8; ++j)
-              if (m0 + j < M) dst[j] = y[j];
-          }
-        } else {
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const int m = m0 + j;
-            if (m < M) {
-              float* dst = C + (int64_t)m * N + wrow;
-              if (split)
-                atomicAdd(dst, y[j]);
-              else
-                *dst = y[j];
-            }
+        for (int j = 0; j < 8; ++j) {
+          const int m = m0 + j;
+          if (m < M) {
+            float* dst = C + (int64_t)m * N + wrow;
+            if (split)
+              atomicAdd(dst, y[j]);
+            else
+              *dst = y[j];
           }
         }
       }
@@ -427,6 +413,7 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
         const uint32_t sf = mx_sf(raw[e] - xref[e], Cfg::PBX, keep);
         constexpr int C = Fmt<FX>::C;
         if constexpr (C == 3) {
+          static_assert(Fmt<FX>::K == L, "three-bit tokens sit on every lattice position");
           // Three curve-index bits.  R block b holds Q_b[k] in byte 2k and Q_{b-PO}[k] in byte 2k + 1 (Q
           // block u < L: the carry copy of plane u, u >= L: plane u - L).  With
           // PO = L/2 the two planes share their two low curve-index bits (class
@@ -471,7 +458,11 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
           }
         } else {
           // Two curve-index bits: the tokens' planes of each word and their
-          // carry copies, then per R block Q_b and Q_{b-PO} interleaved
+          // carry copies, then per R block Q_b and Q_{b-PO} interleaved.  With
+          // WX = 2 (E5C2 tokens against an 8-phase lattice) plane k sits on
+          // lattice position 2k, Q blocks of odd positions are empty, and an
+          // R block whose halves are both empty is never written (the stages
+          // start at zero).
           uint32_t pv[2][8], pc[2][8];
 #pragma unroll
           for (int q = 0; q < 2; ++q) {
@@ -482,12 +473,19 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
             planes_of<C>(v, mk, pv[q]);
             planes_of<C>(vc, mk, pc[q]);
           }
+          constexpr int WXc = Cfg::WX;
+          // Q block u: the carry copy (u < L) or the plane (u >= L) of the
+          // token plane on lattice position u mod L, zero where none sits
+          auto qb = [&](int q, int u) -> uint32_t {
+            const int pos = u < L ? u : u - L;
+            if (pos % WXc) return 0u;
+            return u < L ? pc[q][pos / WXc] : pv[q][pos / WXc];
+          };
 #pragma unroll
           for (int b = Cfg::RB0; b < 2 * L; ++b) {
-            const uint2 lo = interleave2(b < L ? pc[0][b] : pv[0][b - L],
-                                         b - Cfg::PO < L ? pc[0][b - Cfg::PO] : pv[0][b - Cfg::PO - L]);
-            const uint2 hi = interleave2(b < L ? pc[1][b] : pv[1][b - L],
-                                         b - Cfg::PO < L ? pc[1][b - Cfg::PO] : pv[1][b - Cfg::PO - L]);
+            if ((b % WXc) != 0 && ((b - Cfg::PO) % WXc) != 0) continue;
+            const uint2 lo = interleave2(qb(0, b), qb(0, b - Cfg::PO));
+            const uint2 hi = interleave2(qb(1, b), qb(1, b - Cfg::PO));
             *reinterpret_cast<uint4*>(stg + xbase[e] + (b - Cfg::RB0) * bstride) = make_uint4(lo.x, lo.y, hi.x, hi.y);
           }
         }
@@ -576,9 +574,8 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
 
 namespace {
 
-// x: [Mx x K] token codes, w: [Nw x K] weight codes; c: [Mx x Nw], or
-// [Nw x Mx] with TR.
-template <int FX, int FW, bool TR>
+// x: [Mx x K] token codes, w: [Nw x K] weight codes; c: [Mx x Nw].
+template <int FX, int FW>
 cudaError_t launch_tcn_t(int G, const uint8_t* x, const int8_t* sx, const uint8_t* w, const int8_t* sw, int64_t Mx,
                          int64_t Nw, int64_t K, float* c, uint32_t* st, cudaStream_t s, int sms) {
   using Cfg = TcnCfg<FX, FW>;
@@ -588,20 +585,16 @@ cudaError_t launch_tcn_t(int G, const uint8_t* x, const int8_t* sx, const uint8_
   int64_t ng = (Mx + Cfg::MTMAX - 1) / Cfg::MTMAX;
   const int Mt = (int)(((Mx + ng - 1) / ng + 7) / 8 * 8);
   ng = (Mx + Mt - 1) / Mt;
-  auto kern = Mt == Cfg::MTMAX ? gemm_tcn_kernel<FX, FW, TR, true> : gemm_tcn_kernel<FX, FW, TR, false>;
+  auto kern = Mt == Cfg::MTMAX ? gemm_tcn_kernel<FX, FW, true> : gemm_tcn_kernel<FX, FW, false>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg::SMEM);
   if (e != cudaSuccess) return e;
   const int64_t ntw = (Nw + Cfg::BM - 1) / Cfg::BM, tiles = ntw * ng;
   const TailPlan plan = tcn_plan(tiles, sms, (int)(K / Cfg::KS));
   if (plan.nsplit > 0) {
-    // C of the split tiles starts at zero: for C[m][w], the token rows from
-    // the first split tile's group on; for C[w][m], all of C
-    if (TR) {
-      e = cudaMemsetAsync(c, 0, (size_t)(Mx * Nw) * sizeof(float), s);
-    } else {
-      const int64_t row0 = (plan.ntiles_full / ntw) * Mt;
-      e = cudaMemsetAsync(c + row0 * Nw, 0, (size_t)((Mx - row0) * Nw) * sizeof(float), s);
-    }
+    // C of the split tiles starts at zero: the token rows from the first
+    // split tile's group on
+    const int64_t row0 = (plan.ntiles_full / ntw) * Mt;
+    e = cudaMemsetAsync(c + row0 * Nw, 0, (size_t)((Mx - row0) * Nw) * sizeof(float), s);
     if (e != cudaSuccess) return e;
   }
   const unsigned grid = (unsigned)(plan.ntiles_full + 2 * plan.nsplit);
@@ -619,23 +612,21 @@ bool gemm_narrow_supported(int fa, int fb) {
          (fa == CURVEFP_E5C2 && fb == CURVEFP_E5C2) || (fa == CURVEFP_E4C3_R3_4 && fb == CURVEFP_E4C3_R3_4);
 }
 
-// C = A_hat B_hat^T, A [M x K] (format fa), B [N x K] (format fb).  The
-// tokens are A's rows and the weights B's, except for E5C2 x E4C3, which runs
-// transposed (tokens = B's rows, weights = A's rows, C written as C[m][n]
-// with m the weight index) so that the E5C2 operand is on the weight side.
+// C = A_hat B_hat^T, A [M x K] (format fa), B [N x K] (format fb): the
+// tokens are A's rows and the weights B's.
 cudaError_t launch_gemm_tensor_narrow(int fa, int fb, int G, const uint8_t* a, const int8_t* sa, const uint8_t* b,
                                       const int8_t* sb, int64_t M, int64_t N, int64_t K, float* c, uint32_t* status,
                                       cudaStream_t s, int sms) {
   if (fa == CURVEFP_E3C3 && fb == CURVEFP_E3C3)
-    return launch_tcn_t<CURVEFP_E3C3, CURVEFP_E3C3, false>(G, a, sa, b, sb, M, N, K, c, status, s, sms);
+    return launch_tcn_t<CURVEFP_E3C3, CURVEFP_E3C3>(G, a, sa, b, sb, M, N, K, c, status, s, sms);
   if (fa == CURVEFP_E4C3 && fb == CURVEFP_E4C3)
-    return launch_tcn_t<CURVEFP_E4C3, CURVEFP_E4C3, false>(G, a, sa, b, sb, M, N, K, c, status, s, sms);
+    return launch_tcn_t<CURVEFP_E4C3, CURVEFP_E4C3>(G, a, sa, b, sb, M, N, K, c, status, s, sms);
   if (fa == CURVEFP_E4C3 && fb == CURVEFP_E5C2)
-    return launch_tcn_t<CURVEFP_E4C3, CURVEFP_E5C2, false>(G, a, sa, b, sb, M, N, K, c, status, s, sms);
+    return launch_tcn_t<CURVEFP_E4C3, CURVEFP_E5C2>(G, a, sa, b, sb, M, N, K, c, status, s, sms);
   if (fa == CURVEFP_E5C2 && fb == CURVEFP_E4C3)
-    return launch_tcn_t<CURVEFP_E4C3, CURVEFP_E5C2, true>(G, b, sb, a, sa, N, M, K, c, status, s, sms);
+    return launch_tcn_t<CURVEFP_E5C2, CURVEFP_E4C3>(G, a, sa, b, sb, M, N, K, c, status, s, sms);
   if (fa == CURVEFP_E5C2 && fb == CURVEFP_E5C2)
-    return launch_tcn_t<CURVEFP_E5C2, CURVEFP_E5C2, false>(G, a, sa, b, sb, M, N, K, c, status, s, sms);
+    return launch_tcn_t<CURVEFP_E5C2, CURVEFP_E5C2>(G, a, sa, b, sb, M, N, K, c, status, s, sms);
   if (fa == CURVEFP_E4C3_R3_4 && fb == CURVEFP_E4C3_R3_4)  // 32 phases: gemm_tcn_r34.cu
     return launch_gemm_tensor_narrow_r34(G, a, sa, b, sb, M, N, K, c, status, s, sms);
   return cudaErrorInvalidValue;
