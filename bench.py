@@ -183,7 +183,9 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
         r = {"case": name, "algo": algo, "M": Mx, "N": Nx, "K": Kx, "formats": f"{fa}x{fb}", "ms": round(ms, 4),
              "tops": round(tops, 3)}
         if algo in ("tensor", "tensor_narrow"):
-            # the narrow kernel uses 2:4-sparse pair planes: half the MMA work
+            # planes: dense-equivalent MACs the MMAs issue per useful MAC (for
+            # the narrow kernel K_W L, the weights' planes times the lattice's
+            # phase columns; its 2:4-sparse pair planes halve the MMA work)
             issued = planes // 2 if algo == "tensor_narrow" else planes
             r["tensor_work_frac"] = round(tops * issued / fp8_peak, 4)
         if hbm_bound:
@@ -261,9 +263,9 @@ def other_workloads(torch, cfp, inputs, stream, flush_l2, hbm, fp8_peak):
     gemm_case("fwd X.W", q(X, "E4C3", 0), "E4C3", q(Wt, "E4C3", 1), "E4C3", 64)
     gemm_case("fwd X.W narrow", q(X, "E4C3", 0), "E4C3", q(Wt, "E4C3", 1), "E4C3", 64, algo="tensor_narrow")
     gemm_case("dgrad dY.W^T", q(dY, "E5C2", 0), "E5C2", q(Wt, "E4C3", 0), "E4C3", 32)
-    gemm_case("dgrad dY.W^T narrow", q(dY, "E5C2", 0), "E5C2", q(Wt, "E4C3", 0), "E4C3", 32, algo="tensor_narrow")
+    gemm_case("dgrad dY.W^T narrow", q(dY, "E5C2", 0), "E5C2", q(Wt, "E4C3", 0), "E4C3", 64, algo="tensor_narrow")
     gemm_case("wgrad dY^T.X", q(dY, "E5C2", 1), "E5C2", q(X, "E4C3", 1), "E4C3", 32)
-    gemm_case("wgrad dY^T.X narrow", q(dY, "E5C2", 1), "E5C2", q(X, "E4C3", 1), "E4C3", 32, algo="tensor_narrow")
+    gemm_case("wgrad dY^T.X narrow", q(dY, "E5C2", 1), "E5C2", q(X, "E4C3", 1), "E4C3", 64, algo="tensor_narrow")
     # the same triplet on operands quantized once and reused (the backward
     # GEMMs read W, X and dY in the forward pass's block orientation; the
     # timed region includes the operand preparation kernels)
