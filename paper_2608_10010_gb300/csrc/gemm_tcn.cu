@@ -529,29 +529,40 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
     const uint64_t bdesc0 = tc::smem_desc(tc::smem_u32(xstage), 128, 512);
     const uint32_t idesc = idesc_mx_e5m2(NP, true);
     const int gbytes = Mt * Cfg::ROWB;  // bytes of one column block
-    bool ok = true;
-    for (int g = 0; g < total && ok; ++g) {
-      const int st = g % NSB;
-      ok = wait_all(&sh.full[st], (g / NSB) & 1);
-      if ((g & 7) == 0) ok = ok && !read_abort(&sh.abort_flag);
-      if (!ok) break;
-      tc::fence_after_sync();
-      // the step's B factors: columns 0..127 and, for N > 128, 128..255
-      const uint8_t* sfs = sfstage + (size_t)st * Cfg::SFSTAGE;
-      tmem_cp_sf_if(leader, tmem + Cfg::SFB0 + st * 8, sfs);
-      if (NP > 128) tmem_cp_sf_if(leader, tmem + Cfg::SFB0 + st * 8 + 4, sfs + 512);
+    // per pair plane: its accumulator copy and the descriptor of its window
+    // of R blocks (from L - kw WW) in stage 0; the loop below is unrolled
+    // over the stages, so every other offset is a constant of its body
+    uint32_t d_kw[Cfg::NJ];
+    uint64_t b_kw[Cfg::NJ];
 #pragma unroll
-      for (int kw = 0; kw < Cfg::NJ; ++kw) {
-        // pair plane kw against the window of R blocks from L - kw WW
-        const uint32_t a_t = tmem + Cfg::ACOL0 + st * Cfg::AU_COLS + kw * 8;
-        const uint32_t boff = (uint32_t)(st * Cfg::BSTAGE + (L - kw * Cfg::WW - Cfg::RB0) * gbytes);
-        const uint32_t d_t = tmem + (uint32_t)((kw & (nacc - 1)) * NP);
-        const uint32_t acc = (g == 0 && kw < nacc) ? 0u : 1u;
-        mma_sp_mx_if(leader, d_t, a_t, bdesc0 + (uint64_t)(boff >> 4), tmem + Cfg::MCOL0 + st * 8, idesc,
-                     tmem + Cfg::SFA0 + st * 4, tmem + Cfg::SFB0 + st * 8, acc);
+    for (int kw = 0; kw < Cfg::NJ; ++kw) {
+      d_kw[kw] = tmem + (uint32_t)((kw & (nacc - 1)) * NP);
+      b_kw[kw] = bdesc0 + (uint64_t)((uint32_t)((L - kw * Cfg::WW - Cfg::RB0) * gbytes) >> 4);
+    }
+    bool ok = true;
+    for (int g0 = 0, par = 0; g0 < total && ok; g0 += NSB, par ^= 1) {
+#pragma unroll
+      for (int st = 0; st < NSB; ++st) {
+        const int g = g0 + st;
+        if (g >= total) break;
+        ok = wait_all(&sh.full[st], (uint32_t)par);
+        if ((g & 7) == 0) ok = ok && !read_abort(&sh.abort_flag);
+        if (!ok) break;
+        tc::fence_after_sync();
+        // the step's B factors: columns 0..127 and, for N > 128, 128..255
+        const uint8_t* sfs = sfstage + (size_t)st * Cfg::SFSTAGE;
+        tmem_cp_sf_if(leader, tmem + Cfg::SFB0 + st * 8, sfs);
+        if (NP > 128) tmem_cp_sf_if(leader, tmem + Cfg::SFB0 + st * 8 + 4, sfs + 512);
+#pragma unroll
+        for (int kw = 0; kw < Cfg::NJ; ++kw) {
+          const uint32_t acc = (g == 0 && kw < nacc) ? 0u : 1u;
+          mma_sp_mx_if(leader, d_kw[kw], tmem + Cfg::ACOL0 + st * Cfg::AU_COLS + kw * 8,
+                       b_kw[kw] + (uint64_t)((st * Cfg::BSTAGE) >> 4), tmem + Cfg::MCOL0 + st * 8, idesc,
+                       tmem + Cfg::SFA0 + st * 4, tmem + Cfg::SFB0 + st * 8, acc);
+        }
+        tc::mma_commit_if(leader, &sh.empty[st]);
+        if (g == total - 1) tc::mma_commit_if(leader, &sh.acc_full);
       }
-      tc::mma_commit_if(leader, &sh.empty[st]);
-      if (g == total - 1) tc::mma_commit_if(leader, &sh.acc_full);
     }
     if (!ok && lane == 0) {
       raise_flag(status, CURVEFP_DEV_TIMEOUT);

@@ -55,13 +55,18 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16
       : "memory");
 }
 
-// Split plan of the narrow kernel: the tile kernel's tail search extended to
-// grids with fewer tiles than SMs (then every tile is split), with finer
+// Split plan of the narrow kernel: the tile kernel's tail search with finer
 // split points (a narrow tile is short, so its pieces' fixed costs weigh
-// more and the best point moves).
+// more and the best point moves).  With fewer tiles than SMs every tile is
+// split in halves when all pieces fit in one wave, and none is split
+// otherwise: a CTA's fixed cost (about 6 us of set-up and first decode, a
+// sixth of a 128-step tile at few tokens) makes a second wave of short
+// pieces slower than the whole tiles (measured at 112 tiles on 152 SMs:
+// 44.6 us unsplit, 49-53 us with the pieces at 1/2 or 3/4).
 inline TailPlan tcn_plan_search(int64_t tiles, int sms, int nsub) {
   TailPlan best{(int)tiles, 0, 0};
   if (sms <= 0 || nsub < 2 || tiles % sms == 0) return best;
+  if (tiles < sms) return 2 * tiles <= sms ? TailPlan{0, (int)tiles, nsub / 2} : best;
   double best_m = tail_makespan(tiles, sms, 0, 0.5);
   const double xs[5] = {0.5, 0.6, 2.0 / 3.0, 0.75, 0.8};
   for (int64_t s = tiles % sms; s <= tiles && s <= tiles % sms + 2 * (int64_t)sms; s += sms)
