@@ -391,7 +391,7 @@ __global__ void __launch_bounds__(TcCfg<FA, FB>::THREADS, 1)
 #pragma unroll
             for (int q = 0; q < PP; ++q)
               if (pe * PP + q < L) t = fmaf(phase_const(L, pe * PP + q), __uint_as_float(acc[q][c]), t);
-            y[c] = scalbnf(t, ref + sh.refB[c0 + c] - 2 * MX_OFF);
+            y[c] = scale_pow2(t, ref + sh.refB[c0 + c] - 2 * MX_OFF);
           }
           float4* s4 = reinterpret_cast<float4*>(strow + c0);
           if (pe > 0) {

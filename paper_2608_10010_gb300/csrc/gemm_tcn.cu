@@ -314,30 +314,42 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
       float t[8];
 #pragma unroll
       for (int j = 0; j < 8; ++j) t[j] = 0.f;
+      if (nacc == 1) {
+        // one accumulator: all L phase sums in one round of loads
+        uint32_t acc[L][8];
 #pragma unroll
-      for (int h0 = 0; h0 < L; h0 += 4) {
-        // S_h = the sum of the accumulator copies (copy order fixed)
-        float sh4[4][8];
-#pragma unroll 1
-        for (int a = 0; a < nacc; ++a) {
-          uint32_t acc[4][8];
-#pragma unroll
-          for (int h = 0; h < 4; ++h) tc::tmem_ld8(lane_base + a * NP + (h0 + h) * Mt + lt, acc[h]);
-          tc::tmem_wait_ld();
-#pragma unroll
-          for (int h = 0; h < 4; ++h)
-#pragma unroll
-            for (int j = 0; j < 8; ++j) sh4[h][j] = a ? sh4[h][j] + __uint_as_float(acc[h][j]) : __uint_as_float(acc[h][j]);
-        }
+        for (int h = 0; h < L; ++h) tc::tmem_ld8(lane_base + h * Mt + lt, acc[h]);
+        tc::tmem_wait_ld();
 #pragma unroll
         for (int j = 0; j < 8; ++j)
 #pragma unroll
-          for (int h = 0; h < 4; ++h) t[j] = fmaf(phase_const(L, h0 + h), sh4[h][j], t[j]);
+          for (int h = 0; h < L; ++h) t[j] = fmaf(phase_const(L, h), __uint_as_float(acc[h][j]), t[j]);
+      } else {
+#pragma unroll
+        for (int h0 = 0; h0 < L; h0 += 4) {
+          // S_h = the sum of the accumulator copies (copy order fixed)
+          float sh4[4][8];
+#pragma unroll 1
+          for (int a = 0; a < nacc; ++a) {
+            uint32_t acc[4][8];
+#pragma unroll
+            for (int h = 0; h < 4; ++h) tc::tmem_ld8(lane_base + a * NP + (h0 + h) * Mt + lt, acc[h]);
+            tc::tmem_wait_ld();
+#pragma unroll
+            for (int h = 0; h < 4; ++h)
+#pragma unroll
+              for (int j = 0; j < 8; ++j) sh4[h][j] = a ? sh4[h][j] + __uint_as_float(acc[h][j]) : __uint_as_float(acc[h][j]);
+          }
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+#pragma unroll
+            for (int h = 0; h < 4; ++h) t[j] = fmaf(phase_const(L, h0 + h), sh4[h][j], t[j]);
+        }
       }
       if (rowok && ok) {
         float y[8];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) y[j] = scalbnf(t[j], ref + sh.refB[lt + j] - 2 * MX_OFF);
+        for (int j = 0; j < 8; ++j) y[j] = scale_pow2(t[j], ref + sh.refB[lt + j] - 2 * MX_OFF);
         const int m0 = x0 + lt;
 #pragma unroll
         for (int j = 0; j < 8; ++j) {

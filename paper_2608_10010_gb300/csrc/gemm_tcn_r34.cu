@@ -278,7 +278,7 @@ __global__ void __launch_bounds__(R34::THREADS, 1)
       for (int m = 0; m < 4; ++m) {
         const int tok = 4 * hf + m, row = x0 + tok;
         if (row < M) {
-          const float y = scalbnf(t[m], ref + sh.refB[tok] - 2 * MX_OFF);
+          const float y = scale_pow2(t[m], ref + sh.refB[tok] - 2 * MX_OFF);
           float* dst = C + (int64_t)row * N + wrow;
           if (split)
             atomicAdd(dst, y);

@@ -71,6 +71,13 @@ __device__ __forceinline__ void mx_word(uint32_t w, uint32_t& v, uint32_t& vc) {
   }
 }
 
+// t 2^e, the epilogue's output scaling: a multiply by the normal float 2^e
+// where e is in [-126, 127] (one correctly rounded product, the value
+// scalbnf returns), scalbnf itself outside that range.
+__device__ __forceinline__ float scale_pow2(float t, int e) {
+  return (e >= -126 && e <= 127) ? t * __int_as_float((e + 127) << 23) : scalbnf(t, e);
+}
+
 // Scale-factor byte of a block scale relative to its row reference, and
 // whether the block is kept (see the header).
 __device__ __forceinline__ uint32_t mx_sf(int d, int bias, bool& keep) {
