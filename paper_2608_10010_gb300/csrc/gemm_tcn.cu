@@ -172,18 +172,19 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
   }
   const bool is_w = tid < Cfg::NWT, is_x = !is_w && warp < Cfg::MMA_WARP;
   // W threads: weight row (TMEM lane) and group; X threads: group.  The row
-  // references: a weight row per W thread, a token per thread of the first X
-  // group.  The X stages and factor blocks start at zero (padding tokens and
-  // empty lattice positions are never written).
+  // references of the tile's weight rows and tokens (-128 for rows past the
+  // ends) are formed by all threads together from the two contiguous runs of
+  // scale rows.  The X stages and factor blocks start at zero (padding
+  // tokens and empty lattice positions are never written).
   const int wrow = w0 + (warp & 3) * 32 + lane, gw = warp >> 2;
   const int t_x = tid - Cfg::NWT, gx = t_x / (Cfg::XPG * 32);
-  int ref = -128;
-  if (is_w && wrow < N) ref = row_ref(sW + (int64_t)wrow * nb, nb);
-  if (is_x && t_x < Cfg::MTMAX) {
-    int rx = -128;
-    if (t_x < Mt && x0 + t_x < M) rx = row_ref(sX + (int64_t)(x0 + t_x) * nb, nb);
-    sh.refB[t_x] = rx;
+  if (tid < 128) {
+    sh.wref[tid] = -128;
+    sh.refB[tid] = -128;
   }
+  __syncthreads();
+  rows_ref_coop(sW + (int64_t)w0 * nb, min(Cfg::BM, N - w0), nb, sh.wref, tid, Cfg::THREADS);
+  rows_ref_coop(sX + (int64_t)x0 * nb, min(Mt, M - x0), nb, sh.refB, tid, Cfg::THREADS);
   for (int o = tid * 16; o < NSB * (Cfg::BSTAGE + Cfg::SFSTAGE); o += Cfg::THREADS * 16)
     *reinterpret_cast<uint4*>(smem + o) = make_uint4(0, 0, 0, 0);
   tc::fence_proxy_async_smem();
@@ -191,6 +192,7 @@ __global__ void __launch_bounds__(TcnCfg<FX, FW>::THREADS, 1)
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = sh.tmem_base;
+  const int ref = is_w ? sh.wref[(warp & 3) * 32 + lane] : -128;  // this W thread's weight row
 
   if (is_w) {
     // ---------------------------- W producers -----------------------------

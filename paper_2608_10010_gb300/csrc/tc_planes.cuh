@@ -22,6 +22,7 @@ struct TcShared {
   uint32_t tmem_base;
   int abort_flag;
   int refB[128];  // >= BN
+  int wref[128];  // the narrow kernel's weight-row references
 };
 
 __device__ __forceinline__ void raise_flag(uint32_t* status, uint32_t bit) {
@@ -47,6 +48,42 @@ __device__ __forceinline__ int row_ref(const int8_t* s, int nb) {
                      max((int)(int8_t)((m4 >> 16) & 0xFF), (int)(int8_t)(m4 >> 24))));
   for (int b = head + 16 * nv; b < nb; ++b) ref = max(ref, (int)__ldg(s + b));
   return ref;
+}
+
+// Largest of the four signed bytes of v.
+__device__ __forceinline__ int max_s8x4(uint32_t v) {
+  return max(max((int)(int8_t)(v & 0xFF), (int)(int8_t)((v >> 8) & 0xFF)),
+             max((int)(int8_t)((v >> 16) & 0xFF), (int)(int8_t)(v >> 24)));
+}
+
+// Row references of `rows` consecutive rows of nb scale bytes (one run of
+// rows x nb bytes from s), read by threads t = 0 .. nthr - 1 together in
+// chunks of 16, 8 or 4 bytes (the largest that divides nb and the run's
+// alignment, single bytes otherwise; a chunk never spans two rows) and
+// folded into ref[row] by shared-memory atomics; ref[] holds -128 on entry.
+// A warp's loads cover whole lines, where a thread reading its own row
+// touches one line per lane and load.
+__device__ __forceinline__ void rows_ref_coop(const int8_t* s, int rows, int nb, int* ref, int t, int nthr) {
+  const uintptr_t a = reinterpret_cast<uintptr_t>(s);
+  const int64_t bytes = (int64_t)rows * nb;
+  if ((a & 15) == 0 && (nb & 15) == 0) {
+    const uint4* p = reinterpret_cast<const uint4*>(s);
+    for (int64_t i = t; i < bytes / 16; i += nthr) {
+      const uint4 q = __ldg(p + i);
+      atomicMax(ref + (int)(i * 16 / nb), max_s8x4(__vmaxs4(__vmaxs4(q.x, q.y), __vmaxs4(q.z, q.w))));
+    }
+  } else if ((a & 7) == 0 && (nb & 7) == 0) {
+    const uint2* p = reinterpret_cast<const uint2*>(s);
+    for (int64_t i = t; i < bytes / 8; i += nthr) {
+      const uint2 q = __ldg(p + i);
+      atomicMax(ref + (int)(i * 8 / nb), max_s8x4(__vmaxs4(q.x, q.y)));
+    }
+  } else if ((a & 3) == 0 && (nb & 3) == 0) {
+    const uint32_t* p = reinterpret_cast<const uint32_t*>(s);
+    for (int64_t i = t; i < bytes / 4; i += nthr) atomicMax(ref + (int)(i * 4 / nb), max_s8x4(__ldg(p + i)));
+  } else {
+    for (int64_t i = t; i < bytes; i += nthr) atomicMax(ref + (int)(i / nb), (int)__ldg(s + i));
+  }
 }
 
 // ---------------------------------------------------------------------------
