@@ -325,15 +325,26 @@ __global__ void __launch_bounds__(TcCfg<FA, FB>::THREADS, 1)
   const int r = (is_a ? m0 : n0) + rloc;
   const bool rowok = is_prod && r < (is_a ? M : N);
   int ref = -128;
-  if (PES) {
+  if constexpr (PES) {
     if (rowok) ref = __ldg(is_a ? pes.refA + r : pes.refB + r);
-  } else if (rowok) {
-    ref = row_ref((is_a ? sA : sB) + (int64_t)r * nb, nb);
+    if (!is_a && is_prod && part == 0) sh.refB[rloc] = ref;
+  } else {
+    // the references of the tile's A and B rows, formed by all threads from
+    // the two contiguous runs of scale rows (-128 past the ends)
+    if (tid < 128) {
+      sh.wref[tid] = -128;
+      sh.refB[tid] = -128;
+    }
+    __syncthreads();
+    rows_ref_coop(sA + (int64_t)m0 * nb, min(Cfg::BM, M - m0), nb, sh.wref, tid, Cfg::THREADS);
+    rows_ref_coop(sB + (int64_t)n0 * nb, min(BN, N - n0), nb, sh.refB, tid, Cfg::THREADS);
   }
-  if (!is_a && is_prod && part == 0) sh.refB[rloc] = ref;
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
+  if constexpr (!PES) {
+    if (rowok) ref = is_a ? sh.wref[rloc] : sh.refB[rloc];
+  }
   const uint32_t tmem = sh.tmem_base;
 
   if (is_prod) {

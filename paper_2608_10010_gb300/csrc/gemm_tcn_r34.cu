@@ -63,6 +63,7 @@ struct R34Shared {
   uint32_t tmem_base;
   int abort_flag;
   int refB[8];
+  int wref[128];
 };
 
 // Plane bytes of four codes: v = the E5M2 byte of +-2^q (0 for the zero
@@ -146,13 +147,13 @@ __global__ void __launch_bounds__(R34::THREADS, 1)
   const bool is_w = tid < Cf::NWT, is_x = !is_w && warp < Cf::MMA_WARP;
   const int q4 = warp & 3, hf = (warp >> 2) & 1;  // W: row quadrant, half (pair planes 8 hf ..)
   const int wrow = w0 + q4 * 32 + lane;
-  int ref = -128;
-  if (is_w && wrow < N) ref = row_ref(sW + (int64_t)wrow * nb, nb);
-  if (is_x && warp == Cf::NWT / 32 && lane < MT) {
-    int rx = -128;
-    if (x0 + lane < M) rx = row_ref(sX + (int64_t)(x0 + lane) * nb, nb);
-    sh.refB[lane] = rx;
-  }
+  // the references of the tile's weight rows and tokens, formed by all
+  // threads from the two contiguous runs of scale rows (-128 past the ends)
+  if (tid < 128) sh.wref[tid] = -128;
+  if (tid < MT) sh.refB[tid] = -128;
+  __syncthreads();
+  rows_ref_coop(sW + (int64_t)w0 * nb, min(Cf::BM, N - w0), nb, sh.wref, tid, Cf::THREADS);
+  rows_ref_coop(sX + (int64_t)x0 * nb, min(MT, M - x0), nb, sh.refB, tid, Cf::THREADS);
   for (int o = tid * 16; o < Cf::NSX * (Cf::BSTAGE + Cf::SFSTAGE); o += Cf::THREADS * 16)
     *reinterpret_cast<uint4*>(smem + o) = make_uint4(0, 0, 0, 0);
   tc::fence_proxy_async_smem();
@@ -160,6 +161,7 @@ __global__ void __launch_bounds__(R34::THREADS, 1)
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = sh.tmem_base;
+  const int ref = is_w ? sh.wref[q4 * 32 + lane] : -128;  // this W thread's weight row
 
   if (is_w) {
     // ---------------------------- weight producers ---------------------------
