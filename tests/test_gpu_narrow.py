@@ -67,10 +67,10 @@ def test_random_codes_within_tolerance(torch, fa, fb, M):
 @pytest.mark.parametrize("fa,fb", [("E3C3", "E3C3"), ("E4C3", "E4C3"), ("E5C2", "E5C2"), ("E5C2", "E4C3")])
 @pytest.mark.parametrize("M", [512, 601])
 def test_two_token_groups_per_cta(torch, fa, fb, M):
-    """From 512 rows the same-format pairs take two token groups per CTA
-    (accumulators side by side): M = 601 leaves a last CTA whose second group
-    is partly padding; N = 260 a ragged weight tile; the mixed pair keeps one
-    group and checks the same sizes."""
+    """Many token groups of 32 (16 for M = 512; 19 for M = 601, the last
+    with 25 real tokens and 7 padding columns), N = 260 a ragged weight
+    tile, K = 256 (8 scale bytes per row: the 8-byte chunks of the
+    cooperative row references)."""
     rng = np.random.default_rng(M)
     a, sa = rand_operand(rng, fa, M, 256, 32)
     b, sb = rand_operand(rng, fb, 260, 256, 32)
