@@ -30,26 +30,6 @@ __device__ __forceinline__ void raise_flag(uint32_t* status, uint32_t bit) {
 }
 __device__ __forceinline__ int read_abort(const int* f) { return *reinterpret_cast<const volatile int*>(f); }
 
-// Largest block scale of a row (the row reference of the scale factors).
-__device__ __forceinline__ int row_ref(const int8_t* s, int nb) {
-  // bytes up to the first 16-byte boundary, 16-byte loads, then the tail
-  const int head = min(nb, (int)((16 - (reinterpret_cast<uintptr_t>(s) & 15)) & 15));
-  int ref = -128;
-  for (int b = 0; b < head; ++b) ref = max(ref, (int)__ldg(s + b));
-  const int nv = (nb - head) >> 4;
-  const uint4* p = reinterpret_cast<const uint4*>(s + head);
-  uint32_t m4 = 0x80808080u;
-#pragma unroll 8
-  for (int v = 0; v < nv; ++v) {
-    const uint4 q = __ldg(p + v);
-    m4 = __vmaxs4(m4, __vmaxs4(__vmaxs4(q.x, q.y), __vmaxs4(q.z, q.w)));
-  }
-  ref = max(ref, max(max((int)(int8_t)(m4 & 0xFF), (int)(int8_t)((m4 >> 8) & 0xFF)),
-                     max((int)(int8_t)((m4 >> 16) & 0xFF), (int)(int8_t)(m4 >> 24))));
-  for (int b = head + 16 * nv; b < nb; ++b) ref = max(ref, (int)__ldg(s + b));
-  return ref;
-}
-
 // Largest of the four signed bytes of v.
 __device__ __forceinline__ int max_s8x4(uint32_t v) {
   return max(max((int)(int8_t)(v & 0xFF), (int)(int8_t)((v >> 8) & 0xFF)),
