@@ -54,10 +54,11 @@
 //               factor block (copied to TMEM by the MMA warp).
 //   last warp   TMEM allocation, factor copies and MMA issue (one elected
 //               lane).
-// With fewer weight tiles than fill the SMs' last wave, tiles are split in K
-// into two pieces (greedy-dispatch simulation); a piece adds its outputs to
-// zeroed C atomically, two additions per output, so the result does not
-// depend on their order.  Every wait is bounded.
+// Tiles of the last partial wave may be split in K into two pieces (the plan
+// in tcn_common.cuh); a piece adds its outputs to zeroed C atomically, two
+// additions per output, so the result does not depend on their order.  The
+// row references come from the tile's contiguous scale rows, read by all
+// threads together.  Every wait is bounded.
 #include "gemm_tc.cuh"
 #include "tc_mx.cuh"
 #include "tcn_common.cuh"
